@@ -1,0 +1,125 @@
+"""Seeded synthetic workloads for the MALT / MALTER update.
+
+This module only draws inputs; it holds none of the update's arithmetic.  Both
+the CUDA path (tests, benchmark) and the fp64 oracle receive exactly the
+arrays produced here.
+
+Shapes are the 2-D parameter sets of the GPT-2 models the paper trains
+(Section 5.1: GPT-2 Small / Medium / Large with NanoGPT), taken literally as
+rows x cols, plus a single small matrix and a square/rectangular stress set.
+Gradients stand in for the paper's OpenWebText gradients (Section 5.1),
+which are not available here: G_ij = z_ij * a_i * b_j with z ~ N(0, 1) drawn
+fresh every step and row/column scales a_i, b_j = exp(sigma * N(0, 1)) drawn
+once per matrix, the row/column anisotropy that Section 5.4 reports for the
+trained model.  Initial weights follow the GPT-2 init N(0, 0.02^2).
+
+Every draw comes from numpy's PCG64 seeded with the tuple
+(workload id, matrix index, step + 1, stream tag), so any matrix of any step
+can be regenerated on its own.
+"""
+from __future__ import annotations
+
+import dataclasses
+from concurrent.futures import ThreadPoolExecutor
+
+import numpy as np
+
+_TAG_SCALES, _TAG_GRAD, _TAG_WEIGHT = 1, 2, 3
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    name: str
+    wid: int                     # seed component
+    shapes: tuple                # ((rows, cols), ...) in matrix order
+    weight_dtype: str            # "f32" | "bf16"
+    sigma: float                 # log-normal row/col scale spread
+    lr: float
+    variant: str                 # "malt" | "malter"
+    steps: int
+    ns_steps: int = 5
+
+    @property
+    def elements(self) -> int:
+        return int(sum(m * n for m, n in self.shapes))
+
+    def ns_flops_dense(self) -> float:
+        """Dense Newton-Schulz flops of one step: per matrix and iteration
+        4 p^2 q + 2 p^3 with p = min(m, n), q = max(m, n)."""
+        tot = 0.0
+        for m, n in self.shapes:
+            p, q = min(m, n), max(m, n)
+            tot += 4.0 * p * p * q + 2.0 * p ** 3
+        return tot * self.ns_steps
+
+
+def _gpt2(layers, d):
+    # attn.c_attn d x 3d, attn.c_proj d x d, mlp.c_fc d x 4d, mlp.c_proj 4d x d
+    per_layer = ((d, 3 * d), (d, d), (d, 4 * d), (4 * d, d))
+    return tuple(s for _ in range(layers) for s in per_layer)
+
+
+WORKLOADS = {
+    "single_256x512": Workload("single_256x512", 1, ((256, 512),), "f32", 1.0, 0.02, "malt", 3),
+    "gpt2_small": Workload("gpt2_small", 2, _gpt2(12, 768), "bf16", 1.5, 0.0013, "malt", 10),
+    "gpt2_medium": Workload("gpt2_medium", 3, _gpt2(24, 1024), "bf16", 1.5, 0.009, "malter", 10),
+    "gpt2_large": Workload("gpt2_large", 4, _gpt2(36, 1280), "bf16", 1.5, 0.0007, "malt", 10),
+}
+
+
+def stress_workload(rows: int, cols: int, sigma: float, ns_steps: int) -> Workload:
+    """One large matrix in bf16 with fp32 state, 3 MALT steps (stress sweep)."""
+    wid = 5_000 + int(sigma * 10) * 10 + ns_steps
+    return Workload(f"stress_{rows}x{cols}_s{sigma:g}_k{ns_steps}", wid, ((rows, cols),),
+                    "bf16", sigma, 0.02, "malt", 3, ns_steps)
+
+
+def _rng(wid: int, idx: int, step: int, tag: int) -> np.random.Generator:
+    return np.random.Generator(np.random.PCG64([wid, idx, step + 1, tag]))
+
+
+def row_col_scales(wl: Workload, idx: int):
+    """(a, b): per-row and per-column log-normal scales of matrix idx, fp32."""
+    m, n = wl.shapes[idx]
+    rng = _rng(wl.wid, idx, -1, _TAG_SCALES)
+    a = np.exp(wl.sigma * rng.standard_normal(m)).astype(np.float32)
+    b = np.exp(wl.sigma * rng.standard_normal(n)).astype(np.float32)
+    return a, b
+
+
+def gradient(wl: Workload, idx: int, step: int, scales=None) -> np.ndarray:
+    """fp32 gradient of matrix idx at step (0-based): z * a_i * b_j."""
+    m, n = wl.shapes[idx]
+    a, b = scales if scales is not None else row_col_scales(wl, idx)
+    z = _rng(wl.wid, idx, step, _TAG_GRAD).standard_normal((m, n), dtype=np.float32)
+    z *= a[:, None]
+    z *= b[None, :]
+    return z
+
+
+def bf16_representable(x: np.ndarray) -> np.ndarray:
+    """Input preparation only: the bf16 value nearest each fp32 entry
+    (ties to even), returned as fp32 so the same bits can go anywhere."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    u = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    return (u.astype(np.uint32) << 16).view(np.float32)
+
+
+def initial_weight(wl: Workload, idx: int) -> np.ndarray:
+    """W_0 of matrix idx ~ N(0, 0.02^2); bf16-representable for bf16 weights."""
+    m, n = wl.shapes[idx]
+    w = (0.02 * _rng(wl.wid, idx, 0, _TAG_WEIGHT).standard_normal((m, n))).astype(np.float32)
+    return bf16_representable(w) if wl.weight_dtype == "bf16" else w
+
+
+def gradients_for_step(wl: Workload, step: int, indices=None, workers: int = 8):
+    """Gradients of all (or the listed) matrices at one step, drawn in parallel."""
+    idxs = list(range(len(wl.shapes))) if indices is None else list(indices)
+    with ThreadPoolExecutor(max_workers=workers) as ex:
+        return list(ex.map(lambda i: gradient(wl, i, step), idxs))
+
+
+def initial_weights(wl: Workload, indices=None, workers: int = 8):
+    idxs = list(range(len(wl.shapes))) if indices is None else list(indices)
+    with ThreadPoolExecutor(max_workers=workers) as ex:
+        return list(ex.map(lambda i: initial_weight(wl, i), idxs))
