@@ -1,0 +1,168 @@
+/*
+ * malt.h -- C ABI of the GB300 MALT / MALTER optimizer step.
+ *
+ * One call updates every 2-D weight matrix of a model by the MALT update
+ * (Algorithm 1 of "MALT: Lightweight Curvature-Aware Muon via Diagonal
+ * Preconditioning") or the MALTER update (Algorithm 2).  Per matrix W (m x n)
+ * with gradient G, momentum M, row statistics l (m) and column statistics
+ * r (n), one step computes
+ *
+ *   M <- mu1 M + (1 - mu1) G                          (Alg. 1, M_t line)
+ *   l <- mu2 l + (1 - mu2) [||G[i,:]||^2]_i           (Alg. 1, l_t line; eq. dp_preconditioner)
+ *   r <- mu2 r + (1 - mu2) [||G[:,j]||^2]_j           (Alg. 1, r_t line)
+ *   L = Diag((l + eps)^(-1/8)),  R = Diag((r + eps)^(-1/8))
+ *   Mt = L M R,  O = NS_k(Mt),  D = L O R             (Alg. 1; Section 3.2 eq. final-update)
+ *   W <- W - lr * s * ||O||_F / (||D||_F + eps) * D   (Alg. 1 W_t line: s = 1)
+ *
+ * and for MALTER additionally (Algorithm 2 and the alpha_t equation of
+ * Section 3.5)
+ *
+ *   nu    <- mu2 nu + (1 - mu2) ||L G R||_F^2
+ *   alpha  = sqrt(1 - mu2^t) / (1 - mu1^t + eps) * ||Mt||_F / (sqrt(nu) + eps),  s = alpha
+ *
+ * with t the 1-based step count.  NS_k is the quintic Newton-Schulz iteration
+ * (the paper names it, Section 3.1, without its constants): on the wide
+ * orientation of Mt (transposed when m > n), X = Mt / (||Mt||_F + ns_eps),
+ * then k times A = X X^T, B = b A + c A A, X = a X + B X.
+ *
+ * Every call is asynchronous on the given CUDA stream (a cudaStream_t passed
+ * as void*; NULL is the legacy default stream) and returns a status code
+ * immediately; only malt_check, malt_get_scalars, malt_set_scalars and
+ * malt_debug_scalars wait for the stream.  No call allocates memory except
+ * malt_init_state.  All device pointers stay owned by the caller.
+ */
+#ifndef MALT_H
+#define MALT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ------------------------------------------------------ */
+#define MALT_OK                   0
+#define MALT_ERR_INVALID_ARG     -1  /* null pointer, n < 0, bad hyperparameter */
+#define MALT_ERR_UNSUPPORTED     -2  /* rows or cols not a positive multiple of 8, bad dtype */
+#define MALT_ERR_MISALIGNED      -3  /* a device pointer is not 16-byte aligned */
+#define MALT_ERR_SHAPE_CHANGED   -4  /* step called with shapes/dtypes other than at init */
+#define MALT_ERR_CUDA            -5  /* a CUDA runtime call failed (see malt_status_string) */
+#define MALT_ERR_TIMEOUT         -6  /* a device-side wait ran out of its time budget */
+#define MALT_ERR_OUT_OF_MEMORY   -7  /* workspace allocation failed at init */
+
+/* ---- element types ----------------------------------------------------- */
+#define MALT_F32   0
+#define MALT_BF16  1
+
+/* One 2-D parameter.  All pointers are DEVICE pointers owned by the caller,
+ * 16-byte aligned, row-major and densely packed (leading dimension = cols).
+ *   w       W, rows x cols, MALT_F32 or MALT_BF16, updated in place (bf16
+ *           results are rounded to nearest even)
+ *   g       G, rows x cols, MALT_F32 or MALT_BF16, read only
+ *   m       momentum M, rows x cols fp32, updated in place
+ *   l, r    row statistics (rows fp32) and column statistics (cols fp32),
+ *           updated in place
+ * rows and cols must be positive multiples of 8.  W, G and M must not
+ * overlap each other or another parameter's buffers. */
+typedef struct {
+    void*        w;
+    int32_t      w_dtype;
+    const void*  g;
+    int32_t      g_dtype;
+    float*       m;
+    float*       l;
+    float*       r;
+    int64_t      rows;
+    int64_t      cols;
+} malt_param_t;
+
+/* Hyperparameters (the Require line of Algorithms 1 and 2, plus the
+ * Newton-Schulz settings).  Suggested defaults: mu1 0.95, mu2 0.99,
+ * eps 1e-8 (the paper's appendix table), weight_decay 0, ns_steps 5,
+ * (ns_a, ns_b, ns_c) = (3.4445, -4.7750, 2.0315), ns_eps 1e-7.
+ * weight_decay, when non-zero, applies W <- (1 - lr*weight_decay) W before
+ * the update (decoupled; the paper's table lists 0.1 but its algorithms
+ * leave it out).  Constraints: 0 <= mu1, mu2 < 1; eps >= 0; 1 <= ns_steps <= 64. */
+typedef struct {
+    float   lr;
+    float   mu1;
+    float   mu2;
+    float   eps;
+    float   weight_decay;
+    int32_t ns_steps;
+    float   ns_a;
+    float   ns_b;
+    float   ns_c;
+    float   ns_eps;
+} malt_hparams_t;
+
+/* Opaque per-model state: the library-owned workspace (Newton-Schulz operand
+ * buffers grouped by shape, statistics partials, L and R, the per-matrix
+ * MALTER scalar nu, the step counter t, the device status word). */
+typedef struct malt_state malt_state_t;
+
+/* Plan the step for these n parameters (their shapes and dtypes are fixed
+ * from here on), allocate the workspace on the current CUDA device, and
+ * zero M, l, r of every parameter on `stream` (Algorithm 1 INITIALIZE line;
+ * nu_0 = 0 and t = 0 as in Algorithm 2).  W is left untouched.
+ * n = 0 is allowed (every later step is a no-op).
+ * On success *out receives a state the caller frees with malt_destroy_state;
+ * on failure *out is NULL and nothing stays allocated. */
+int malt_init_state(malt_state_t** out, const malt_param_t* params, int32_t n, void* stream);
+
+/* One MALT step (Algorithm 1) of all n parameters, enqueued on `stream`.
+ * params must describe the same shapes and dtypes, in the same order, as at
+ * init (MALT_ERR_SHAPE_CHANGED otherwise); the pointers may differ. */
+int malt_step(malt_state_t* st, const malt_param_t* params, int32_t n,
+              const malt_hparams_t* hp, void* stream);
+
+/* One MALTER step (Algorithm 2): as malt_step plus the nu / alpha scalars.
+ * MALT and MALTER steps may be mixed on one state; nu only advances on
+ * MALTER steps while t advances on both. */
+int malter_step(malt_state_t* st, const malt_param_t* params, int32_t n,
+                const malt_hparams_t* hp, void* stream);
+
+/* Checkpoint support: copy the n per-matrix nu values and the step counter t
+ * to host memory (get) or from host memory (set).  Both synchronise with the
+ * stream of the state's last call.  M, l, r and W are caller-owned and are
+ * saved by the caller. */
+int malt_get_scalars(malt_state_t* st, float* nu_host, int32_t n, int64_t* t_host);
+int malt_set_scalars(malt_state_t* st, const float* nu_host, int32_t n, int64_t t_host);
+
+/* Wait for the stream of the state's last call, then return (and clear) the
+ * device-side status word: MALT_OK, or MALT_ERR_TIMEOUT when a kernel gave up
+ * on a bounded wait, or MALT_ERR_CUDA when the stream reported an error. */
+int malt_check(malt_state_t* st);
+
+/* Test hooks.
+ * malt_debug_direction: enqueue on `stream` a copy of the last step's
+ *   orthogonalised direction O of parameter idx (rows x cols, bf16,
+ *   row-major, same orientation as W) into the device buffer out.
+ * malt_debug_scalars: synchronise, then write 8 floats per parameter to host
+ *   memory: ||O||_F, ||D||_F, ||Mt||_F, ||L G R||_F^2 (MALTER steps, else 0),
+ *   nu, alpha (1 on MALT steps), the applied scale lr*alpha*||O||/(||D||+eps),
+ *   and 1/(||Mt||_F + ns_eps). */
+int malt_debug_direction(malt_state_t* st, int32_t idx, void* out, void* stream);
+int malt_debug_scalars(malt_state_t* st, float* out_host, int32_t n);
+
+/* Exercise the bounded device-side wait used by the kernels: launch one
+ * block that waits on a flag nothing ever sets, for at most budget_ns
+ * nanoseconds, then synchronise.  Returns MALT_ERR_TIMEOUT when the wait gave
+ * up as designed (the expected result), MALT_OK if it somehow completed. */
+int malt_debug_wait_timeout(int64_t budget_ns, void* stream);
+
+/* Bytes of device workspace the state holds. */
+size_t malt_workspace_bytes(const malt_state_t* st);
+
+/* Static text for a status code. */
+const char* malt_status_string(int code);
+
+/* Free the workspace (synchronises with the state's last stream first). */
+void malt_destroy_state(malt_state_t* st);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MALT_H */

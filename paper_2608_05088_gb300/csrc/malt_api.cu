@@ -1,0 +1,611 @@
+// malt_api.cu -- host runtime behind include/malt.h.
+//
+// At init the parameters are planned once: each matrix gets its Newton-Schulz
+// frame (transposed when m > n), matrices with the same frame shape p x q form
+// a shape class whose NS buffers are stored batched ([batch][p][q] etc.) so one
+// 3-D TMA descriptor serves the whole class, and every grouped element-wise
+// launch gets a block-prefix table.  A step then enqueues, on the caller's
+// stream and without any host synchronisation:
+//   bind (caller pointers) -> stats -> finalize -> prescale -> norms
+//   -> k x (Gram, Poly, BX) over all classes -> scalars -> apply.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <utility>
+#include <vector>
+
+#include "../../include/malt.h"
+#include "common.cuh"
+#include "kernels.h"
+
+using namespace malt;
+
+namespace {
+
+constexpr uint64_t kWaitBudgetNs = 1000000000ull;  // 1 s per device-side wait
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+bool get_encoder() {
+    if (g_encode != nullptr) return true;
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || fn == nullptr)
+        return false;
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    return true;
+}
+
+// 3-D bf16 tensor [batch][rows][cols], box kBK x box_rows x 1, 128-byte swizzle,
+// zero fill outside the tensor.
+bool encode_3d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint64_t batch,
+               uint32_t box_rows) {
+    const cuuint64_t dims[3] = {cols, rows, batch};
+    const cuuint64_t strides[2] = {cols * 2, rows * cols * 2};
+    const cuuint32_t box[3] = {static_cast<cuuint32_t>(kBK), box_rows, 1};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    const CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base),
+                                dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+struct ShapeClass {
+    int p = 0, q = 0, batch = 0;
+    std::vector<int> mats;
+    int32_t* d_mat_of = nullptr;
+    __nv_bfloat16* X[2] = {nullptr, nullptr};
+    __nv_bfloat16* Xt[2] = {nullptr, nullptr};
+    __nv_bfloat16* A = nullptr;
+    __nv_bfloat16* B = nullptr;
+    CUtensorMap tmXa[2], tmXb[2], tmXtb[2], tmAa, tmAb, tmBa;
+};
+
+struct Carver {
+    size_t off = 0;
+    size_t take(size_t bytes) {
+        const size_t o = off;
+        off += (bytes + 255) & ~static_cast<size_t>(255);
+        return o;
+    }
+};
+
+int cuda_fail(cudaError_t e, const char* what) {
+    if (e == cudaSuccess) return MALT_OK;
+    std::fprintf(stderr, "malt: %s failed: %s\n", what, cudaGetErrorString(e));
+    return MALT_ERR_CUDA;
+}
+
+#define MALT_CUDA(call, what)                              \
+    do {                                                   \
+        const int rc_ = cuda_fail((call), (what));         \
+        if (rc_ != MALT_OK) return rc_;                    \
+    } while (0)
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+struct malt_state {
+    int device = 0;
+    int nmat = 0;
+    int num_sms = 0;
+    std::vector<malt_param_t> shape0;      // shapes / dtypes fixed at init
+    std::vector<MatDesc> hmats;
+    std::vector<ShapeClass> classes;
+    void* ws = nullptr;
+    size_t ws_bytes = 0;
+    MatDesc* d_mats = nullptr;
+    UserPtrs* d_ptrs = nullptr;
+    MatScalars* d_scal = nullptr;
+    long long* d_t = nullptr;
+    int32_t* d_status = nullptr;
+    int32_t* d_pref[4] = {nullptr, nullptr, nullptr, nullptr};  // stats, fin, pre, apply
+    int32_t blocks_stats = 0, total_fin = 0, blocks_pre = 0, blocks_apply = 0;
+    cudaStream_t last_stream = nullptr;
+};
+
+namespace {
+
+int validate_param(const malt_param_t& p) {
+    if (p.w == nullptr || p.g == nullptr || p.m == nullptr || p.l == nullptr || p.r == nullptr)
+        return MALT_ERR_INVALID_ARG;
+    if (p.rows <= 0 || p.cols <= 0 || (p.rows % 8) != 0 || (p.cols % 8) != 0)
+        return MALT_ERR_UNSUPPORTED;
+    if (p.rows * p.cols >= (static_cast<int64_t>(1) << 31)) return MALT_ERR_UNSUPPORTED;
+    if ((p.w_dtype != MALT_F32 && p.w_dtype != MALT_BF16) ||
+        (p.g_dtype != MALT_F32 && p.g_dtype != MALT_BF16))
+        return MALT_ERR_UNSUPPORTED;
+    if (!aligned16(p.w) || !aligned16(p.g) || !aligned16(p.m) || !aligned16(p.l) ||
+        !aligned16(p.r))
+        return MALT_ERR_MISALIGNED;
+    return MALT_OK;
+}
+
+int validate_hparams(const malt_hparams_t* hp) {
+    if (hp == nullptr) return MALT_ERR_INVALID_ARG;
+    if (!(hp->mu1 >= 0.f && hp->mu1 < 1.f) || !(hp->mu2 >= 0.f && hp->mu2 < 1.f))
+        return MALT_ERR_INVALID_ARG;
+    if (!(hp->eps >= 0.f) || !(hp->ns_eps >= 0.f) || hp->ns_steps < 1 || hp->ns_steps > 64)
+        return MALT_ERR_INVALID_ARG;
+    if (!(hp->lr == hp->lr) || !(hp->weight_decay == hp->weight_decay)) return MALT_ERR_INVALID_ARG;
+    return MALT_OK;
+}
+
+void free_state(malt_state* st) {
+    if (st == nullptr) return;
+    if (st->ws != nullptr) cudaFree(st->ws);
+    delete st;
+}
+
+int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
+    st->nmat = n;
+    st->shape0.assign(params, params + n);
+    st->hmats.resize(n);
+    // Shape classes by NS frame.
+    std::map<std::pair<int, int>, int> cls_of;
+    for (int i = 0; i < n; ++i) {
+        const int m = static_cast<int>(params[i].rows), c = static_cast<int>(params[i].cols);
+        const int p = std::min(m, c), q = std::max(m, c);
+        auto it = cls_of.find({p, q});
+        int k;
+        if (it == cls_of.end()) {
+            k = static_cast<int>(st->classes.size());
+            cls_of[{p, q}] = k;
+            st->classes.emplace_back();
+            st->classes.back().p = p;
+            st->classes.back().q = q;
+        } else {
+            k = it->second;
+        }
+        MatDesc& d = st->hmats[i];
+        std::memset(&d, 0, sizeof(d));
+        d.m = m;
+        d.n = c;
+        d.trans = m > c ? 1 : 0;
+        d.p = p;
+        d.q = q;
+        d.w_bf16 = params[i].w_dtype == MALT_BF16;
+        d.g_bf16 = params[i].g_dtype == MALT_BF16;
+        d.cls = k;
+        d.bidx = st->classes[k].batch++;
+        st->classes[k].mats.push_back(i);
+        d.stat_rb = (m + kStatRows - 1) / kStatRows;
+        d.stat_cb = (c + kStatCols - 1) / kStatCols;
+        d.pre_tr = (m + kPreTile - 1) / kPreTile;
+        d.pre_tc = (c + kPreTile - 1) / kPreTile;
+        d.ns_tiles = ((p + kBM - 1) / kBM) * ((q + kBN - 1) / kBN);
+    }
+
+    // Workspace layout.
+    Carver cv;
+    std::vector<size_t> o_row(n), o_col(n), o_L(n), o_R(n), o_pre(n), o_ns(n), o_O(n);
+    for (int i = 0; i < n; ++i) {
+        const MatDesc& d = st->hmats[i];
+        o_row[i] = cv.take(sizeof(float) * static_cast<size_t>(d.stat_cb) * d.m);
+        o_col[i] = cv.take(sizeof(float) * static_cast<size_t>(d.stat_rb) * d.n);
+        o_L[i] = cv.take(sizeof(float) * d.m);
+        o_R[i] = cv.take(sizeof(float) * d.n);
+        o_pre[i] = cv.take(sizeof(float) * 2 * static_cast<size_t>(d.pre_tr) * d.pre_tc);
+        o_ns[i] = cv.take(sizeof(float) * 8 * static_cast<size_t>(d.ns_tiles));
+        o_O[i] = cv.take(2 * static_cast<size_t>(d.m) * d.n);
+    }
+    const int nc = static_cast<int>(st->classes.size());
+    std::vector<size_t> o_X0(nc), o_X1(nc), o_Xt0(nc), o_Xt1(nc), o_A(nc), o_B(nc), o_matof(nc);
+    for (int k = 0; k < nc; ++k) {
+        const ShapeClass& C = st->classes[k];
+        const size_t pq = static_cast<size_t>(C.batch) * C.p * C.q * 2;
+        const size_t pp = static_cast<size_t>(C.batch) * C.p * C.p * 2;
+        o_X0[k] = cv.take(pq);
+        o_X1[k] = cv.take(pq);
+        o_Xt0[k] = cv.take(pq);
+        o_Xt1[k] = cv.take(pq);
+        o_A[k] = cv.take(pp);
+        o_B[k] = cv.take(pp);
+        o_matof[k] = cv.take(sizeof(int32_t) * C.batch);
+    }
+    const size_t o_mats = cv.take(sizeof(MatDesc) * std::max(n, 1));
+    const size_t o_ptrs = cv.take(sizeof(UserPtrs) * std::max(n, 1));
+    const size_t o_scal = cv.take(sizeof(MatScalars) * std::max(n, 1));
+    const size_t o_t = cv.take(sizeof(long long));
+    const size_t o_status = cv.take(sizeof(int32_t));
+    size_t o_pref[4];
+    for (int j = 0; j < 4; ++j) o_pref[j] = cv.take(sizeof(int32_t) * (n + 1));
+
+    st->ws_bytes = cv.off;
+    if (cudaMalloc(&st->ws, st->ws_bytes) != cudaSuccess) {
+        st->ws = nullptr;
+        cudaGetLastError();
+        return MALT_ERR_OUT_OF_MEMORY;
+    }
+    uint8_t* base = static_cast<uint8_t*>(st->ws);
+    auto F = [&](size_t o) { return reinterpret_cast<float*>(base + o); };
+    auto H = [&](size_t o) { return reinterpret_cast<__nv_bfloat16*>(base + o); };
+    for (int k = 0; k < nc; ++k) {
+        ShapeClass& C = st->classes[k];
+        C.X[0] = H(o_X0[k]);
+        C.X[1] = H(o_X1[k]);
+        C.Xt[0] = H(o_Xt0[k]);
+        C.Xt[1] = H(o_Xt1[k]);
+        C.A = H(o_A[k]);
+        C.B = H(o_B[k]);
+        C.d_mat_of = reinterpret_cast<int32_t*>(base + o_matof[k]);
+    }
+    for (int i = 0; i < n; ++i) {
+        MatDesc& d = st->hmats[i];
+        const ShapeClass& C = st->classes[d.cls];
+        d.rowpart = F(o_row[i]);
+        d.colpart = F(o_col[i]);
+        d.L = F(o_L[i]);
+        d.R = F(o_R[i]);
+        d.prepart = F(o_pre[i]);
+        d.nspart = F(o_ns[i]);
+        d.O = H(o_O[i]);
+        const size_t slot = static_cast<size_t>(d.bidx) * C.p * C.q;
+        d.Xdir = d.trans ? C.Xt[0] + slot : C.X[0] + slot;
+        d.Xtrn = d.trans ? C.X[0] + slot : C.Xt[0] + slot;
+    }
+    st->d_mats = reinterpret_cast<MatDesc*>(base + o_mats);
+    st->d_ptrs = reinterpret_cast<UserPtrs*>(base + o_ptrs);
+    st->d_scal = reinterpret_cast<MatScalars*>(base + o_scal);
+    st->d_t = reinterpret_cast<long long*>(base + o_t);
+    st->d_status = reinterpret_cast<int32_t*>(base + o_status);
+    for (int j = 0; j < 4; ++j) st->d_pref[j] = reinterpret_cast<int32_t*>(base + o_pref[j]);
+
+    // Block-prefix tables.
+    std::vector<int32_t> pref[4];
+    for (int j = 0; j < 4; ++j) pref[j].assign(n + 1, 0);
+    for (int i = 0; i < n; ++i) {
+        const MatDesc& d = st->hmats[i];
+        const int64_t elems = static_cast<int64_t>(d.m) * d.n;
+        pref[0][i + 1] = pref[0][i] + d.stat_rb * d.stat_cb;
+        pref[1][i + 1] = pref[1][i] + d.m + d.n;
+        pref[2][i + 1] = pref[2][i] + d.pre_tr * d.pre_tc;
+        pref[3][i + 1] = pref[3][i] + static_cast<int32_t>((elems + kApplyElems - 1) / kApplyElems);
+    }
+    st->blocks_stats = pref[0][n];
+    st->total_fin = pref[1][n];
+    st->blocks_pre = pref[2][n];
+    st->blocks_apply = pref[3][n];
+
+    // Tensor maps of every class buffer.
+    if (nc > 0 && !get_encoder()) return MALT_ERR_CUDA;
+    for (int k = 0; k < nc; ++k) {
+        ShapeClass& C = st->classes[k];
+        bool ok = true;
+        for (int b = 0; b < 2; ++b) {
+            ok &= encode_3d(&C.tmXa[b], C.X[b], C.q, C.p, C.batch, kBM);
+            ok &= encode_3d(&C.tmXb[b], C.X[b], C.q, C.p, C.batch, kBN);
+            ok &= encode_3d(&C.tmXtb[b], C.Xt[b], C.p, C.q, C.batch, kBN);
+        }
+        ok &= encode_3d(&C.tmAa, C.A, C.p, C.p, C.batch, kBM);
+        ok &= encode_3d(&C.tmAb, C.A, C.p, C.p, C.batch, kBN);
+        ok &= encode_3d(&C.tmBa, C.B, C.p, C.p, C.batch, kBM);
+        if (!ok) {
+            std::fprintf(stderr, "malt: cuTensorMapEncodeTiled failed for class %d x %d\n", C.p, C.q);
+            return MALT_ERR_CUDA;
+        }
+    }
+
+    // Upload the static tables (init is allowed to synchronise).
+    MALT_CUDA(cudaMemset(st->ws, 0, st->ws_bytes), "cudaMemset(workspace)");
+    if (n > 0) {
+        MALT_CUDA(cudaMemcpy(st->d_mats, st->hmats.data(), sizeof(MatDesc) * n,
+                             cudaMemcpyHostToDevice), "cudaMemcpy(mats)");
+        for (int j = 0; j < 4; ++j)
+            MALT_CUDA(cudaMemcpy(st->d_pref[j], pref[j].data(), sizeof(int32_t) * (n + 1),
+                                 cudaMemcpyHostToDevice), "cudaMemcpy(prefix)");
+        for (int k = 0; k < nc; ++k) {
+            const ShapeClass& C = st->classes[k];
+            MALT_CUDA(cudaMemcpy(C.d_mat_of, C.mats.data(), sizeof(int32_t) * C.batch,
+                                 cudaMemcpyHostToDevice), "cudaMemcpy(mat_of)");
+        }
+    }
+    return MALT_OK;
+}
+
+int bind_pointers(malt_state* st, const malt_param_t* params, cudaStream_t s) {
+    BindParams bp;
+    for (int off = 0; off < st->nmat; off += kBindChunk) {
+        const int cnt = std::min(kBindChunk, st->nmat - off);
+        std::memset(&bp, 0, sizeof(bp));
+        bp.count = cnt;
+        bp.offset = off;
+        for (int i = 0; i < cnt; ++i) {
+            const malt_param_t& p = params[off + i];
+            bp.p[i] = UserPtrs{p.w, p.g, p.m, p.l, p.r};
+        }
+        MALT_CUDA(launch_bind(bp, st->d_ptrs, s), "bind_kernel");
+    }
+    return MALT_OK;
+}
+
+// One GEMM phase of NS iteration `it` over every class, in launches of at
+// most kMaxClasses classes, heaviest K first.
+int run_gemm_phase(malt_state* st, int phase, int it, int last, const malt_hparams_t* hp,
+                   cudaStream_t s) {
+    const int cur = it & 1, nxt = cur ^ 1;
+    std::vector<int> order(st->classes.size());
+    for (size_t k = 0; k < order.size(); ++k) order[k] = static_cast<int>(k);
+    std::stable_sort(order.begin(), order.end(), [&](int x, int y) {
+        const ShapeClass& a = st->classes[x];
+        const ShapeClass& b = st->classes[y];
+        const int ka = phase == kGram ? a.q : a.p;
+        const int kb = phase == kGram ? b.q : b.p;
+        return ka > kb;
+    });
+    static GemmParams P;  // large (kMaxClasses tensor-map pairs): keep off the stack
+    for (size_t start = 0; start < order.size(); start += kMaxClasses) {
+        std::memset(&P, 0, sizeof(P));
+        const size_t cnt = std::min(order.size() - start, static_cast<size_t>(kMaxClasses));
+        int tiles = 0;
+        for (size_t j = 0; j < cnt; ++j) {
+            const ShapeClass& C = st->classes[order[start + j]];
+            GemmClass& G = P.cls[j];
+            G.batch = C.batch;
+            G.mat_of = C.d_mat_of;
+            if (phase == kGram) {
+                G.tmA = C.tmXa[cur];
+                G.tmB = C.tmXb[cur];
+                G.M = C.p; G.N = C.p; G.K = C.q;
+                G.ein = nullptr;
+                G.out = C.A;
+                G.outT = nullptr;
+            } else if (phase == kPoly) {
+                G.tmA = C.tmAa;
+                G.tmB = C.tmAb;
+                G.M = C.p; G.N = C.p; G.K = C.p;
+                G.ein = C.A;
+                G.out = C.B;
+                G.outT = nullptr;
+            } else {
+                G.tmA = C.tmBa;
+                G.tmB = C.tmXtb[cur];
+                G.M = C.p; G.N = C.q; G.K = C.p;
+                G.ein = C.X[cur];
+                G.out = last ? nullptr : C.X[nxt];
+                G.outT = last ? nullptr : C.Xt[nxt];
+            }
+            G.tiles_m = (G.M + kBM - 1) / kBM;
+            G.tiles_n = (G.N + kBN - 1) / kBN;
+            G.tile_begin = tiles;
+            tiles += G.tiles_m * G.tiles_n * G.batch;
+        }
+        P.nclasses = static_cast<int32_t>(cnt);
+        P.total_tiles = tiles;
+        P.phase = phase;
+        P.first = it == 0;
+        P.last = last;
+        P.a = hp->ns_a;
+        P.b = hp->ns_b;
+        P.c = hp->ns_c;
+        P.mats = st->d_mats;
+        P.scal = st->d_scal;
+        P.status = st->d_status;
+        P.budget_ns = kWaitBudgetNs;
+        const int grid = std::max(1, std::min(tiles, st->num_sms));
+        MALT_CUDA(launch_ns_gemm(P, grid, s), "ns_gemm_kernel");
+    }
+    return MALT_OK;
+}
+
+int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_hparams_t* hp,
+             void* stream, int malter) {
+    if (st == nullptr || (n > 0 && params == nullptr)) return MALT_ERR_INVALID_ARG;
+    int rc = validate_hparams(hp);
+    if (rc != MALT_OK) return rc;
+    if (n != st->nmat) return MALT_ERR_SHAPE_CHANGED;
+    for (int i = 0; i < n; ++i) {
+        rc = validate_param(params[i]);
+        if (rc != MALT_OK) return rc;
+        const malt_param_t& a = st->shape0[i];
+        if (a.rows != params[i].rows || a.cols != params[i].cols ||
+            a.w_dtype != params[i].w_dtype || a.g_dtype != params[i].g_dtype)
+            return MALT_ERR_SHAPE_CHANGED;
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    st->last_stream = s;
+    if (n == 0) return MALT_OK;
+    MALT_CUDA(cudaSetDevice(st->device), "cudaSetDevice");
+    rc = bind_pointers(st, params, s);
+    if (rc != MALT_OK) return rc;
+    const int nm = st->nmat;
+    MALT_CUDA(launch_stats(st->d_mats, st->d_ptrs, st->d_pref[0], nm, st->blocks_stats, hp->mu1, s),
+              "stats_kernel");
+    MALT_CUDA(launch_finalize(st->d_mats, st->d_ptrs, st->d_pref[1], nm, st->total_fin, hp->mu2,
+                              hp->eps, st->d_t, s), "finalize_kernel");
+    MALT_CUDA(launch_prescale(st->d_mats, st->d_ptrs, st->d_pref[2], nm, st->blocks_pre, malter, s),
+              "prescale_kernel");
+    MALT_CUDA(launch_norms(st->d_mats, st->d_scal, nm, hp->ns_eps, malter, s), "norms_kernel");
+    for (int it = 0; it < hp->ns_steps; ++it) {
+        const int last = it == hp->ns_steps - 1;
+        for (int phase = kGram; phase <= kBX; ++phase) {
+            rc = run_gemm_phase(st, phase, it, last, hp, s);
+            if (rc != MALT_OK) return rc;
+        }
+    }
+    StepHyper sh;
+    sh.lr = hp->lr;
+    sh.mu1 = hp->mu1;
+    sh.mu2 = hp->mu2;
+    sh.eps = hp->eps;
+    sh.weight_decay = hp->weight_decay;
+    sh.ns_a = hp->ns_a;
+    sh.ns_b = hp->ns_b;
+    sh.ns_c = hp->ns_c;
+    sh.ns_eps = hp->ns_eps;
+    sh.malter = malter;
+    MALT_CUDA(launch_scalars(st->d_mats, st->d_scal, st->d_t, nm, sh, s), "scalars_kernel");
+    MALT_CUDA(launch_apply(st->d_mats, st->d_ptrs, st->d_scal, st->d_pref[3], nm, st->blocks_apply,
+                           1.f - hp->lr * hp->weight_decay, s), "apply_kernel");
+    return MALT_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int malt_init_state(malt_state_t** out, const malt_param_t* params, int32_t n, void* stream) {
+    if (out == nullptr) return MALT_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (n < 0 || (n > 0 && params == nullptr)) return MALT_ERR_INVALID_ARG;
+    for (int i = 0; i < n; ++i) {
+        const int rc = validate_param(params[i]);
+        if (rc != MALT_OK) return rc;
+    }
+    malt_state* st = new malt_state();
+    int rc = cuda_fail(cudaGetDevice(&st->device), "cudaGetDevice");
+    if (rc == MALT_OK)
+        rc = cuda_fail(cudaDeviceGetAttribute(&st->num_sms, cudaDevAttrMultiProcessorCount, st->device),
+                       "cudaDeviceGetAttribute");
+    if (rc == MALT_OK) rc = plan_and_allocate(st, params, n);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    for (int i = 0; rc == MALT_OK && i < n; ++i) {
+        const malt_param_t& p = params[i];
+        const size_t e = static_cast<size_t>(p.rows) * p.cols;
+        rc = cuda_fail(cudaMemsetAsync(p.m, 0, e * sizeof(float), s), "cudaMemsetAsync(M)");
+        if (rc == MALT_OK) rc = cuda_fail(cudaMemsetAsync(p.l, 0, p.rows * sizeof(float), s), "memset(l)");
+        if (rc == MALT_OK) rc = cuda_fail(cudaMemsetAsync(p.r, 0, p.cols * sizeof(float), s), "memset(r)");
+    }
+    if (rc != MALT_OK) {
+        free_state(st);
+        return rc;
+    }
+    st->last_stream = s;
+    *out = st;
+    return MALT_OK;
+}
+
+int malt_step(malt_state_t* st, const malt_param_t* params, int32_t n, const malt_hparams_t* hp,
+              void* stream) {
+    return run_step(st, params, n, hp, stream, 0);
+}
+
+int malter_step(malt_state_t* st, const malt_param_t* params, int32_t n, const malt_hparams_t* hp,
+                void* stream) {
+    return run_step(st, params, n, hp, stream, 1);
+}
+
+int malt_check(malt_state_t* st) {
+    if (st == nullptr) return MALT_ERR_INVALID_ARG;
+    MALT_CUDA(cudaStreamSynchronize(st->last_stream), "cudaStreamSynchronize");
+    if (st->ws == nullptr) return MALT_OK;
+    int32_t status = 0;
+    MALT_CUDA(cudaMemcpy(&status, st->d_status, sizeof(status), cudaMemcpyDeviceToHost),
+              "cudaMemcpy(status)");
+    if (status != 0) {
+        MALT_CUDA(cudaMemset(st->d_status, 0, sizeof(int32_t)), "cudaMemset(status)");
+        return MALT_ERR_TIMEOUT;
+    }
+    return MALT_OK;
+}
+
+int malt_get_scalars(malt_state_t* st, float* nu_host, int32_t n, int64_t* t_host) {
+    if (st == nullptr || n != st->nmat || (n > 0 && nu_host == nullptr) || t_host == nullptr)
+        return MALT_ERR_INVALID_ARG;
+    MALT_CUDA(cudaStreamSynchronize(st->last_stream), "cudaStreamSynchronize");
+    long long t = 0;
+    MALT_CUDA(cudaMemcpy(&t, st->d_t, sizeof(t), cudaMemcpyDeviceToHost), "cudaMemcpy(t)");
+    *t_host = t;
+    if (n > 0) {
+        std::vector<MatScalars> s(n);
+        MALT_CUDA(cudaMemcpy(s.data(), st->d_scal, sizeof(MatScalars) * n, cudaMemcpyDeviceToHost),
+                  "cudaMemcpy(scalars)");
+        for (int i = 0; i < n; ++i) nu_host[i] = s[i].nu;
+    }
+    return MALT_OK;
+}
+
+int malt_set_scalars(malt_state_t* st, const float* nu_host, int32_t n, int64_t t_host) {
+    if (st == nullptr || n != st->nmat || (n > 0 && nu_host == nullptr) || t_host < 0)
+        return MALT_ERR_INVALID_ARG;
+    MALT_CUDA(cudaStreamSynchronize(st->last_stream), "cudaStreamSynchronize");
+    const long long t = t_host;
+    MALT_CUDA(cudaMemcpy(st->d_t, &t, sizeof(t), cudaMemcpyHostToDevice), "cudaMemcpy(t)");
+    if (n > 0) {
+        std::vector<MatScalars> s(n);
+        MALT_CUDA(cudaMemcpy(s.data(), st->d_scal, sizeof(MatScalars) * n, cudaMemcpyDeviceToHost),
+                  "cudaMemcpy(scalars)");
+        for (int i = 0; i < n; ++i) s[i].nu = nu_host[i];
+        MALT_CUDA(cudaMemcpy(st->d_scal, s.data(), sizeof(MatScalars) * n, cudaMemcpyHostToDevice),
+                  "cudaMemcpy(scalars)");
+    }
+    return MALT_OK;
+}
+
+int malt_debug_direction(malt_state_t* st, int32_t idx, void* out, void* stream) {
+    if (st == nullptr || idx < 0 || idx >= st->nmat || out == nullptr) return MALT_ERR_INVALID_ARG;
+    const MatDesc& d = st->hmats[idx];
+    MALT_CUDA(cudaMemcpyAsync(out, d.O, static_cast<size_t>(d.m) * d.n * 2, cudaMemcpyDeviceToDevice,
+                              static_cast<cudaStream_t>(stream)),
+              "cudaMemcpyAsync(O)");
+    return MALT_OK;
+}
+
+int malt_debug_scalars(malt_state_t* st, float* out_host, int32_t n) {
+    if (st == nullptr || n != st->nmat || (n > 0 && out_host == nullptr)) return MALT_ERR_INVALID_ARG;
+    MALT_CUDA(cudaStreamSynchronize(st->last_stream), "cudaStreamSynchronize");
+    if (n == 0) return MALT_OK;
+    std::vector<MatScalars> s(n);
+    MALT_CUDA(cudaMemcpy(s.data(), st->d_scal, sizeof(MatScalars) * n, cudaMemcpyDeviceToHost),
+              "cudaMemcpy(scalars)");
+    for (int i = 0; i < n; ++i) {
+        float* o = out_host + static_cast<size_t>(i) * kScalarsPerMat;
+        o[0] = s[i].norm_o;
+        o[1] = s[i].norm_d;
+        o[2] = s[i].norm_mt;
+        o[3] = s[i].lgr_sq;
+        o[4] = s[i].nu;
+        o[5] = s[i].alpha;
+        o[6] = s[i].scale;
+        o[7] = s[i].k;
+    }
+    return MALT_OK;
+}
+
+int malt_debug_wait_timeout(int64_t budget_ns, void* stream) {
+    if (budget_ns <= 0) return MALT_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int32_t* d = nullptr;
+    MALT_CUDA(cudaMalloc(&d, sizeof(int32_t)), "cudaMalloc(probe)");
+    int rc = cuda_fail(cudaMemsetAsync(d, 0, sizeof(int32_t), s), "cudaMemsetAsync(probe)");
+    if (rc == MALT_OK) rc = cuda_fail(launch_wait_probe(d, static_cast<uint64_t>(budget_ns), s), "wait_probe");
+    if (rc == MALT_OK) rc = cuda_fail(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+    int32_t h = 0;
+    if (rc == MALT_OK) rc = cuda_fail(cudaMemcpy(&h, d, sizeof(h), cudaMemcpyDeviceToHost), "cudaMemcpy(probe)");
+    cudaFree(d);
+    if (rc != MALT_OK) return rc;
+    return h != 0 ? MALT_ERR_TIMEOUT : MALT_OK;
+}
+
+size_t malt_workspace_bytes(const malt_state_t* st) { return st == nullptr ? 0 : st->ws_bytes; }
+
+const char* malt_status_string(int code) {
+    switch (code) {
+        case MALT_OK: return "ok";
+        case MALT_ERR_INVALID_ARG: return "invalid argument";
+        case MALT_ERR_UNSUPPORTED: return "unsupported shape or dtype (rows and cols must be positive multiples of 8, rows*cols < 2^31)";
+        case MALT_ERR_MISALIGNED: return "device pointer not 16-byte aligned";
+        case MALT_ERR_SHAPE_CHANGED: return "parameter shapes or dtypes differ from init";
+        case MALT_ERR_CUDA: return "CUDA runtime error";
+        case MALT_ERR_TIMEOUT: return "device-side wait timed out";
+        case MALT_ERR_OUT_OF_MEMORY: return "workspace allocation failed";
+        default: return "unknown status";
+    }
+}
+
+void malt_destroy_state(malt_state_t* st) {
+    if (st == nullptr) return;
+    cudaStreamSynchronize(st->last_stream);
+    free_state(st);
+}
+
+}  // extern "C"

@@ -1,0 +1,351 @@
+// ns_gemm.cu -- the Newton-Schulz engine: batched same-shape bf16 GEMMs on the
+// sm_103a tensor cores (tcgen05.mma, fp32 accumulators in TMEM, operands
+// staged into shared memory by TMA with 128-byte swizzle).
+//
+// One Newton-Schulz iteration (the Orth step of Algorithm 1, run on the wide
+// orientation X of Mt, p x q) is three launches of this kernel:
+//   kGram  A  = X X^T           (M = N = p, K = q)   operands: rows of X, rows of X
+//   kPoly  B  = b A + c A A     (M = N = p, K = p)   operands: rows of A, rows of A (A = A^T)
+//   kBX    X' = a X + B X       (M = p, N = q, K = p) operands: rows of B, rows of X^T
+// Every operand is read K-major, so X is kept in both orientations: the kBX
+// epilogue writes X' and X'^T.  The 1/(||Mt||_F + ns_eps) normalisation is
+// folded into the first iteration's epilogues (A scaled by k^2, X' by k).  The
+// last iteration's epilogue writes O in W's orientation and per-warp partial
+// sums of O^2 and of D^2 with D = L O R (Algorithm 1, D_t line) for the graft.
+//
+// Each launch is persistent (one CTA per SM) over a tile list that spans all
+// shape classes and all matrices of each class.  Per CTA: warp 0 issues TMA
+// loads into a kStages-deep ring, warp 1 issues tcgen05.mma into one of two
+// TMEM accumulators, warps 2-5 drain the other accumulator (tcgen05.ld) and
+// run the epilogue, so the epilogue of tile i overlaps the MMAs of tile i+1.
+// Every wait is bounded; a timeout sets the status word and the CTA winds down.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "ptx.cuh"
+
+namespace malt {
+
+namespace {
+
+constexpr int kThreads = 192;
+constexpr uint32_t kABytes = kBM * kBK * 2;
+constexpr uint32_t kBBytes = kBN * kBK * 2;
+constexpr uint32_t kStageBytes = kABytes + kBBytes;
+constexpr uint32_t kTmemCols = 2 * kBN;
+constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, kBN);
+constexpr size_t kSmemBytes = static_cast<size_t>(kStages) * kStageBytes + 1024;
+
+static_assert(kBK * 2 == 128, "one K slice must be one 128-byte swizzle row");
+static_assert(kTmemCols <= 512, "two accumulators must fit in TMEM");
+
+struct Tile {
+    int cls, b, mt, nt, local;
+};
+
+__device__ __forceinline__ Tile decode_tile(const GemmParams& P, int tile) {
+    int c = 0;
+    while (c + 1 < P.nclasses && tile >= P.cls[c + 1].tile_begin) ++c;
+    const GemmClass& C = P.cls[c];
+    const int local = tile - C.tile_begin;
+    const int per = C.tiles_m * C.tiles_n;
+    const int b = local / per;
+    const int rem = local - b * per;
+    const int mt = rem / C.tiles_n;
+    return Tile{c, b, mt, rem - mt * C.tiles_n, rem};
+}
+
+__device__ __forceinline__ void unpack8(const uint4& u, float* v) {
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float2 f = __bfloat1622float2(h[k]);
+        v[2 * k] = f.x;
+        v[2 * k + 1] = f.y;
+    }
+}
+
+__device__ __forceinline__ uint4 pack8(const float* v) {
+    uint4 u;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&u);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) h[k] = __floats2bfloat162_rn(v[2 * k], v[2 * k + 1]);
+    return u;
+}
+
+__device__ __forceinline__ void raise_timeout(const GemmParams& P, volatile int* abort_flag) {
+    atomicOr(P.status, kStatusTimeout);
+    *abort_flag = 1;
+}
+
+}  // namespace
+
+__global__ void __launch_bounds__(kThreads, 1)
+ns_gemm_kernel(const __grid_constant__ GemmParams P) {
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t full_bar[kStages];
+    __shared__ __align__(8) uint64_t empty_bar[kStages];
+    __shared__ __align__(8) uint64_t tfull_bar[2];
+    __shared__ __align__(8) uint64_t tempty_bar[2];
+    __shared__ __align__(8) uint64_t drain_bar;
+    __shared__ uint32_t tmem_slot;
+    __shared__ int abort_sh;
+    volatile int* abort_flag = &abort_sh;
+
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint64_t budget = P.budget_ns;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full_bar[s], 1);
+            mbar_init(&empty_bar[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&tfull_bar[a], 1);
+            mbar_init(&tempty_bar[a], 128);
+        }
+        mbar_init(&drain_bar, 1);
+        abort_sh = 0;
+        fence_barrier_init();
+        fence_proxy_async_smem();
+    }
+    if (warp == 0 && lane == 0) {
+        for (int c = 0; c < P.nclasses; ++c) {
+            tma_prefetch_desc(&P.cls[c].tmA);
+            tma_prefetch_desc(&P.cls[c].tmB);
+        }
+    }
+    if (warp == 1) {
+        tmem_alloc(&tmem_slot, kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = tmem_slot;
+
+    if (warp == 0) {
+        // ---------------------------------------------------- TMA producer
+        if (lane == 0) {
+            uint32_t stage = 0, phase = 0;
+            for (int tile = blockIdx.x; tile < P.total_tiles; tile += gridDim.x) {
+                const Tile t = decode_tile(P, tile);
+                const GemmClass& C = P.cls[t.cls];
+                const int nkb = (C.K + kBK - 1) / kBK;
+                bool ok = true;
+                for (int kb = 0; kb < nkb; ++kb) {
+                    if (!mbar_wait_bounded(&empty_bar[stage], phase ^ 1u, budget, abort_flag)) {
+                        raise_timeout(P, abort_flag);
+                        ok = false;
+                        break;
+                    }
+                    uint8_t* sa = smem + stage * kStageBytes;
+                    mbar_arrive_expect_tx(&full_bar[stage], kStageBytes);
+                    tma_load_3d(sa, &C.tmA, kb * kBK, t.mt * kBM, t.b, &full_bar[stage]);
+                    tma_load_3d(sa + kABytes, &C.tmB, kb * kBK, t.nt * kBN, t.b, &full_bar[stage]);
+                    if (++stage == kStages) { stage = 0; phase ^= 1u; }
+                }
+                if (!ok) break;
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            uint32_t stage = 0, phase = 0;
+            int it = 0;
+            for (int tile = blockIdx.x; tile < P.total_tiles; tile += gridDim.x, ++it) {
+                const Tile t = decode_tile(P, tile);
+                const GemmClass& C = P.cls[t.cls];
+                const int nkb = (C.K + kBK - 1) / kBK;
+                const uint32_t acc = it & 1, acc_phase = (it >> 1) & 1;
+                if (!mbar_wait_bounded(&tempty_bar[acc], acc_phase ^ 1u, budget, abort_flag)) {
+                    raise_timeout(P, abort_flag);
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + acc * kBN;
+                bool ok = true;
+                for (int kb = 0; kb < nkb; ++kb) {
+                    if (!mbar_wait_bounded(&full_bar[stage], phase, budget, abort_flag)) {
+                        raise_timeout(P, abort_flag);
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(smem + stage * kStageBytes);
+                    const uint64_t da = smem_desc_k_sw128(sa);
+                    const uint64_t db = smem_desc_k_sw128(sa + kABytes);
+#pragma unroll
+                    for (int kk = 0; kk < kBK / 16; ++kk) {
+                        // +32 bytes along K per 16-element MMA slice (encoded >> 4).
+                        tc_mma_bf16(d_tmem, da + 2 * kk, db + 2 * kk, kIdesc,
+                                    (kb | kk) != 0 ? 1u : 0u);
+                    }
+                    tc_commit(&empty_bar[stage]);
+                    if (++stage == kStages) { stage = 0; phase ^= 1u; }
+                }
+                if (!ok) break;
+                tc_commit(&tfull_bar[acc]);
+            }
+            // Do not release TMEM while MMAs may still be in flight.
+            tc_commit(&drain_bar);
+            if (!mbar_wait_bounded(&drain_bar, 0, budget, nullptr)) raise_timeout(P, abort_flag);
+        }
+    } else {
+        // -------------------------------------------------------- epilogue
+        const int ew = warp - 2;          // epilogue warp 0..3
+        const int quarter = warp & 3;     // TMEM lanes this warp may read
+        int it = 0;
+        for (int tile = blockIdx.x; tile < P.total_tiles; tile += gridDim.x, ++it) {
+            const Tile t = decode_tile(P, tile);
+            const GemmClass& C = P.cls[t.cls];
+            const uint32_t acc = it & 1, acc_phase = (it >> 1) & 1;
+            if (!mbar_wait_bounded(&tfull_bar[acc], acc_phase, budget, abort_flag)) {
+                raise_timeout(P, abort_flag);
+                break;
+            }
+            tc_fence_after();
+            const int M = C.M, N = C.N;
+            const int row = t.mt * kBM + quarter * 32 + lane;
+            const bool rok = row < M;
+            const int g = C.mat_of[t.b];
+            const MatDesc& md = P.mats[g];
+            const float kx = P.first ? P.scal[g].k : 1.f;
+            const size_t bs = static_cast<size_t>(M) * N;
+            const __nv_bfloat16* ein = C.ein != nullptr ? C.ein + t.b * bs : nullptr;
+            __nv_bfloat16* out = C.out != nullptr ? C.out + t.b * bs : nullptr;
+            __nv_bfloat16* outT = C.outT != nullptr ? C.outT + t.b * bs : nullptr;
+            const bool need_ein = (P.phase != kGram);
+            const bool last_bx = (P.phase == kBX) && P.last;
+            // NS frame row / column scalings of D = L O R (swapped when transposed).
+            const float* uvec = md.trans ? md.R : md.L;
+            const float* vvec = md.trans ? md.L : md.R;
+            const float urow = (last_bx && rok) ? uvec[row] : 0.f;
+            float sum_o = 0.f, sum_d = 0.f;
+
+            const int nch = min(kBN / 32, (N - t.nt * kBN + 31) / 32);
+            uint4 xnext[4];
+            auto load_ein = [&](int ch, uint4 (&dst)[4]) {
+                const int col0 = t.nt * kBN + ch * 32;
+#pragma unroll
+                for (int q8 = 0; q8 < 4; ++q8) {
+                    if (rok && col0 + q8 * 8 < N)
+                        dst[q8] = __ldg(reinterpret_cast<const uint4*>(
+                            ein + static_cast<size_t>(row) * N + col0 + q8 * 8));
+                    else
+                        dst[q8] = make_uint4(0u, 0u, 0u, 0u);
+                }
+            };
+            if (need_ein) load_ein(0, xnext);
+
+            for (int ch = 0; ch < nch; ++ch) {
+                const int col0 = t.nt * kBN + ch * 32;
+                uint4 xin[4];
+#pragma unroll
+                for (int q8 = 0; q8 < 4; ++q8) xin[q8] = xnext[q8];
+                if (need_ein && ch + 1 < nch) load_ein(ch + 1, xnext);
+                float v[32];
+                tmem_ld_32cols(tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                                   acc * kBN + ch * 32, v);
+                if (P.phase == kGram) {
+                    const float sc = kx * kx;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] *= sc;
+                } else {
+                    float x[32];
+#pragma unroll
+                    for (int q8 = 0; q8 < 4; ++q8) unpack8(xin[q8], x + 8 * q8);
+                    if (P.phase == kPoly) {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) v[j] = fmaf(P.b, x[j], P.c * v[j]);
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) v[j] = kx * fmaf(P.a, x[j], v[j]);
+                    }
+                }
+                if (!rok) continue;
+                if (!last_bx) {
+#pragma unroll
+                    for (int q8 = 0; q8 < 4; ++q8)
+                        if (col0 + q8 * 8 < N)
+                            *reinterpret_cast<uint4*>(out + static_cast<size_t>(row) * N + col0 +
+                                                      q8 * 8) = pack8(v + 8 * q8);
+                    if (outT != nullptr) {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (col0 + j < N)
+                                outT[static_cast<size_t>(col0 + j) * M + row] = __float2bfloat16_rn(v[j]);
+                    }
+                } else {
+                    // O in W's orientation, then partial sums of O^2 and D^2.
+                    float ob[32];
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) ob[j] = __bfloat162float(__float2bfloat16_rn(v[j]));
+                    if (!md.trans) {
+#pragma unroll
+                        for (int q8 = 0; q8 < 4; ++q8)
+                            if (col0 + q8 * 8 < N)
+                                *reinterpret_cast<uint4*>(md.O + static_cast<size_t>(row) * N + col0 +
+                                                          q8 * 8) = pack8(v + 8 * q8);
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (col0 + j < N)
+                                md.O[static_cast<size_t>(col0 + j) * M + row] = __float2bfloat16_rn(v[j]);
+                    }
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        if (col0 + j < N) {
+                            const float o = ob[j];
+                            const float dv = urow * o * vvec[col0 + j];
+                            sum_o = fmaf(o, o, sum_o);
+                            sum_d = fmaf(dv, dv, sum_d);
+                        }
+                    }
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(&tempty_bar[acc]);
+            if (last_bx) {
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    sum_o += __shfl_xor_sync(0xffffffffu, sum_o, o);
+                    sum_d += __shfl_xor_sync(0xffffffffu, sum_d, o);
+                }
+                if (lane == 0) {
+                    float* dst = md.nspart + (static_cast<size_t>(t.local) * 4 + ew) * 2;
+                    dst[0] = sum_o;
+                    dst[1] = sum_d;
+                }
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, kTmemCols);
+    }
+}
+
+size_t ns_gemm_smem_bytes() { return kSmemBytes; }
+
+cudaError_t launch_ns_gemm(const GemmParams& P, int grid, cudaStream_t s) {
+    static bool configured = false;
+    if (!configured) {
+        const cudaError_t e = cudaFuncSetAttribute(
+            ns_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kSmemBytes));
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    ns_gemm_kernel<<<grid, kThreads, kSmemBytes, s>>>(P);
+    return cudaGetLastError();
+}
+
+}  // namespace malt

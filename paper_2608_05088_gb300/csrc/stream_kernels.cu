@@ -1,0 +1,476 @@
+// stream_kernels.cu -- the HBM-bound stages of the MALT / MALTER step.
+//
+//   stats     Algorithm 1, M_t / l_t / r_t lines: one pass over G and M that
+//             updates the momentum and writes per-tile partial sums of G^2 for
+//             every row and every column (eq. dp_preconditioner).
+//   finalize  l, r EMAs from the partials and L = (l+eps)^(-1/8),
+//             R = (r+eps)^(-1/8) (Algorithm 1, L_t / R_t line); bumps t.
+//   prescale  Mt = L M R (Algorithm 1, Mt line), written as bf16 in both
+//             orientations for the Newton-Schulz GEMMs, with partial sums of
+//             Mt^2 (and of (L G R)^2 for MALTER, Algorithm 2 nu_t line).
+//   norms     ||Mt||_F and ||L G R||_F^2 per matrix from those partials.
+//   scalars   ||O||_F, ||D||_F, MALTER's nu and alpha (Section 3.5) and the
+//             grafted scale lr * alpha * ||O|| / (||D|| + eps) per matrix.
+//   apply     W <- (1 - lr wd) W - scale * L O R (Algorithm 1, W_t line).
+//
+// All reductions run in a fixed order (no atomics), so a step is bitwise
+// reproducible.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "ptx.cuh"
+
+namespace malt {
+
+namespace {
+
+__device__ __forceinline__ int find_mat(const int32_t* __restrict__ pref, int nmat, int32_t x) {
+    int lo = 0, hi = nmat - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (__ldg(pref + mid) <= x) lo = mid; else hi = mid - 1;
+    }
+    return lo;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Sum of v over a block of blockDim.x threads (multiple of 32, <= 1024), fixed
+// order; the result is valid in thread 0.
+__device__ __forceinline__ float block_sum(float v, float* sh /* >= 32 floats */) {
+    v = warp_sum(v);
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) sh[w] = v;
+    __syncthreads();
+    float s = 0.f;
+    if (threadIdx.x == 0) {
+        const int nw = blockDim.x >> 5;
+        for (int i = 0; i < nw; ++i) s += sh[i];
+    }
+    __syncthreads();
+    return s;
+}
+
+__device__ __forceinline__ void load8(const void* base, bool bf16, size_t off, float (&v)[8]) {
+    if (bf16) {
+        const uint4 u = __ldg(reinterpret_cast<const uint4*>(
+            static_cast<const __nv_bfloat16*>(base) + off));
+        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float2 f = __bfloat1622float2(h[k]);
+            v[2 * k] = f.x;
+            v[2 * k + 1] = f.y;
+        }
+    } else {
+        const float4* p = reinterpret_cast<const float4*>(static_cast<const float*>(base) + off);
+        const float4 a = __ldg(p), b = __ldg(p + 1);
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+        v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    }
+}
+
+__device__ __forceinline__ uint4 pack8_bf16(const float (&v)[8]) {
+    uint4 u;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&u);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) h[k] = __floats2bfloat162_rn(v[2 * k], v[2 * k + 1]);
+    return u;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------- binding
+__global__ void bind_kernel(const __grid_constant__ BindParams P, UserPtrs* __restrict__ table) {
+    const int i = threadIdx.x;
+    if (i < P.count) table[P.offset + i] = P.p[i];
+}
+
+// ------------------------------------------------------------------ stats
+// One block = kStatRows x kStatCols of one matrix; warp w owns 8 rows, lane
+// owns 8 consecutive columns.  Row sums reduce across the warp; column sums
+// accumulate in registers over the warp's rows, then across the 8 warps in
+// shared memory.
+constexpr int kStatRowsPerWarp = kStatRows / 8;
+constexpr int kStatBatch = 4;
+
+__global__ void __launch_bounds__(256)
+stats_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
+             const int32_t* __restrict__ pref, int nmat, float mu1) {
+    __shared__ __align__(16) float colsh[8][kStatCols];
+    const int g = find_mat(pref, nmat, blockIdx.x);
+    const MatDesc& d = mats[g];
+    const int m = d.m, n = d.n;
+    const int local = blockIdx.x - __ldg(pref + g);
+    const int rb = local / d.stat_cb, cb = local - rb * d.stat_cb;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int col = cb * kStatCols + lane * 8;
+    const bool colok = col < n;
+    const int row0 = rb * kStatRows + warp * kStatRowsPerWarp;
+    const UserPtrs up = ptrs[g];
+    const bool gbf = d.g_bf16 != 0;
+    float* __restrict__ Mp = up.m;
+    const float om = 1.f - mu1;
+
+    float csum[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) csum[j] = 0.f;
+    float myrow = 0.f;
+
+#pragma unroll
+    for (int rb4 = 0; rb4 < kStatRowsPerWarp; rb4 += kStatBatch) {
+        float gv[kStatBatch][8], mv[kStatBatch][8];
+        bool ok[kStatBatch];
+#pragma unroll
+        for (int u = 0; u < kStatBatch; ++u) {
+            const int row = row0 + rb4 + u;
+            ok[u] = colok && row < m;
+            if (ok[u]) {
+                const size_t off = static_cast<size_t>(row) * n + col;
+                load8(up.g, gbf, off, gv[u]);
+                const float4* mp = reinterpret_cast<const float4*>(Mp + off);
+                const float4 a = mp[0], b = mp[1];
+                mv[u][0] = a.x; mv[u][1] = a.y; mv[u][2] = a.z; mv[u][3] = a.w;
+                mv[u][4] = b.x; mv[u][5] = b.y; mv[u][6] = b.z; mv[u][7] = b.w;
+            } else {
+#pragma unroll
+                for (int j = 0; j < 8; ++j) { gv[u][j] = 0.f; mv[u][j] = 0.f; }
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kStatBatch; ++u) {
+            float rs = 0.f;
+            float nm[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const float gj = gv[u][j];
+                nm[j] = fmaf(mu1, mv[u][j], om * gj);
+                const float sq = gj * gj;
+                rs += sq;
+                csum[j] += sq;
+            }
+            if (ok[u]) {
+                const size_t off = static_cast<size_t>(row0 + rb4 + u) * n + col;
+                float4* mp = reinterpret_cast<float4*>(Mp + off);
+                mp[0] = make_float4(nm[0], nm[1], nm[2], nm[3]);
+                mp[1] = make_float4(nm[4], nm[5], nm[6], nm[7]);
+            }
+            rs = warp_sum(rs);
+            if (lane == rb4 + u) myrow = rs;
+        }
+    }
+    if (lane < kStatRowsPerWarp && row0 + lane < m)
+        d.rowpart[static_cast<size_t>(cb) * m + row0 + lane] = myrow;
+
+    float4* cs = reinterpret_cast<float4*>(&colsh[warp][lane * 8]);
+    cs[0] = make_float4(csum[0], csum[1], csum[2], csum[3]);
+    cs[1] = make_float4(csum[4], csum[5], csum[6], csum[7]);
+    __syncthreads();
+    const int c = threadIdx.x;
+    const int gc = cb * kStatCols + c;
+    if (gc < n) {
+        float s = 0.f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) s += colsh[w][c];
+        d.colpart[static_cast<size_t>(rb) * n + gc] = s;
+    }
+}
+
+// --------------------------------------------------------------- finalize
+__global__ void __launch_bounds__(256)
+finalize_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
+                const int32_t* __restrict__ pref, int nmat, int32_t total,
+                float mu2, float eps, long long* tcount) {
+    const int32_t x = blockIdx.x * blockDim.x + threadIdx.x;
+    if (x == 0) *tcount += 1;                 // 1-based step count
+    if (x >= total) return;
+    const int g = find_mat(pref, nmat, x);
+    const MatDesc& d = mats[g];
+    const int local = x - __ldg(pref + g);
+    const UserPtrs up = ptrs[g];
+    if (local < d.m) {
+        const int i = local;
+        float s = 0.f;
+        for (int cb = 0; cb < d.stat_cb; ++cb) s += d.rowpart[static_cast<size_t>(cb) * d.m + i];
+        const float l = fmaf(mu2, up.l[i], (1.f - mu2) * s);
+        up.l[i] = l;
+        d.L[i] = powf(l + eps, -0.125f);
+    } else {
+        const int j = local - d.m;
+        float s = 0.f;
+        for (int rb = 0; rb < d.stat_rb; ++rb) s += d.colpart[static_cast<size_t>(rb) * d.n + j];
+        const float r = fmaf(mu2, up.r[j], (1.f - mu2) * s);
+        up.r[j] = r;
+        d.R[j] = powf(r + eps, -0.125f);
+    }
+}
+
+// --------------------------------------------------------------- prescale
+__global__ void __launch_bounds__(256)
+prescale_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
+                const int32_t* __restrict__ pref, int nmat, int malter) {
+    __shared__ float tile[kPreTile][kPreTile + 1];
+    __shared__ float red[32];
+    const int g = find_mat(pref, nmat, blockIdx.x);
+    const MatDesc& d = mats[g];
+    const int m = d.m, n = d.n;
+    const int local = blockIdx.x - __ldg(pref + g);
+    const int tr = local / d.pre_tc, tc = local - tr * d.pre_tc;
+    const int r0 = tr * kPreTile, c0 = tc * kPreTile;
+    const int t = threadIdx.x;
+    const UserPtrs up = ptrs[g];
+    const float* __restrict__ Lv = d.L;
+    const float* __restrict__ Rv = d.R;
+
+    float s_mt = 0.f, s_lgr = 0.f;
+    const int cc = (t & 15) * 4;
+    const int col = c0 + cc;
+    float4 R4 = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (col < n) R4 = *reinterpret_cast<const float4*>(Rv + col);
+#pragma unroll
+    for (int pass = 0; pass < 4; ++pass) {
+        const int rr = pass * 16 + (t >> 4);
+        const int row = r0 + rr;
+        float v0 = 0.f, v1 = 0.f, v2 = 0.f, v3 = 0.f;
+        if (row < m && col < n) {
+            const size_t off = static_cast<size_t>(row) * n + col;
+            const float Li = Lv[row];
+            const float4 mv = *reinterpret_cast<const float4*>(up.m + off);
+            v0 = Li * mv.x * R4.x; v1 = Li * mv.y * R4.y;
+            v2 = Li * mv.z * R4.z; v3 = Li * mv.w * R4.w;
+            s_mt += v0 * v0 + v1 * v1 + v2 * v2 + v3 * v3;
+            uint2 pk;
+            *reinterpret_cast<__nv_bfloat162*>(&pk.x) = __floats2bfloat162_rn(v0, v1);
+            *reinterpret_cast<__nv_bfloat162*>(&pk.y) = __floats2bfloat162_rn(v2, v3);
+            *reinterpret_cast<uint2*>(d.Xdir + off) = pk;
+            if (malter) {
+                float gq[4];
+                if (d.g_bf16) {
+                    const uint2 u = *reinterpret_cast<const uint2*>(
+                        static_cast<const __nv_bfloat16*>(up.g) + off);
+                    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+                    const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+                    gq[0] = a.x; gq[1] = a.y; gq[2] = b.x; gq[3] = b.y;
+                } else {
+                    const float4 gf = *reinterpret_cast<const float4*>(
+                        static_cast<const float*>(up.g) + off);
+                    gq[0] = gf.x; gq[1] = gf.y; gq[2] = gf.z; gq[3] = gf.w;
+                }
+                const float a0 = Li * gq[0] * R4.x, a1 = Li * gq[1] * R4.y;
+                const float a2 = Li * gq[2] * R4.z, a3 = Li * gq[3] * R4.w;
+                s_lgr += a0 * a0 + a1 * a1 + a2 * a2 + a3 * a3;
+            }
+        }
+        tile[rr][cc + 0] = v0; tile[rr][cc + 1] = v1;
+        tile[rr][cc + 2] = v2; tile[rr][cc + 3] = v3;
+    }
+    __syncthreads();
+    // Transposed write: output row = column of Mt, 8 consecutive rows of Mt per thread.
+#pragma unroll
+    for (int pass = 0; pass < 2; ++pass) {
+        const int oc = pass * 32 + (t >> 3);
+        const int seg = (t & 7) * 8;
+        const int gcol = c0 + oc, grow = r0 + seg;
+        if (gcol < n && grow < m) {
+            float v[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) v[j] = tile[seg + j][oc];
+            *reinterpret_cast<uint4*>(d.Xtrn + static_cast<size_t>(gcol) * m + grow) = pack8_bf16(v);
+        }
+    }
+    const float a = block_sum(s_mt, red);
+    const float b = block_sum(s_lgr, red);
+    if (t == 0) {
+        d.prepart[2 * local + 0] = a;
+        d.prepart[2 * local + 1] = b;
+    }
+}
+
+// ------------------------------------------------------------------ norms
+__global__ void __launch_bounds__(256)
+norms_kernel(const MatDesc* __restrict__ mats, MatScalars* __restrict__ scal, float ns_eps,
+             int malter) {
+    __shared__ float red[32];
+    const int g = blockIdx.x;
+    const MatDesc& d = mats[g];
+    const int tiles = d.pre_tr * d.pre_tc;
+    float a = 0.f, b = 0.f;
+    for (int i = threadIdx.x; i < tiles; i += blockDim.x) {
+        a += d.prepart[2 * i];
+        b += d.prepart[2 * i + 1];
+    }
+    a = block_sum(a, red);
+    b = block_sum(b, red);
+    if (threadIdx.x == 0) {
+        const float nrm = sqrtf(a);
+        scal[g].norm_mt = nrm;
+        scal[g].k = 1.f / (nrm + ns_eps);
+        scal[g].lgr_sq = malter ? b : 0.f;
+    }
+}
+
+// ---------------------------------------------------------------- scalars
+__global__ void __launch_bounds__(128)
+scalars_kernel(const MatDesc* __restrict__ mats, MatScalars* __restrict__ scal,
+               const long long* __restrict__ tcount, StepHyper hp) {
+    __shared__ float red[32];
+    const int g = blockIdx.x;
+    const MatDesc& d = mats[g];
+    float a = 0.f, b = 0.f;
+    // Four partials (one per epilogue warp) per GEMM tile of the last iteration.
+    for (int i = threadIdx.x; i < 4 * d.ns_tiles; i += blockDim.x) {
+        a += d.nspart[2 * i];
+        b += d.nspart[2 * i + 1];
+    }
+    a = block_sum(a, red);
+    b = block_sum(b, red);
+    if (threadIdx.x == 0) {
+        MatScalars s = scal[g];
+        const double norm_o = sqrt(static_cast<double>(a));
+        const double norm_d = sqrt(static_cast<double>(b));
+        double alpha = 1.0;
+        if (hp.malter) {
+            // Algorithm 2, nu_t line; alpha_t as displayed in Section 3.5.
+            const double t = static_cast<double>(*tcount);
+            const double nu = static_cast<double>(hp.mu2) * s.nu +
+                              (1.0 - static_cast<double>(hp.mu2)) * s.lgr_sq;
+            const double bc = sqrt(1.0 - pow(static_cast<double>(hp.mu2), t)) /
+                              (1.0 - pow(static_cast<double>(hp.mu1), t) + hp.eps);
+            alpha = bc * s.norm_mt / (sqrt(nu) + hp.eps);
+            s.nu = static_cast<float>(nu);
+        }
+        s.norm_o = static_cast<float>(norm_o);
+        s.norm_d = static_cast<float>(norm_d);
+        s.alpha = static_cast<float>(alpha);
+        s.scale = static_cast<float>(hp.lr * alpha * norm_o / (norm_d + hp.eps));
+        scal[g] = s;
+    }
+}
+
+// ------------------------------------------------------------------ apply
+__global__ void __launch_bounds__(256)
+apply_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
+             const MatScalars* __restrict__ scal, const int32_t* __restrict__ pref, int nmat,
+             float decay) {
+    const int g = find_mat(pref, nmat, blockIdx.x);
+    const MatDesc& d = mats[g];
+    const int n = d.n;
+    const int32_t total = d.m * n;
+    const int32_t e0 = (blockIdx.x - __ldg(pref + g)) * kApplyElems;
+    const float s = scal[g].scale;
+    const UserPtrs up = ptrs[g];
+    const bool wbf = d.w_bf16 != 0;
+#pragma unroll
+    for (int v = 0; v < kApplyElems / (256 * 8); ++v) {
+        const int32_t e = e0 + (v * 256 + threadIdx.x) * 8;
+        if (e >= total) break;
+        const int i = e / n, j = e - i * n;
+        float o[8];
+        load8(d.O, true, static_cast<size_t>(e), o);
+        const float Li = d.L[i];
+        const float4 r0 = *reinterpret_cast<const float4*>(d.R + j);
+        const float4 r1 = *reinterpret_cast<const float4*>(d.R + j + 4);
+        const float rj[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
+        float w[8];
+        if (wbf) {
+            const uint4 u = *reinterpret_cast<const uint4*>(static_cast<__nv_bfloat16*>(up.w) + e);
+            const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float2 f = __bfloat1622float2(h[k]);
+                w[2 * k] = f.x;
+                w[2 * k + 1] = f.y;
+            }
+        } else {
+            const float4* wp = reinterpret_cast<const float4*>(static_cast<float*>(up.w) + e);
+            const float4 a = wp[0], b = wp[1];
+            w[0] = a.x; w[1] = a.y; w[2] = a.z; w[3] = a.w;
+            w[4] = b.x; w[5] = b.y; w[6] = b.z; w[7] = b.w;
+        }
+        const float sl = s * Li;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) w[k] = fmaf(-sl * o[k], rj[k], decay * w[k]);
+        if (wbf) {
+            *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(up.w) + e) = pack8_bf16(w);
+        } else {
+            float4* wp = reinterpret_cast<float4*>(static_cast<float*>(up.w) + e);
+            wp[0] = make_float4(w[0], w[1], w[2], w[3]);
+            wp[1] = make_float4(w[4], w[5], w[6], w[7]);
+        }
+    }
+}
+
+// ------------------------------------------------------------- wait probe
+// One thread waits on an mbarrier that nothing ever arrives on, for at most
+// budget_ns, and records whether the wait gave up.
+__global__ void wait_probe_kernel(int32_t* status, uint64_t budget_ns) {
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        fence_barrier_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const bool ok = mbar_wait_bounded(&bar, 0, budget_ns, nullptr);
+        *status = ok ? 0 : kStatusTimeout;
+    }
+}
+
+// ------------------------------------------------------------------ launch
+cudaError_t launch_bind(const BindParams& P, UserPtrs* table, cudaStream_t s) {
+    bind_kernel<<<1, kBindChunk, 0, s>>>(P, table);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_stats(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* pref,
+                         int nmat, int32_t blocks, float mu1, cudaStream_t s) {
+    stats_kernel<<<blocks, 256, 0, s>>>(mats, ptrs, pref, nmat, mu1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_finalize(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* pref,
+                            int nmat, int32_t total, float mu2, float eps, long long* tcount,
+                            cudaStream_t s) {
+    const int blocks = (total + 255) / 256 > 0 ? (total + 255) / 256 : 1;
+    finalize_kernel<<<blocks, 256, 0, s>>>(mats, ptrs, pref, nmat, total, mu2, eps, tcount);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_prescale(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* pref,
+                            int nmat, int32_t blocks, int malter, cudaStream_t s) {
+    prescale_kernel<<<blocks, 256, 0, s>>>(mats, ptrs, pref, nmat, malter);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_norms(const MatDesc* mats, MatScalars* scal, int nmat, float ns_eps,
+                         int malter, cudaStream_t s) {
+    norms_kernel<<<nmat, 256, 0, s>>>(mats, scal, ns_eps, malter);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_scalars(const MatDesc* mats, MatScalars* scal, const long long* tcount,
+                           int nmat, const StepHyper& hp, cudaStream_t s) {
+    scalars_kernel<<<nmat, 128, 0, s>>>(mats, scal, tcount, hp);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_apply(const MatDesc* mats, const UserPtrs* ptrs, const MatScalars* scal,
+                         const int32_t* pref, int nmat, int32_t blocks, float decay,
+                         cudaStream_t s) {
+    apply_kernel<<<blocks, 256, 0, s>>>(mats, ptrs, scal, pref, nmat, decay);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_wait_probe(int32_t* status, uint64_t budget_ns, cudaStream_t s) {
+    wait_probe_kernel<<<1, 32, 0, s>>>(status, budget_ns);
+    return cudaGetLastError();
+}
+
+}  // namespace malt

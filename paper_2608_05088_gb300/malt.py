@@ -1,0 +1,251 @@
+"""ctypes binding of include/malt.h, names unchanged, argument marshalling only.
+
+Every step of the optimizer runs in libmalt.so's CUDA kernels; this module
+turns torch tensors into device pointers and sizes, passes the current CUDA
+stream, and raises on non-zero status codes.  Loading fails loudly when the
+library has not been built (there is no fallback of any kind).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+from . import build as _build
+
+MALT_OK = 0
+MALT_ERR_INVALID_ARG = -1
+MALT_ERR_UNSUPPORTED = -2
+MALT_ERR_MISALIGNED = -3
+MALT_ERR_SHAPE_CHANGED = -4
+MALT_ERR_CUDA = -5
+MALT_ERR_TIMEOUT = -6
+MALT_ERR_OUT_OF_MEMORY = -7
+MALT_F32 = 0
+MALT_BF16 = 1
+SCALARS_PER_MAT = 8
+
+# Exported entry points declared in include/malt.h.
+EXPORTS = ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
+           "malt_set_scalars", "malt_check", "malt_debug_direction", "malt_debug_scalars",
+           "malt_debug_wait_timeout", "malt_workspace_bytes", "malt_status_string",
+           "malt_destroy_state")
+
+
+class malt_param_t(ctypes.Structure):
+    _fields_ = [("w", ctypes.c_void_p), ("w_dtype", ctypes.c_int32),
+                ("g", ctypes.c_void_p), ("g_dtype", ctypes.c_int32),
+                ("m", ctypes.c_void_p), ("l", ctypes.c_void_p), ("r", ctypes.c_void_p),
+                ("rows", ctypes.c_int64), ("cols", ctypes.c_int64)]
+
+
+class malt_hparams_t(ctypes.Structure):
+    _fields_ = [("lr", ctypes.c_float), ("mu1", ctypes.c_float), ("mu2", ctypes.c_float),
+                ("eps", ctypes.c_float), ("weight_decay", ctypes.c_float),
+                ("ns_steps", ctypes.c_int32), ("ns_a", ctypes.c_float),
+                ("ns_b", ctypes.c_float), ("ns_c", ctypes.c_float), ("ns_eps", ctypes.c_float)]
+
+
+class MaltError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: {status_string(code)} ({code})")
+
+
+_LIB = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = False) -> ctypes.CDLL:
+    """Load libmalt.so (built by build.build()).  Raises if it is missing."""
+    global _LIB
+    if _LIB is not None:
+        return _LIB
+    path = library_path()
+    if not os.path.exists(path):
+        if not build_if_missing:
+            raise RuntimeError(f"libmalt.so not built ({path}); run paper_2608_05088_gb300.build.build()")
+        _build.build()
+    lib = ctypes.CDLL(path)
+    vp, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+    P = ctypes.POINTER
+    lib.malt_init_state.argtypes = [P(vp), P(malt_param_t), i32, vp]
+    lib.malt_step.argtypes = [vp, P(malt_param_t), i32, P(malt_hparams_t), vp]
+    lib.malter_step.argtypes = [vp, P(malt_param_t), i32, P(malt_hparams_t), vp]
+    lib.malt_get_scalars.argtypes = [vp, P(ctypes.c_float), i32, P(i64)]
+    lib.malt_set_scalars.argtypes = [vp, P(ctypes.c_float), i32, i64]
+    lib.malt_check.argtypes = [vp]
+    lib.malt_debug_direction.argtypes = [vp, i32, vp, vp]
+    lib.malt_debug_scalars.argtypes = [vp, P(ctypes.c_float), i32]
+    lib.malt_debug_wait_timeout.argtypes = [i64, vp]
+    lib.malt_workspace_bytes.argtypes = [vp]
+    lib.malt_workspace_bytes.restype = ctypes.c_size_t
+    lib.malt_status_string.argtypes = [ctypes.c_int]
+    lib.malt_status_string.restype = ctypes.c_char_p
+    lib.malt_destroy_state.argtypes = [vp]
+    lib.malt_destroy_state.restype = None
+    for name in ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
+                 "malt_set_scalars", "malt_check", "malt_debug_direction",
+                 "malt_debug_scalars", "malt_debug_wait_timeout"):
+        getattr(lib, name).restype = ctypes.c_int
+    _LIB = lib
+    return lib
+
+
+def status_string(code: int) -> str:
+    return load().malt_status_string(int(code)).decode()
+
+
+def _check(code: int, where: str):
+    if code != MALT_OK:
+        raise MaltError(code, where)
+
+
+def hparams(lr=0.02, mu1=0.95, mu2=0.99, eps=1e-8, weight_decay=0.0, ns_steps=5,
+            ns_coeffs=(3.4445, -4.7750, 2.0315), ns_eps=1e-7) -> malt_hparams_t:
+    a, b, c = ns_coeffs
+    return malt_hparams_t(lr, mu1, mu2, eps, weight_decay, ns_steps, a, b, c, ns_eps)
+
+
+def _dtype_code(t) -> int:
+    import torch
+    if t.dtype == torch.float32:
+        return MALT_F32
+    if t.dtype == torch.bfloat16:
+        return MALT_BF16
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def params_array(params):
+    """params: sequence of (W, G, M, l, r) CUDA tensors -> ctypes array."""
+    arr = (malt_param_t * max(len(params), 1))()
+    for i, (W, G, M, l, r) in enumerate(params):
+        for t in (W, G, M, l, r):
+            if not t.is_contiguous():
+                raise ValueError("all tensors must be contiguous")
+        rows, cols = W.shape
+        arr[i] = malt_param_t(W.data_ptr(), _dtype_code(W), G.data_ptr(), _dtype_code(G),
+                              M.data_ptr(), l.data_ptr(), r.data_ptr(), rows, cols)
+    return arr
+
+
+def _stream_handle(stream=None):
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+# --- C-ABI names ------------------------------------------------------------
+
+def malt_init_state(params, stream=None) -> ctypes.c_void_p:
+    lib = load()
+    st = ctypes.c_void_p()
+    arr = params_array(params)
+    _check(lib.malt_init_state(ctypes.byref(st), arr, len(params), _stream_handle(stream)),
+           "malt_init_state")
+    return st
+
+
+def malt_step(st, params, hp: malt_hparams_t, stream=None):
+    arr = params_array(params)
+    _check(load().malt_step(st, arr, len(params), ctypes.byref(hp), _stream_handle(stream)),
+           "malt_step")
+
+
+def malter_step(st, params, hp: malt_hparams_t, stream=None):
+    arr = params_array(params)
+    _check(load().malter_step(st, arr, len(params), ctypes.byref(hp), _stream_handle(stream)),
+           "malter_step")
+
+
+def malt_check(st) -> int:
+    return load().malt_check(st)
+
+
+def malt_get_scalars(st, n: int):
+    nu = (ctypes.c_float * max(n, 1))()
+    t = ctypes.c_int64()
+    _check(load().malt_get_scalars(st, nu, n, ctypes.byref(t)), "malt_get_scalars")
+    return np.array(nu[:n], dtype=np.float32), int(t.value)
+
+
+def malt_set_scalars(st, nu, t: int):
+    n = len(nu)
+    arr = (ctypes.c_float * max(n, 1))(*[float(x) for x in nu])
+    _check(load().malt_set_scalars(st, arr, n, int(t)), "malt_set_scalars")
+
+
+def malt_debug_direction(st, idx: int, out, stream=None):
+    _check(load().malt_debug_direction(st, idx, ctypes.c_void_p(out.data_ptr()),
+                                       _stream_handle(stream)), "malt_debug_direction")
+
+
+def malt_debug_scalars(st, n: int) -> np.ndarray:
+    buf = (ctypes.c_float * max(n * SCALARS_PER_MAT, 1))()
+    _check(load().malt_debug_scalars(st, buf, n), "malt_debug_scalars")
+    return np.array(buf[: n * SCALARS_PER_MAT], dtype=np.float32).reshape(n, SCALARS_PER_MAT)
+
+
+def malt_debug_wait_timeout(budget_ns: int, stream=None) -> int:
+    return load().malt_debug_wait_timeout(int(budget_ns), _stream_handle(stream))
+
+
+def malt_workspace_bytes(st) -> int:
+    return int(load().malt_workspace_bytes(st))
+
+
+def malt_destroy_state(st):
+    load().malt_destroy_state(st)
+
+
+# --- convenience wrapper ------------------------------------------------------
+
+class MaltOptimizer:
+    """Owns a malt_state for a fixed list of (W, G, M, l, r) device tensors.
+    M, l, r are zeroed at construction (Algorithm 1 INITIALIZE line)."""
+
+    def __init__(self, params, stream=None):
+        self.params = list(params)
+        self.n = len(self.params)
+        self.state = malt_init_state(self.params, stream)
+
+    def step(self, hp: malt_hparams_t, malter: bool = False, stream=None, params=None):
+        ps = self.params if params is None else params
+        (malter_step if malter else malt_step)(self.state, ps, hp, stream)
+
+    def check(self) -> int:
+        return malt_check(self.state)
+
+    def scalars(self):
+        return malt_get_scalars(self.state, self.n)
+
+    def set_scalars(self, nu, t):
+        malt_set_scalars(self.state, nu, t)
+
+    def debug_scalars(self):
+        return malt_debug_scalars(self.state, self.n)
+
+    def direction(self, idx: int, stream=None):
+        import torch
+        W = self.params[idx][0]
+        out = torch.empty(W.shape, dtype=torch.bfloat16, device=W.device)
+        malt_debug_direction(self.state, idx, out, stream)
+        return out
+
+    def workspace_bytes(self) -> int:
+        return malt_workspace_bytes(self.state)
+
+    def close(self):
+        if self.state is not None:
+            malt_destroy_state(self.state)
+            self.state = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,78 @@
+"""The C ABI library: builds, loads without a GPU, exports every entry point
+include/malt.h declares, and validates arguments on the host (CPU only)."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+import paper_2608_05088_gb300.malt as malt
+from paper_2608_05088_gb300 import build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def header_functions():
+    names = set()
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", fn)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            for m in re.finditer(r"^\s*[A-Za-z_][\w\s\*]*?\b(malt\w*)\s*\(", src, flags=re.M):
+                names.add(m.group(1))
+    return names
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return malt.load()
+
+
+def test_header_declares_the_binding_names():
+    assert header_functions() == set(malt.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    out = subprocess.run(["nm", "-D", "--defined-only", build.LIB], capture_output=True,
+                         text=True, check=True).stdout
+    exported = {line.split()[-1] for line in out.splitlines() if " T " in line}
+    missing = header_functions() - exported
+    assert not missing, missing
+    for name in header_functions():
+        assert hasattr(lib, name)
+
+
+def test_status_strings(lib):
+    for code in (0, -1, -2, -3, -4, -5, -6, -7):
+        assert malt.status_string(code) != "unknown status"
+    assert malt.status_string(12345) == "unknown status"
+
+
+def _param(rows=64, cols=64, w=16, g=16, m=16, l=16, r=16, wd=malt.MALT_F32):
+    return malt.malt_param_t(w, wd, g, malt.MALT_F32, m, l, r, rows, cols)
+
+
+def test_host_validation_without_gpu(lib):
+    st = ctypes.c_void_p()
+    assert lib.malt_init_state(None, None, 0, None) == malt.MALT_ERR_INVALID_ARG
+    assert lib.malt_init_state(ctypes.byref(st), None, -1, None) == malt.MALT_ERR_INVALID_ARG
+    cases = [
+        (_param(rows=7), malt.MALT_ERR_UNSUPPORTED),
+        (_param(cols=12), malt.MALT_ERR_UNSUPPORTED),
+        (_param(rows=0), malt.MALT_ERR_UNSUPPORTED),
+        (_param(rows=65536, cols=65536), malt.MALT_ERR_UNSUPPORTED),
+        (_param(w=0), malt.MALT_ERR_INVALID_ARG),
+        (_param(m=24), malt.MALT_ERR_MISALIGNED),
+        (_param(wd=7), malt.MALT_ERR_UNSUPPORTED),
+    ]
+    for p, want in cases:
+        arr = (malt.malt_param_t * 1)(p)
+        assert lib.malt_init_state(ctypes.byref(st), arr, 1, None) == want
+        assert not st.value
+    hp = malt.hparams()
+    assert lib.malt_step(None, None, 0, ctypes.byref(hp), None) == malt.MALT_ERR_INVALID_ARG
+    assert lib.malt_debug_wait_timeout(0, None) == malt.MALT_ERR_INVALID_ARG
+    assert lib.malt_workspace_bytes(None) == 0
+    lib.malt_destroy_state(None)

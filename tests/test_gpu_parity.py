@@ -1,0 +1,147 @@
+"""CUDA path vs the fp64 oracle, element by element, on seeded inputs.
+
+Bars: momentum / statistics / ||Mt|| within 1e-5 relative (fp32 arithmetic);
+orthogonalised direction O and the grafting norms within 2e-2 relative
+Frobenius (bf16 Newton-Schulz operands with fp32 accumulation); final weights
+within 5e-3 relative Frobenius and the update W_0 - W_t within 2e-2; bf16
+weights within one bf16 ulp of the oracle's round-to-nearest-even result.
+"""
+import numpy as np
+import pytest
+
+from paper_2608_05088_gb300 import inputs
+from tests.gpu_harness import Run
+
+pytestmark = pytest.mark.gpu
+
+
+def test_single_256x512_malt():
+    """The 256 x 512 fp32 matrix, 3 MALT steps, checked after every step."""
+    wl = inputs.WORKLOADS["single_256x512"]
+    run = Run(wl)
+    for s in range(wl.steps):
+        run.step()
+        assert run.status() == 0
+        run.assert_close(0, f"step {s}")
+    run.close()
+
+
+RAGGED = ((200, 328), (392, 136), (8, 8), (136, 1000), (520, 520), (64, 2056), (1032, 264),
+          (256, 512))
+
+
+@pytest.mark.parametrize("variant", ["malt", "malter"])
+def test_ragged_mixed_shapes(variant):
+    """Shapes that leave ragged tiles in every direction, tall matrices (NS on
+    the transpose), several shape classes in one grouped launch, fp32 and bf16
+    weights side by side."""
+    wl = inputs.Workload("ragged", 31, RAGGED, "f32", 1.5, 0.02, variant, 3)
+    w_dtypes = ["f32", "bf16"] * (len(RAGGED) // 2)
+    run = Run(wl, w_dtypes=w_dtypes)
+    for s in range(wl.steps):
+        run.step()
+        assert run.status() == 0
+        for i in range(len(RAGGED)):
+            run.assert_close(i, f"{variant} step {s}")
+    run.close()
+
+
+def test_bf16_gradients_and_k8():
+    """bf16 gradients, 8 Newton-Schulz iterations, strong anisotropy (sigma 3)."""
+    wl = inputs.Workload("bf16g", 32, ((512, 768), (768, 256)), "bf16", 3.0, 0.02, "malt", 3,
+                         ns_steps=8)
+    run = Run(wl, g_dtype="bf16")
+    for _ in range(wl.steps):
+        run.step()
+    assert run.status() == 0
+    for i in range(2):
+        run.assert_close(i)
+    run.close()
+
+
+def test_zero_gradient_leaves_weights():
+    """G = 0 at t = 1: Mt = 0, O = 0, the grafted scale is 0, W is unchanged."""
+    wl = inputs.Workload("zero", 33, ((128, 256), (264, 136)), "f32", 1.0, 0.02, "malter", 1)
+    run = Run(wl)
+    W0 = [run.host(w).copy() for w in run.W]
+    run.step(grads=[np.zeros(s, np.float32) for s in wl.shapes])
+    assert run.status() == 0
+    for i in range(2):
+        assert np.array_equal(run.host(run.W[i]), W0[i])
+        assert not np.any(run.host(run.opt.direction(i)))
+    run.close()
+
+
+def test_bitwise_deterministic():
+    """Two identical runs give bitwise identical W, M, l, r (no atomics)."""
+    wl = inputs.Workload("det", 34, RAGGED[:5], "bf16", 1.5, 0.02, "malter", 2)
+    outs = []
+    for _ in range(2):
+        run = Run(wl, check=[])
+        for _ in range(wl.steps):
+            run.step(oracle=False)
+        assert run.status() == 0
+        outs.append([run.host(t) for t in run.W + run.M + run.l + run.r])
+        run.close()
+    for a, b in zip(*outs):
+        assert np.array_equal(a, b)
+
+
+def test_checkpoint_roundtrip():
+    """3 steps straight == 1 step, save (M, l, r, nu, t), fresh state, restore,
+    2 more steps; bitwise."""
+    import torch
+    wl = inputs.Workload("ckpt", 35, ((256, 384), (392, 136)), "f32", 1.5, 0.02, "malter", 3)
+    a = Run(wl, check=[])
+    for _ in range(3):
+        a.step(oracle=False)
+    b = Run(wl, check=[])
+    b.step(oracle=False)
+    nu, t = b.opt.scalars()
+    assert t == 1
+    saved = [[x.clone() for x in (b.W[i], b.M[i], b.l[i], b.r[i])] for i in range(2)]
+    b.close()
+    c = Run(wl, check=[])
+    for i in range(2):
+        for dst, src in zip((c.W[i], c.M[i], c.l[i], c.r[i]), saved[i]):
+            dst.copy_(src)
+    c.opt.set_scalars(nu, t)
+    c.steps_done = 1
+    for _ in range(2):
+        c.step(oracle=False)
+    torch.cuda.synchronize()
+    for i in range(2):
+        for x, y in zip((a.W[i], a.M[i], a.l[i], a.r[i]), (c.W[i], c.M[i], c.l[i], c.r[i])):
+            assert torch.equal(x, y)
+    nu_a, t_a = a.opt.scalars()
+    nu_c, t_c = c.opt.scalars()
+    assert t_a == t_c == 3 and np.array_equal(nu_a, nu_c)
+    a.close()
+    c.close()
+
+
+def test_gpt2_small_sampled():
+    """GPT-2 Small 2-D parameter set (48 matrices, bf16 W), 2 MALT steps in one
+    grouped step; one matrix of each shape checked in full against the oracle."""
+    wl = inputs.WORKLOADS["gpt2_small"]
+    check = [0, 1, 2, 3, 45, 46, 47]
+    run = Run(wl, check=check)
+    for _ in range(2):
+        run.step()
+    assert run.status() == 0
+    for i in check:
+        run.assert_close(i)
+    run.close()
+
+
+def test_gpt2_medium_malter_sampled():
+    """GPT-2 Medium (96 matrices), 2 MALTER steps, one matrix per shape checked."""
+    wl = inputs.WORKLOADS["gpt2_medium"]
+    check = [4, 5, 6, 7]
+    run = Run(wl, check=check)
+    for _ in range(2):
+        run.step()
+    assert run.status() == 0
+    for i in check:
+        run.assert_close(i)
+    run.close()
