@@ -1,0 +1,401 @@
+#!/usr/bin/env python
+"""Optimizer steps/s of the MALT update over the GPT-2 Large 2-D parameter set.
+
+One step = one malt_step over all 144 matrices (36 layers x {1280x3840,
+1280x1280, 1280x5120, 5120x1280}, bf16 weights, fp32 state and gradients,
+5 Newton-Schulz iterations): statistics + momentum, preconditioners,
+prescale, the Newton-Schulz GEMMs, graft and apply.  The working set
+(about 15 GB) is far larger than L2, so no flush is needed between steps.
+
+  python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+
+N > 1 runs under torch.distributed.run with one process per GPU; each rank
+updates its own replica of the parameter set (independent problems, no
+collective on the data path) and the value is N * K / (max over ranks of the
+timed region).  Prints one JSON line on rank 0.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "optimizer steps/sec (full GPT-2 param set, 1 GB300)"
+UNIT = "steps/s"
+DEFAULT_WORKLOAD = "gpt2_large"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+NCU_SUMMARY = os.path.join(ROOT, "profiles", "ns_gemm_gpt2_large_ncu.json")
+NS_SOURCE = os.path.join(ROOT, "paper_2608_05088_gb300", "csrc", "ns_gemm.cu")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+# --------------------------------------------------------------------- ranks
+def rank_env():
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def init_dist(backend: str):
+    import torch.distributed as dist
+    rank, world, _ = rank_env()
+    if world > 1 and not dist.is_initialized():
+        dist.init_process_group(backend=backend)
+    return rank, world
+
+
+def barrier():
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized():
+        dist.barrier()
+
+
+def max_over_ranks(x: float, device=None) -> float:
+    """Maximum of a host scalar over all ranks (timing only, never data)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# -------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi sampled every 200 ms while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+
+        def num(v):
+            try:
+                return float(v)
+            except ValueError:
+                return float("nan")
+        sm = [num(r[1]) for r in rows]
+        mx = max(num(r[2]) for r in rows)
+        reasons = set()
+        for r in rows:
+            for name, v in zip(("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                                "sw_power_cap"), r[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        good = [s for s in sm if not math.isnan(s)]
+        return {"sm_mhz": statistics.median(good) if good else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(rows)}
+
+
+# -------------------------------------------------------------------- peaks
+def peaks():
+    try:
+        with open(PEAKS_FILE) as f:
+            p = json.load(f)
+        return p, "measured"
+    except Exception:
+        return FALLBACK_PEAKS, "fallback"
+
+
+def ncu_traffic_per_launch():
+    """DRAM bytes per NS GEMM launch from the committed ncu summary, or None
+    when the kernel source changed since the capture."""
+    try:
+        with open(NCU_SUMMARY) as f:
+            s = json.load(f)
+        with open(NS_SOURCE, "rb") as f:
+            h = hashlib.sha256(f.read()).hexdigest()
+        if s.get("ns_gemm_sha256") != h:
+            return None
+        return float(s["dram_bytes_per_launch_full_size"])
+    except Exception:
+        return None
+
+
+# ------------------------------------------------------------ CPU baseline
+def oracle_sample_time(wl, layer_indices, reps_budget_s=10.0):
+    """Seconds for one oracle step over the given matrices (fp64, all cores),
+    averaged over as many repetitions as fit in about reps_budget_s."""
+    import numpy as np
+    import oracle.malt_ref as ref
+    from paper_2608_05088_gb300 import inputs
+    Ws = [inputs.initial_weight(wl, i).astype(np.float64) for i in layer_indices]
+    Gs = [inputs.gradient(wl, i, 0).astype(np.float64) for i in layer_indices]
+    hp = ref.Hyper(lr=wl.lr, ns_steps=wl.ns_steps)
+    times = []
+    t_all = time.perf_counter()
+    while True:
+        sts = [ref.State.zeros(*wl.shapes[i]) for i in layer_indices]
+        t0 = time.perf_counter()
+        for W, G, st in zip(Ws, Gs, sts):
+            ref.malt_step_ref(W, G, st, hp, variant=wl.variant, weight_dtype=wl.weight_dtype)
+        times.append(time.perf_counter() - t0)
+        if time.perf_counter() - t_all > reps_budget_s:
+            break
+    return statistics.median(times), len(times)
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+# ----------------------------------------------------------------- reference
+def run_reference(args):
+    """The fp64 oracle timed on the host cores, one bounded sample per step
+    (the 4 matrices of one GPT-2 layer, scaled to the full 36-layer set)."""
+    rank, world, _ = rank_env()
+    if rank != 0:
+        return
+    import numpy as np
+    import oracle.malt_ref as ref
+    from paper_2608_05088_gb300 import inputs
+    wl = inputs.WORKLOADS[args.workload]
+    per_layer = 4 if wl.name.startswith("gpt2") else len(wl.shapes)
+    layers = len(wl.shapes) // per_layer
+    idx = list(range(per_layer))
+    Ws = [inputs.initial_weight(wl, i).astype(np.float64) for i in idx]
+    sts = [ref.State.zeros(*wl.shapes[i]) for i in idx]
+    hp = ref.Hyper(lr=wl.lr, ns_steps=wl.ns_steps)
+    times = []
+    for s in range(args.warmup + args.steps):
+        Gs = [inputs.gradient(wl, i, s).astype(np.float64) for i in idx]
+        t0 = time.perf_counter()
+        for j in range(per_layer):
+            Ws[j], _ = ref.malt_step_ref(Ws[j], Gs[j], sts[j], hp, variant=wl.variant,
+                                         weight_dtype=wl.weight_dtype)
+        if s >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    t_step = sum(times) / len(times) * layers
+    value = 1.0 / t_step
+    sample = (f"one layer ({per_layer} matrices) of {wl.name} per step, scaled x{layers} "
+              f"to the full set")
+    out = {"metric": METRIC, "value": value, "unit": UNIT, "impl": "reference",
+           "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": t_step * 1e3, "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": workload_config(wl),
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(),
+                            "kind": "oracle", "sample": sample},
+           "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def workload_config(wl):
+    return {"workload": wl.name, "matrices": len(wl.shapes),
+            "shapes": sorted(set(f"{m}x{n}" for m, n in wl.shapes)),
+            "elements": wl.elements, "variant": wl.variant, "ns_steps": wl.ns_steps,
+            "weights": wl.weight_dtype, "state": "f32", "gradients": "f32",
+            "lr": wl.lr, "l2": "inputs larger than L2 (working set ~%.0f GB)" % (
+                wl.elements * 26 / 1e9)}
+
+
+# --------------------------------------------------------------------- MALT
+def run_malt(args):
+    import numpy as np
+    import torch
+    rank, world = init_dist("nccl")
+    _, _, local = rank_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    import paper_2608_05088_gb300.malt as malt
+    from paper_2608_05088_gb300 import build, inputs
+    build.build()
+    wl = inputs.WORKLOADS[args.workload]
+    n = len(wl.shapes)
+    wdt = torch.bfloat16 if wl.weight_dtype == "bf16" else torch.float32
+
+    # Inputs: drawn on the host once, made resident in HBM before timing.
+    W0 = inputs.initial_weights(wl)
+    G_host = [torch.from_numpy(g).pin_memory() for g in inputs.gradients_for_step(wl, 0)]
+    W = [torch.from_numpy(w).to(dev).to(wdt) for w in W0]
+    G = [g.to(dev) for g in G_host]
+    M = [torch.empty(s, dtype=torch.float32, device=dev) for s in wl.shapes]
+    l = [torch.empty(s[0], dtype=torch.float32, device=dev) for s in wl.shapes]
+    r = [torch.empty(s[1], dtype=torch.float32, device=dev) for s in wl.shapes]
+    params = list(zip(W, G, M, l, r))
+    opt = malt.MaltOptimizer(params)
+    hp = malt.hparams(lr=wl.lr, ns_steps=wl.ns_steps)
+    malter = wl.variant == "malter"
+    stream = torch.cuda.current_stream()
+
+    for _ in range(args.warmup):
+        opt.step(hp, malter=malter)
+    torch.cuda.synchronize()
+    status = opt.check()
+    if status != malt.MALT_OK:
+        raise SystemExit(f"warm-up step failed: {malt.status_string(status)}")
+
+    # ---- device-resident timed region
+    opt.profile(True)
+    opt.profile_read()
+    clocks = ClockSampler(local)
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        opt.step(hp, malter=malter)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    prof = opt.profile_read()
+    opt.profile(False)
+    status = opt.check()
+    if status != malt.MALT_OK:
+        raise SystemExit(f"timed step failed: {malt.status_string(status)}")
+    t_ms = max_over_ranks(e0.elapsed_time(e1), dev)
+    value = world * args.steps / (t_ms / 1e3)
+
+    # ---- end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        W_host = [torch.empty(w.shape, dtype=w.dtype, pin_memory=True) for w in W]
+        h2d = sum(g.numel() * g.element_size() for g in G_host)
+        d2h = sum(w.numel() * w.element_size() for w in W)
+
+        def e2e_step():
+            for g_dev, g_h in zip(G, G_host):
+                g_dev.copy_(g_h, non_blocking=True)
+            opt.step(hp, malter=malter)
+            for w_h, w_dev in zip(W_host, W):
+                w_h.copy_(w_dev, non_blocking=True)
+
+        for _ in range(max(1, args.warmup // 2)):
+            e2e_step()
+        torch.cuda.synchronize()
+        barrier()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        te = max_over_ranks(a.elapsed_time(b), dev)
+        e2e = {"value": world * args.steps / (te / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+        if opt.check() != malt.MALT_OK:
+            raise SystemExit("e2e step failed")
+
+    if rank != 0:
+        return
+
+    # ---- roofline of the dominant kernel (the Newton-Schulz GEMMs)
+    pk, pk_src = peaks()
+    ns_ms = sum(prof[k][0] for k in ("ns_gram", "ns_poly", "ns_bx"))
+    ns_launches = sum(prof[k][1] for k in ("ns_gram", "ns_poly", "ns_bx"))
+    flops = wl.ns_flops_dense() * args.steps
+    achieved = flops / (ns_ms / 1e3) / 1e12
+    peak = float(pk["bf16_tflops_sustained"])
+    traffic = ncu_traffic_per_launch()
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "traffic": traffic,
+                "kernel": "ns_gemm_kernel (Gram, Poly, BX launches)",
+                "peak_source": f"{pk_src}: bf16_tflops_sustained",
+                "launch_avg_ms": ns_ms / max(ns_launches, 1)}
+    elems = wl.elements
+    wbytes = 2 if wl.weight_dtype == "bf16" else 4
+    mem = {}
+    for kind, bytes_per_elem in (("stats", 12.0), ("prescale", 8.0 + (4.0 if malter else 0.0)),
+                                 ("apply", 2.0 * wbytes + 2.0)):
+        ms = prof[kind][0]
+        gbs = bytes_per_elem * elems * args.steps / (ms / 1e3) / 1e9 if ms > 0 else None
+        mem[kind] = {"ms_per_step": ms / args.steps, "bytes_per_elem": bytes_per_elem,
+                     "achieved_gbs": gbs,
+                     "frac_of_hbm": (gbs / float(pk["hbm_gbs"])) if gbs else None}
+    breakdown = {k: round(v[0] / args.steps, 4) for k, v in prof.items()}
+    launches = sum(v[1] for v in prof.values())
+
+    cpu = None
+    if not args.no_cpu_baseline and world == 1:
+        per_layer = 4
+        t_layer, reps = oracle_sample_time(wl, list(range(per_layer)))
+        layers = len(wl.shapes) // per_layer
+        cpu = {"value": 1.0 / (t_layer * layers), "unit": UNIT, "cores": cpu_cores(),
+               "kind": "oracle",
+               "sample": f"one MALT step of layer 0 ({per_layer} matrices) in fp64, "
+                         f"median of {reps}, scaled x{layers} to the full set"}
+
+    out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_ms / args.steps,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+           "dtype": "bf16", "data": "synthetic", "config": workload_config(wl),
+           "clocks": clk, "e2e": e2e, "gpu_launches": launches, "roofline": roofline,
+           "hbm_kernels": mem, "ms_per_step_by_kernel": breakdown,
+           "cpu_baseline": cpu, "workspace_bytes": opt.workspace_bytes()}
+    print(json.dumps(out), flush=True)
+    opt.close()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("malt", "reference"), default="malt")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_malt(args)
+
+
+if __name__ == "__main__":
+    main()

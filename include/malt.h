@@ -152,6 +152,26 @@ int malt_debug_scalars(malt_state_t* st, float* out_host, int32_t n);
  * up as designed (the expected result), MALT_OK if it somehow completed. */
 int malt_debug_wait_timeout(int64_t budget_ns, void* stream);
 
+/* Per-kernel timing.  While enabled, every kernel launch of a step is
+ * bracketed by CUDA events recorded on the step's stream; malt_profile_read
+ * synchronises, adds the elapsed device time (milliseconds) and the launch
+ * count of each kernel kind into ms_out[kind] / launches_out[kind]
+ * (nkinds entries, up to MALT_NUM_KINDS) and resets the accumulators.
+ * Profiling only adds event records; it changes no result. */
+#define MALT_KIND_BIND      0
+#define MALT_KIND_STATS     1
+#define MALT_KIND_FINALIZE  2
+#define MALT_KIND_PRESCALE  3
+#define MALT_KIND_NORMS     4
+#define MALT_KIND_NS_GRAM   5
+#define MALT_KIND_NS_POLY   6
+#define MALT_KIND_NS_BX     7
+#define MALT_KIND_SCALARS   8
+#define MALT_KIND_APPLY     9
+#define MALT_NUM_KINDS     10
+int malt_profile_enable(malt_state_t* st, int32_t enable);
+int malt_profile_read(malt_state_t* st, double* ms_out, int64_t* launches_out, int32_t nkinds);
+
 /* Bytes of device workspace the state holds. */
 size_t malt_workspace_bytes(const malt_state_t* st);
 

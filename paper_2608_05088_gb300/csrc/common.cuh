@@ -24,6 +24,7 @@ constexpr int kBM = 128;
 constexpr int kBN = 256;
 constexpr int kBK = 64;
 constexpr int kStages = 4;
+constexpr int kBMN = 64;           // MN extent of one 128-byte swizzle atom (bf16)
 constexpr int kMaxClasses = 8;     // shape classes per GEMM launch
 constexpr int kBindChunk = 128;    // parameters per pointer-binding launch
 constexpr int kScalarsPerMat = 8;  // debug scalars per matrix
@@ -57,8 +58,7 @@ struct MatDesc {
     float* R;                // [n]  (r + eps)^(-1/8)
     float* prepart;          // [pre_tiles][2]  sum Mt^2, sum (L G R)^2
     float* nspart;           // [ns_tiles][4][2]  per epilogue warp: sum O^2, sum D^2
-    __nv_bfloat16* Xdir;     // Mt in W's orientation (m x n), NS buffer 0
-    __nv_bfloat16* Xtrn;     // Mt^T (n x m), NS buffer 0
+    __nv_bfloat16* X0;       // NS-frame Mt (p x q, bf16): Mt, or Mt^T when trans
     __nv_bfloat16* O;        // [m][n] orthogonalised direction, W's orientation
 };
 
@@ -81,17 +81,17 @@ struct StepHyper {
 enum GemmPhase : int32_t { kGram = 0, kPoly = 1, kBX = 2 };
 
 struct GemmClass {  // 64-byte aligned through its CUtensorMap members
-    CUtensorMap tmA;              // operand A rows (box kBK x kBM)
-    CUtensorMap tmB;              // operand B rows (box kBK x kBN)
+    CUtensorMap tmA;              // operand A: rows of a K-major matrix (box kBK x kBM)
+    CUtensorMap tmB;              // operand B: K-major rows (box kBK x kBN), or for kBX
+                                  // an MN-major [K][N] matrix (box kBMN x kBK)
     int32_t M, N, K;              // per-matrix product shape
     int32_t batch;
     int32_t tiles_m, tiles_n;
     int32_t tile_begin;           // first global tile of this class in the launch
     int32_t pad_;
     const int32_t* mat_of;        // [batch] -> matrix index
-    const __nv_bfloat16* ein;     // epilogue input (A for kPoly, X for kBX), [batch][M][N]
-    __nv_bfloat16* out;           // direct output [batch][M][N]
-    __nv_bfloat16* outT;          // transposed output [batch][N][M] (kBX, not last)
+    const __nv_bfloat16* ein;     // epilogue input (A for kPoly), [batch][M][N]
+    __nv_bfloat16* out;           // output [batch][M][N] (unused by the last kBX)
 };
 
 struct GemmParams {

@@ -62,11 +62,10 @@ struct ShapeClass {
     int p = 0, q = 0, batch = 0;
     std::vector<int> mats;
     int32_t* d_mat_of = nullptr;
-    __nv_bfloat16* X[2] = {nullptr, nullptr};
-    __nv_bfloat16* Xt[2] = {nullptr, nullptr};
-    __nv_bfloat16* A = nullptr;
-    __nv_bfloat16* B = nullptr;
-    CUtensorMap tmXa[2], tmXb[2], tmXtb[2], tmAa, tmAb, tmBa;
+    __nv_bfloat16* X[2] = {nullptr, nullptr};   // ping-pong NS iterates [batch][p][q]
+    __nv_bfloat16* A = nullptr;                  // X X^T        [batch][p][p]
+    __nv_bfloat16* B = nullptr;                  // aI + bA + cA^2 [batch][p][p]
+    CUtensorMap tmXa[2], tmXb[2], tmXmn[2], tmAa, tmAb, tmBa;
 };
 
 struct Carver {
@@ -111,6 +110,12 @@ struct malt_state {
     int32_t* d_pref[4] = {nullptr, nullptr, nullptr, nullptr};  // stats, fin, pre, apply
     int32_t blocks_stats = 0, total_fin = 0, blocks_pre = 0, blocks_apply = 0;
     cudaStream_t last_stream = nullptr;
+    // Profiling: event pairs recorded around launches, folded in on read.
+    bool profiling = false;
+    std::vector<cudaEvent_t> ev_pool;
+    std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> ev_pending;
+    double prof_ms[MALT_NUM_KINDS] = {};
+    int64_t prof_launches[MALT_NUM_KINDS] = {};
 };
 
 namespace {
@@ -142,9 +147,49 @@ int validate_hparams(const malt_hparams_t* hp) {
 
 void free_state(malt_state* st) {
     if (st == nullptr) return;
+    for (auto& p : st->ev_pending) {
+        cudaEventDestroy(p.second.first);
+        cudaEventDestroy(p.second.second);
+    }
+    for (cudaEvent_t e : st->ev_pool) cudaEventDestroy(e);
     if (st->ws != nullptr) cudaFree(st->ws);
     delete st;
 }
+
+cudaEvent_t take_event(malt_state* st) {
+    if (!st->ev_pool.empty()) {
+        cudaEvent_t e = st->ev_pool.back();
+        st->ev_pool.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    return e;
+}
+
+// Bracket one launch (or launch group) of a kernel kind with events when
+// profiling is on; always counts the launches.
+struct LaunchScope {
+    malt_state* st;
+    int kind;
+    cudaStream_t s;
+    cudaEvent_t a = nullptr;
+    LaunchScope(malt_state* st_, int kind_, cudaStream_t s_, int launches = 1)
+        : st(st_), kind(kind_), s(s_) {
+        st->prof_launches[kind] += launches;
+        if (st->profiling) {
+            a = take_event(st);
+            if (a != nullptr) cudaEventRecord(a, s);
+        }
+    }
+    ~LaunchScope() {
+        if (a == nullptr) return;
+        cudaEvent_t b = take_event(st);
+        if (b == nullptr) return;
+        cudaEventRecord(b, s);
+        st->ev_pending.push_back({kind, {a, b}});
+    }
+};
 
 int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
     st->nmat = n;
@@ -199,15 +244,13 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         o_O[i] = cv.take(2 * static_cast<size_t>(d.m) * d.n);
     }
     const int nc = static_cast<int>(st->classes.size());
-    std::vector<size_t> o_X0(nc), o_X1(nc), o_Xt0(nc), o_Xt1(nc), o_A(nc), o_B(nc), o_matof(nc);
+    std::vector<size_t> o_X0(nc), o_X1(nc), o_A(nc), o_B(nc), o_matof(nc);
     for (int k = 0; k < nc; ++k) {
         const ShapeClass& C = st->classes[k];
         const size_t pq = static_cast<size_t>(C.batch) * C.p * C.q * 2;
         const size_t pp = static_cast<size_t>(C.batch) * C.p * C.p * 2;
         o_X0[k] = cv.take(pq);
         o_X1[k] = cv.take(pq);
-        o_Xt0[k] = cv.take(pq);
-        o_Xt1[k] = cv.take(pq);
         o_A[k] = cv.take(pp);
         o_B[k] = cv.take(pp);
         o_matof[k] = cv.take(sizeof(int32_t) * C.batch);
@@ -233,8 +276,6 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         ShapeClass& C = st->classes[k];
         C.X[0] = H(o_X0[k]);
         C.X[1] = H(o_X1[k]);
-        C.Xt[0] = H(o_Xt0[k]);
-        C.Xt[1] = H(o_Xt1[k]);
         C.A = H(o_A[k]);
         C.B = H(o_B[k]);
         C.d_mat_of = reinterpret_cast<int32_t*>(base + o_matof[k]);
@@ -250,8 +291,7 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         d.nspart = F(o_ns[i]);
         d.O = H(o_O[i]);
         const size_t slot = static_cast<size_t>(d.bidx) * C.p * C.q;
-        d.Xdir = d.trans ? C.Xt[0] + slot : C.X[0] + slot;
-        d.Xtrn = d.trans ? C.X[0] + slot : C.Xt[0] + slot;
+        d.X0 = C.X[0] + slot;
     }
     st->d_mats = reinterpret_cast<MatDesc*>(base + o_mats);
     st->d_ptrs = reinterpret_cast<UserPtrs*>(base + o_ptrs);
@@ -284,7 +324,7 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         for (int b = 0; b < 2; ++b) {
             ok &= encode_3d(&C.tmXa[b], C.X[b], C.q, C.p, C.batch, kBM);
             ok &= encode_3d(&C.tmXb[b], C.X[b], C.q, C.p, C.batch, kBN);
-            ok &= encode_3d(&C.tmXtb[b], C.Xt[b], C.p, C.q, C.batch, kBN);
+            ok &= encode_3d(&C.tmXmn[b], C.X[b], C.q, C.p, C.batch, kBK);
         }
         ok &= encode_3d(&C.tmAa, C.A, C.p, C.p, C.batch, kBM);
         ok &= encode_3d(&C.tmAb, C.A, C.p, C.p, C.batch, kBN);
@@ -323,6 +363,7 @@ int bind_pointers(malt_state* st, const malt_param_t* params, cudaStream_t s) {
             const malt_param_t& p = params[off + i];
             bp.p[i] = UserPtrs{p.w, p.g, p.m, p.l, p.r};
         }
+        LaunchScope ls(st, MALT_KIND_BIND, s);
         MALT_CUDA(launch_bind(bp, st->d_ptrs, s), "bind_kernel");
     }
     return MALT_OK;
@@ -358,21 +399,18 @@ int run_gemm_phase(malt_state* st, int phase, int it, int last, const malt_hpara
                 G.M = C.p; G.N = C.p; G.K = C.q;
                 G.ein = nullptr;
                 G.out = C.A;
-                G.outT = nullptr;
             } else if (phase == kPoly) {
                 G.tmA = C.tmAa;
                 G.tmB = C.tmAb;
                 G.M = C.p; G.N = C.p; G.K = C.p;
                 G.ein = C.A;
                 G.out = C.B;
-                G.outT = nullptr;
             } else {
                 G.tmA = C.tmBa;
-                G.tmB = C.tmXtb[cur];
+                G.tmB = C.tmXmn[cur];
                 G.M = C.p; G.N = C.q; G.K = C.p;
-                G.ein = C.X[cur];
+                G.ein = nullptr;
                 G.out = last ? nullptr : C.X[nxt];
-                G.outT = last ? nullptr : C.Xt[nxt];
             }
             G.tiles_m = (G.M + kBM - 1) / kBM;
             G.tiles_n = (G.N + kBN - 1) / kBN;
@@ -392,6 +430,7 @@ int run_gemm_phase(malt_state* st, int phase, int it, int last, const malt_hpara
         P.status = st->d_status;
         P.budget_ns = kWaitBudgetNs;
         const int grid = std::max(1, std::min(tiles, st->num_sms));
+        LaunchScope ls(st, MALT_KIND_NS_GRAM + phase, s);
         MALT_CUDA(launch_ns_gemm(P, grid, s), "ns_gemm_kernel");
     }
     return MALT_OK;
@@ -418,13 +457,25 @@ int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_h
     rc = bind_pointers(st, params, s);
     if (rc != MALT_OK) return rc;
     const int nm = st->nmat;
-    MALT_CUDA(launch_stats(st->d_mats, st->d_ptrs, st->d_pref[0], nm, st->blocks_stats, hp->mu1, s),
-              "stats_kernel");
-    MALT_CUDA(launch_finalize(st->d_mats, st->d_ptrs, st->d_pref[1], nm, st->total_fin, hp->mu2,
-                              hp->eps, st->d_t, s), "finalize_kernel");
-    MALT_CUDA(launch_prescale(st->d_mats, st->d_ptrs, st->d_pref[2], nm, st->blocks_pre, malter, s),
-              "prescale_kernel");
-    MALT_CUDA(launch_norms(st->d_mats, st->d_scal, nm, hp->ns_eps, malter, s), "norms_kernel");
+    {
+        LaunchScope ls(st, MALT_KIND_STATS, s);
+        MALT_CUDA(launch_stats(st->d_mats, st->d_ptrs, st->d_pref[0], nm, st->blocks_stats,
+                               hp->mu1, s), "stats_kernel");
+    }
+    {
+        LaunchScope ls(st, MALT_KIND_FINALIZE, s);
+        MALT_CUDA(launch_finalize(st->d_mats, st->d_ptrs, st->d_pref[1], nm, st->total_fin,
+                                  hp->mu2, hp->eps, st->d_t, s), "finalize_kernel");
+    }
+    {
+        LaunchScope ls(st, MALT_KIND_PRESCALE, s);
+        MALT_CUDA(launch_prescale(st->d_mats, st->d_ptrs, st->d_pref[2], nm, st->blocks_pre,
+                                  malter, s), "prescale_kernel");
+    }
+    {
+        LaunchScope ls(st, MALT_KIND_NORMS, s);
+        MALT_CUDA(launch_norms(st->d_mats, st->d_scal, nm, hp->ns_eps, malter, s), "norms_kernel");
+    }
     for (int it = 0; it < hp->ns_steps; ++it) {
         const int last = it == hp->ns_steps - 1;
         for (int phase = kGram; phase <= kBX; ++phase) {
@@ -443,9 +494,16 @@ int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_h
     sh.ns_c = hp->ns_c;
     sh.ns_eps = hp->ns_eps;
     sh.malter = malter;
-    MALT_CUDA(launch_scalars(st->d_mats, st->d_scal, st->d_t, nm, sh, s), "scalars_kernel");
-    MALT_CUDA(launch_apply(st->d_mats, st->d_ptrs, st->d_scal, st->d_pref[3], nm, st->blocks_apply,
-                           1.f - hp->lr * hp->weight_decay, s), "apply_kernel");
+    {
+        LaunchScope ls(st, MALT_KIND_SCALARS, s);
+        MALT_CUDA(launch_scalars(st->d_mats, st->d_scal, st->d_t, nm, sh, s), "scalars_kernel");
+    }
+    {
+        LaunchScope ls(st, MALT_KIND_APPLY, s);
+        MALT_CUDA(launch_apply(st->d_mats, st->d_ptrs, st->d_scal, st->d_pref[3], nm,
+                               st->blocks_apply, 1.f - hp->lr * hp->weight_decay, s),
+                  "apply_kernel");
+    }
     return MALT_OK;
 }
 
@@ -584,6 +642,36 @@ int malt_debug_wait_timeout(int64_t budget_ns, void* stream) {
     cudaFree(d);
     if (rc != MALT_OK) return rc;
     return h != 0 ? MALT_ERR_TIMEOUT : MALT_OK;
+}
+
+int malt_profile_enable(malt_state_t* st, int32_t enable) {
+    if (st == nullptr) return MALT_ERR_INVALID_ARG;
+    st->profiling = enable != 0;
+    return MALT_OK;
+}
+
+int malt_profile_read(malt_state_t* st, double* ms_out, int64_t* launches_out, int32_t nkinds) {
+    if (st == nullptr || nkinds < 0 || nkinds > MALT_NUM_KINDS ||
+        (nkinds > 0 && (ms_out == nullptr || launches_out == nullptr)))
+        return MALT_ERR_INVALID_ARG;
+    MALT_CUDA(cudaStreamSynchronize(st->last_stream), "cudaStreamSynchronize");
+    for (auto& p : st->ev_pending) {
+        float ms = 0.f;
+        MALT_CUDA(cudaEventElapsedTime(&ms, p.second.first, p.second.second), "cudaEventElapsedTime");
+        st->prof_ms[p.first] += ms;
+        st->ev_pool.push_back(p.second.first);
+        st->ev_pool.push_back(p.second.second);
+    }
+    st->ev_pending.clear();
+    for (int k = 0; k < nkinds; ++k) {
+        ms_out[k] = st->prof_ms[k];
+        launches_out[k] = st->prof_launches[k];
+    }
+    for (int k = 0; k < MALT_NUM_KINDS; ++k) {
+        st->prof_ms[k] = 0.0;
+        st->prof_launches[k] = 0;
+    }
+    return MALT_OK;
 }
 
 size_t malt_workspace_bytes(const malt_state_t* st) { return st == nullptr ? 0 : st->ws_bytes; }

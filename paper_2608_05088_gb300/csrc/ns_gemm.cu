@@ -4,14 +4,16 @@
 //
 // One Newton-Schulz iteration (the Orth step of Algorithm 1, run on the wide
 // orientation X of Mt, p x q) is three launches of this kernel:
-//   kGram  A  = X X^T           (M = N = p, K = q)   operands: rows of X, rows of X
-//   kPoly  B  = b A + c A A     (M = N = p, K = p)   operands: rows of A, rows of A (A = A^T)
-//   kBX    X' = a X + B X       (M = p, N = q, K = p) operands: rows of B, rows of X^T
-// Every operand is read K-major, so X is kept in both orientations: the kBX
-// epilogue writes X' and X'^T.  The 1/(||Mt||_F + ns_eps) normalisation is
-// folded into the first iteration's epilogues (A scaled by k^2, X' by k).  The
-// last iteration's epilogue writes O in W's orientation and per-warp partial
-// sums of O^2 and of D^2 with D = L O R (Algorithm 1, D_t line) for the graft.
+//   kGram  A  = X X^T               (M = N = p, K = q)    operands: rows of X, rows of X
+//   kPoly  B' = a I + b A + c A A   (M = N = p, K = p)    operands: rows of A, rows of A (A = A^T)
+//   kBX    X' = B' X                (M = p, N = q, K = p) operands: rows of B', X read MN-major
+// so a X + (b A + c A A) X = B' X with the a X term folded into B' (its error
+// is that of the bf16 B it rides on).  The kBX B operand is X itself, read as
+// an MN-major [K][N] matrix, so no transposed copy of X is ever written.  The
+// 1/(||Mt||_F + ns_eps) normalisation is folded into the first iteration's
+// epilogues (A scaled by k^2, X' by k).  The last iteration's epilogue writes O
+// in W's orientation and per-warp partial sums of O^2 and of D^2 with
+// D = L O R (Algorithm 1, D_t line) for the graft.
 //
 // Each launch is persistent (one CTA per SM) over a tile list that spans all
 // shape classes and all matrices of each class.  Per CTA: warp 0 issues TMA
@@ -37,6 +39,10 @@ constexpr uint32_t kBBytes = kBN * kBK * 2;
 constexpr uint32_t kStageBytes = kABytes + kBBytes;
 constexpr uint32_t kTmemCols = 2 * kBN;
 constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, kBN);
+constexpr uint32_t kIdescBmn = idesc_bf16_f32(kBM, kBN, true);
+constexpr uint32_t kMnBoxBytes = kBMN * kBK * 2;        // one 64 x 64 MN-major box
+constexpr uint32_t kMnLbo = kMnBoxBytes;                // next 64 MN-elements
+static_assert(kBN % kBMN == 0, "N tile must be whole MN-major boxes");
 constexpr size_t kSmemBytes = static_cast<size_t>(kStages) * kStageBytes + 1024;
 
 static_assert(kBK * 2 == 128, "one K slice must be one 128-byte swizzle row");
@@ -99,6 +105,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint64_t budget = P.budget_ns;
+    const bool b_mn = (P.phase == kBX);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -145,9 +152,22 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                         break;
                     }
                     uint8_t* sa = smem + stage * kStageBytes;
-                    mbar_arrive_expect_tx(&full_bar[stage], kStageBytes);
-                    tma_load_3d(sa, &C.tmA, kb * kBK, t.mt * kBM, t.b, &full_bar[stage]);
-                    tma_load_3d(sa + kABytes, &C.tmB, kb * kBK, t.nt * kBN, t.b, &full_bar[stage]);
+                    if (b_mn) {
+                        // B = X as [K][N]: boxes of 64 N-elements x kBK K-rows.  Boxes
+                        // wholly past N only feed output columns that are never
+                        // stored, so they are not fetched.
+                        const int nbox = min(kBN / kBMN, (C.N - t.nt * kBN + kBMN - 1) / kBMN);
+                        mbar_arrive_expect_tx(&full_bar[stage], kABytes + nbox * kMnBoxBytes);
+                        tma_load_3d(sa, &C.tmA, kb * kBK, t.mt * kBM, t.b, &full_bar[stage]);
+                        for (int j = 0; j < nbox; ++j)
+                            tma_load_3d(sa + kABytes + j * kMnBoxBytes, &C.tmB,
+                                        t.nt * kBN + j * kBMN, kb * kBK, t.b, &full_bar[stage]);
+                    } else {
+                        mbar_arrive_expect_tx(&full_bar[stage], kStageBytes);
+                        tma_load_3d(sa, &C.tmA, kb * kBK, t.mt * kBM, t.b, &full_bar[stage]);
+                        tma_load_3d(sa + kABytes, &C.tmB, kb * kBK, t.nt * kBN, t.b,
+                                    &full_bar[stage]);
+                    }
                     if (++stage == kStages) { stage = 0; phase ^= 1u; }
                 }
                 if (!ok) break;
@@ -179,12 +199,22 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                     tc_fence_after();
                     const uint32_t sa = smem_u32(smem + stage * kStageBytes);
                     const uint64_t da = smem_desc_k_sw128(sa);
-                    const uint64_t db = smem_desc_k_sw128(sa + kABytes);
+                    if (b_mn) {
+                        const uint64_t db = smem_desc_mn_sw128(sa + kABytes, kMnLbo);
 #pragma unroll
-                    for (int kk = 0; kk < kBK / 16; ++kk) {
-                        // +32 bytes along K per 16-element MMA slice (encoded >> 4).
-                        tc_mma_bf16(d_tmem, da + 2 * kk, db + 2 * kk, kIdesc,
-                                    (kb | kk) != 0 ? 1u : 0u);
+                        for (int kk = 0; kk < kBK / 16; ++kk) {
+                            // A: +32 bytes along K; B: +16 K-rows = two 1024-byte atoms.
+                            tc_mma_bf16(d_tmem, da + 2 * kk, db + (2048u >> 4) * kk, kIdescBmn,
+                                        (kb | kk) != 0 ? 1u : 0u);
+                        }
+                    } else {
+                        const uint64_t db = smem_desc_k_sw128(sa + kABytes);
+#pragma unroll
+                        for (int kk = 0; kk < kBK / 16; ++kk) {
+                            // +32 bytes along K per 16-element MMA slice (encoded >> 4).
+                            tc_mma_bf16(d_tmem, da + 2 * kk, db + 2 * kk, kIdesc,
+                                        (kb | kk) != 0 ? 1u : 0u);
+                        }
                     }
                     tc_commit(&empty_bar[stage]);
                     if (++stage == kStages) { stage = 0; phase ^= 1u; }
@@ -219,8 +249,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
             const size_t bs = static_cast<size_t>(M) * N;
             const __nv_bfloat16* ein = C.ein != nullptr ? C.ein + t.b * bs : nullptr;
             __nv_bfloat16* out = C.out != nullptr ? C.out + t.b * bs : nullptr;
-            __nv_bfloat16* outT = C.outT != nullptr ? C.outT + t.b * bs : nullptr;
-            const bool need_ein = (P.phase != kGram);
+            const bool need_ein = (P.phase == kPoly);
             const bool last_bx = (P.phase == kBX) && P.last;
             // NS frame row / column scalings of D = L O R (swapped when transposed).
             const float* uvec = md.trans ? md.R : md.L;
@@ -229,7 +258,8 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
             float sum_o = 0.f, sum_d = 0.f;
 
             const int nch = min(kBN / 32, (N - t.nt * kBN + 31) / 32);
-            uint4 xnext[4];
+            uint4 xnext[4] = {make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u),
+                              make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
             auto load_ein = [&](int ch, uint4 (&dst)[4]) {
                 const int col0 = t.nt * kBN + ch * 32;
 #pragma unroll
@@ -256,17 +286,16 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                     const float sc = kx * kx;
 #pragma unroll
                     for (int j = 0; j < 32; ++j) v[j] *= sc;
-                } else {
+                } else if (P.phase == kPoly) {
                     float x[32];
 #pragma unroll
                     for (int q8 = 0; q8 < 4; ++q8) unpack8(xin[q8], x + 8 * q8);
-                    if (P.phase == kPoly) {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) v[j] = fmaf(P.b, x[j], P.c * v[j]);
-                    } else {
+                    for (int j = 0; j < 32; ++j)
+                        v[j] = fmaf(P.b, x[j], P.c * v[j]) + (col0 + j == row ? P.a : 0.f);
+                } else {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) v[j] = kx * fmaf(P.a, x[j], v[j]);
-                    }
+                    for (int j = 0; j < 32; ++j) v[j] *= kx;
                 }
                 if (!rok) continue;
                 if (!last_bx) {
@@ -275,12 +304,6 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                         if (col0 + q8 * 8 < N)
                             *reinterpret_cast<uint4*>(out + static_cast<size_t>(row) * N + col0 +
                                                       q8 * 8) = pack8(v + 8 * q8);
-                    if (outT != nullptr) {
-#pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if (col0 + j < N)
-                                outT[static_cast<size_t>(col0 + j) * M + row] = __float2bfloat16_rn(v[j]);
-                    }
                 } else {
                     // O in W's orientation, then partial sums of O^2 and D^2.
                     float ob[32];

@@ -5,9 +5,9 @@
 //             every row and every column (eq. dp_preconditioner).
 //   finalize  l, r EMAs from the partials and L = (l+eps)^(-1/8),
 //             R = (r+eps)^(-1/8) (Algorithm 1, L_t / R_t line); bumps t.
-//   prescale  Mt = L M R (Algorithm 1, Mt line), written as bf16 in both
-//             orientations for the Newton-Schulz GEMMs, with partial sums of
-//             Mt^2 (and of (L G R)^2 for MALTER, Algorithm 2 nu_t line).
+//   prescale  Mt = L M R (Algorithm 1, Mt line), written as bf16 in the
+//             Newton-Schulz frame (transposed when m > n), with partial sums
+//             of Mt^2 (and of (L G R)^2 for MALTER, Algorithm 2 nu_t line).
 //   norms     ||Mt||_F and ||L G R||_F^2 per matrix from those partials.
 //   scalars   ||O||_F, ||D||_F, MALTER's nu and alpha (Section 3.5) and the
 //             grafted scale lr * alpha * ||O|| / (||D|| + eps) per matrix.
@@ -228,6 +228,7 @@ prescale_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ p
     const UserPtrs up = ptrs[g];
     const float* __restrict__ Lv = d.L;
     const float* __restrict__ Rv = d.R;
+    const bool trans = d.trans != 0;
 
     float s_mt = 0.f, s_lgr = 0.f;
     const int cc = (t & 15) * 4;
@@ -246,10 +247,12 @@ prescale_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ p
             v0 = Li * mv.x * R4.x; v1 = Li * mv.y * R4.y;
             v2 = Li * mv.z * R4.z; v3 = Li * mv.w * R4.w;
             s_mt += v0 * v0 + v1 * v1 + v2 * v2 + v3 * v3;
-            uint2 pk;
-            *reinterpret_cast<__nv_bfloat162*>(&pk.x) = __floats2bfloat162_rn(v0, v1);
-            *reinterpret_cast<__nv_bfloat162*>(&pk.y) = __floats2bfloat162_rn(v2, v3);
-            *reinterpret_cast<uint2*>(d.Xdir + off) = pk;
+            if (!trans) {
+                uint2 pk;
+                *reinterpret_cast<__nv_bfloat162*>(&pk.x) = __floats2bfloat162_rn(v0, v1);
+                *reinterpret_cast<__nv_bfloat162*>(&pk.y) = __floats2bfloat162_rn(v2, v3);
+                *reinterpret_cast<uint2*>(d.X0 + off) = pk;
+            }
             if (malter) {
                 float gq[4];
                 if (d.g_bf16) {
@@ -272,9 +275,10 @@ prescale_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ p
         tile[rr][cc + 2] = v2; tile[rr][cc + 3] = v3;
     }
     __syncthreads();
-    // Transposed write: output row = column of Mt, 8 consecutive rows of Mt per thread.
+    // NS frame of a tall matrix is Mt^T: output row = column of Mt, 8
+    // consecutive rows of Mt per thread.
 #pragma unroll
-    for (int pass = 0; pass < 2; ++pass) {
+    for (int pass = 0; pass < 2 && trans; ++pass) {
         const int oc = pass * 32 + (t >> 3);
         const int seg = (t & 7) * 8;
         const int gcol = c0 + oc, grow = r0 + seg;
@@ -282,7 +286,7 @@ prescale_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ p
             float v[8];
 #pragma unroll
             for (int j = 0; j < 8; ++j) v[j] = tile[seg + j][oc];
-            *reinterpret_cast<uint4*>(d.Xtrn + static_cast<size_t>(gcol) * m + grow) = pack8_bf16(v);
+            *reinterpret_cast<uint4*>(d.X0 + static_cast<size_t>(gcol) * m + grow) = pack8_bf16(v);
         }
     }
     const float a = block_sum(s_mt, red);

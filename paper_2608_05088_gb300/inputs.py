@@ -100,15 +100,19 @@ def gradient(wl: Workload, idx: int, step: int, scales=None) -> np.ndarray:
 def bf16_representable(x: np.ndarray) -> np.ndarray:
     """Input preparation only: the bf16 value nearest each fp32 entry
     (ties to even), returned as fp32 so the same bits can go anywhere."""
-    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
-    u = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
-    return (u.astype(np.uint32) << 16).view(np.float32)
+    u = np.array(x, dtype=np.float32, copy=True).view(np.uint32)   # finite inputs only
+    lsb = (u >> 16) & np.uint32(1)
+    u += np.uint32(0x7FFF)
+    u += lsb
+    u &= np.uint32(0xFFFF0000)
+    return u.view(np.float32)
 
 
 def initial_weight(wl: Workload, idx: int) -> np.ndarray:
     """W_0 of matrix idx ~ N(0, 0.02^2); bf16-representable for bf16 weights."""
     m, n = wl.shapes[idx]
-    w = (0.02 * _rng(wl.wid, idx, 0, _TAG_WEIGHT).standard_normal((m, n))).astype(np.float32)
+    w = _rng(wl.wid, idx, 0, _TAG_WEIGHT).standard_normal((m, n), dtype=np.float32)
+    w *= np.float32(0.02)
     return bf16_representable(w) if wl.weight_dtype == "bf16" else w
 
 

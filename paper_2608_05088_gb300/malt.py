@@ -29,8 +29,10 @@ SCALARS_PER_MAT = 8
 # Exported entry points declared in include/malt.h.
 EXPORTS = ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
            "malt_set_scalars", "malt_check", "malt_debug_direction", "malt_debug_scalars",
-           "malt_debug_wait_timeout", "malt_workspace_bytes", "malt_status_string",
-           "malt_destroy_state")
+           "malt_debug_wait_timeout", "malt_profile_enable", "malt_profile_read",
+           "malt_workspace_bytes", "malt_status_string", "malt_destroy_state")
+KIND_NAMES = ("bind", "stats", "finalize", "prescale", "norms", "ns_gram", "ns_poly", "ns_bx",
+              "scalars", "apply")
 
 
 class malt_param_t(ctypes.Structure):
@@ -82,6 +84,8 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.malt_debug_direction.argtypes = [vp, i32, vp, vp]
     lib.malt_debug_scalars.argtypes = [vp, P(ctypes.c_float), i32]
     lib.malt_debug_wait_timeout.argtypes = [i64, vp]
+    lib.malt_profile_enable.argtypes = [vp, i32]
+    lib.malt_profile_read.argtypes = [vp, P(ctypes.c_double), P(i64), i32]
     lib.malt_workspace_bytes.argtypes = [vp]
     lib.malt_workspace_bytes.restype = ctypes.c_size_t
     lib.malt_status_string.argtypes = [ctypes.c_int]
@@ -90,7 +94,8 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.malt_destroy_state.restype = None
     for name in ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
                  "malt_set_scalars", "malt_check", "malt_debug_direction",
-                 "malt_debug_scalars", "malt_debug_wait_timeout"):
+                 "malt_debug_scalars", "malt_debug_wait_timeout", "malt_profile_enable",
+                 "malt_profile_read"):
         getattr(lib, name).restype = ctypes.c_int
     _LIB = lib
     return lib
@@ -194,6 +199,19 @@ def malt_debug_wait_timeout(budget_ns: int, stream=None) -> int:
     return load().malt_debug_wait_timeout(int(budget_ns), _stream_handle(stream))
 
 
+def malt_profile_enable(st, enable: bool = True):
+    _check(load().malt_profile_enable(st, 1 if enable else 0), "malt_profile_enable")
+
+
+def malt_profile_read(st):
+    """{kind: (milliseconds, launches)} accumulated since the last read."""
+    n = len(KIND_NAMES)
+    ms = (ctypes.c_double * n)()
+    cnt = (ctypes.c_int64 * n)()
+    _check(load().malt_profile_read(st, ms, cnt, n), "malt_profile_read")
+    return {KIND_NAMES[k]: (float(ms[k]), int(cnt[k])) for k in range(n)}
+
+
 def malt_workspace_bytes(st) -> int:
     return int(load().malt_workspace_bytes(st))
 
@@ -235,6 +253,12 @@ class MaltOptimizer:
         out = torch.empty(W.shape, dtype=torch.bfloat16, device=W.device)
         malt_debug_direction(self.state, idx, out, stream)
         return out
+
+    def profile(self, enable: bool = True):
+        malt_profile_enable(self.state, enable)
+
+    def profile_read(self):
+        return malt_profile_read(self.state)
 
     def workspace_bytes(self) -> int:
         return malt_workspace_bytes(self.state)
