@@ -249,6 +249,8 @@ def run_malt(args):
     from paper_2608_05088_gb300 import build, inputs
     build.build()
     wl = inputs.WORKLOADS[args.workload]
+    if args.layers:
+        wl = inputs.first_layers(wl, args.layers)
     n = len(wl.shapes)
     wdt = torch.bfloat16 if wl.weight_dtype == "bf16" else torch.float32
 
@@ -348,7 +350,7 @@ def run_malt(args):
     elems = wl.elements
     wbytes = 2 if wl.weight_dtype == "bf16" else 4
     mem = {}
-    for kind, bytes_per_elem in (("stats", 12.0), ("prescale", 8.0 + (4.0 if malter else 0.0)),
+    for kind, bytes_per_elem in (("stats", 12.0), ("prescale", 6.0 + (4.0 if malter else 0.0)),
                                  ("apply", 2.0 * wbytes + 2.0)):
         ms = prof[kind][0]
         gbs = bytes_per_elem * elems * args.steps / (ms / 1e3) / 1e9 if ms > 0 else None
@@ -388,6 +390,8 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="profiling only: the first N layers of the workload")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -25,6 +25,7 @@ constexpr int kBN = 256;
 constexpr int kBK = 64;
 constexpr int kStages = 4;
 constexpr int kBMN = 64;           // MN extent of one 128-byte swizzle atom (bf16)
+constexpr int kNsPartsPerTile = 8; // graft partial pairs per GEMM tile (one per epilogue warp)
 constexpr int kMaxClasses = 8;     // shape classes per GEMM launch
 constexpr int kBindChunk = 128;    // parameters per pointer-binding launch
 constexpr int kScalarsPerMat = 8;  // debug scalars per matrix
@@ -57,7 +58,7 @@ struct MatDesc {
     float* L;                // [m]  (l + eps)^(-1/8)
     float* R;                // [n]  (r + eps)^(-1/8)
     float* prepart;          // [pre_tiles][2]  sum Mt^2, sum (L G R)^2
-    float* nspart;           // [ns_tiles][4][2]  per epilogue warp: sum O^2, sum D^2
+    float* nspart;           // [ns_tiles][kNsPartsPerTile][2]: sum O^2, sum D^2
     __nv_bfloat16* X0;       // NS-frame Mt (p x q, bf16): Mt, or Mt^T when trans
     __nv_bfloat16* O;        // [m][n] orthogonalised direction, W's orientation
 };

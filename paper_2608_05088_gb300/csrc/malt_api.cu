@@ -240,7 +240,7 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         o_L[i] = cv.take(sizeof(float) * d.m);
         o_R[i] = cv.take(sizeof(float) * d.n);
         o_pre[i] = cv.take(sizeof(float) * 2 * static_cast<size_t>(d.pre_tr) * d.pre_tc);
-        o_ns[i] = cv.take(sizeof(float) * 8 * static_cast<size_t>(d.ns_tiles));
+        o_ns[i] = cv.take(sizeof(float) * 2 * kNsPartsPerTile * static_cast<size_t>(d.ns_tiles));
         o_O[i] = cv.take(2 * static_cast<size_t>(d.m) * d.n);
     }
     const int nc = static_cast<int>(st->classes.size());

@@ -18,8 +18,9 @@
 // Each launch is persistent (one CTA per SM) over a tile list that spans all
 // shape classes and all matrices of each class.  Per CTA: warp 0 issues TMA
 // loads into a kStages-deep ring, warp 1 issues tcgen05.mma into one of two
-// TMEM accumulators, warps 2-5 drain the other accumulator (tcgen05.ld) and
-// run the epilogue, so the epilogue of tile i overlaps the MMAs of tile i+1.
+// TMEM accumulators, warps 2-9 drain the other accumulator (tcgen05.ld; two
+// warps per 32-lane quarter, each taking half the columns) and run the
+// epilogue, so the epilogue of tile i overlaps the MMAs of tile i+1.
 // Every wait is bounded; a timeout sets the status word and the CTA winds down.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -33,7 +34,10 @@ namespace malt {
 
 namespace {
 
-constexpr int kThreads = 192;
+constexpr int kEpiWarps = kNsPartsPerTile;           // two per TMEM lane quarter
+constexpr int kThreads = 64 + 32 * kEpiWarps;
+constexpr int kEpiCols = kBN / (kEpiWarps / 4);        // accumulator columns per warp
+constexpr int kEpiChunks = kEpiCols / 32;
 constexpr uint32_t kABytes = kBM * kBK * 2;
 constexpr uint32_t kBBytes = kBN * kBK * 2;
 constexpr uint32_t kStageBytes = kABytes + kBBytes;
@@ -114,7 +118,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull_bar[a], 1);
-            mbar_init(&tempty_bar[a], 128);
+            mbar_init(&tempty_bar[a], 32 * kEpiWarps);
         }
         mbar_init(&drain_bar, 1);
         abort_sh = 0;
@@ -228,8 +232,9 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
         }
     } else {
         // -------------------------------------------------------- epilogue
-        const int ew = warp - 2;          // epilogue warp 0..3
-        const int quarter = warp & 3;     // TMEM lanes this warp may read
+        const int ew = warp - 2;                  // epilogue warp 0..kEpiWarps-1
+        const int quarter = warp & 3;             // TMEM lanes this warp may read
+        const int colw = (ew >> 2) * kEpiCols;    // first accumulator column of this warp
         int it = 0;
         for (int tile = blockIdx.x; tile < P.total_tiles; tile += gridDim.x, ++it) {
             const Tile t = decode_tile(P, tile);
@@ -257,11 +262,12 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
             const float urow = (last_bx && rok) ? uvec[row] : 0.f;
             float sum_o = 0.f, sum_d = 0.f;
 
-            const int nch = min(kBN / 32, (N - t.nt * kBN + 31) / 32);
-            uint4 xnext[4] = {make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u),
-                              make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
+            const int col_base = t.nt * kBN + colw;     // first output column of this warp
+            const int nch = max(0, min(kEpiChunks, (N - col_base + 31) / 32));
+            const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                                   acc * kBN + colw;
             auto load_ein = [&](int ch, uint4 (&dst)[4]) {
-                const int col0 = t.nt * kBN + ch * 32;
+                const int col0 = col_base + ch * 32;
 #pragma unroll
                 for (int q8 = 0; q8 < 4; ++q8) {
                     if (rok && col0 + q8 * 8 < N)
@@ -271,17 +277,26 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                         dst[q8] = make_uint4(0u, 0u, 0u, 0u);
                 }
             };
-            if (need_ein) load_ein(0, xnext);
-
-            for (int ch = 0; ch < nch; ++ch) {
-                const int col0 = t.nt * kBN + ch * 32;
-                uint4 xin[4];
+            uint4 xin[2][4];
+            uint32_t rv[2][32];
+            if (nch > 0) {
+                if (need_ein) load_ein(0, xin[0]);
+                tmem_ld_issue(tbase, rv[0]);
+                tmem_ld_wait(rv[0]);
+            }
 #pragma unroll
-                for (int q8 = 0; q8 < 4; ++q8) xin[q8] = xnext[q8];
-                if (need_ein && ch + 1 < nch) load_ein(ch + 1, xnext);
+            for (int ch = 0; ch < kEpiChunks; ++ch) {
+                if (ch >= nch) break;
+                const int cur = ch & 1;
+                // Keep the next chunk's TMEM load (and epilogue input) in flight.
+                if (ch + 1 < nch) {
+                    if (need_ein) load_ein(ch + 1, xin[cur ^ 1]);
+                    tmem_ld_issue(tbase + (ch + 1) * 32, rv[cur ^ 1]);
+                }
+                const int col0 = col_base + ch * 32;
                 float v[32];
-                tmem_ld_32cols(tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
-                                   acc * kBN + ch * 32, v);
+#pragma unroll
+                for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(rv[cur][j]);
                 if (P.phase == kGram) {
                     const float sc = kx * kx;
 #pragma unroll
@@ -289,7 +304,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                 } else if (P.phase == kPoly) {
                     float x[32];
 #pragma unroll
-                    for (int q8 = 0; q8 < 4; ++q8) unpack8(xin[q8], x + 8 * q8);
+                    for (int q8 = 0; q8 < 4; ++q8) unpack8(xin[cur][q8], x + 8 * q8);
 #pragma unroll
                     for (int j = 0; j < 32; ++j)
                         v[j] = fmaf(P.b, x[j], P.c * v[j]) + (col0 + j == row ? P.a : 0.f);
@@ -297,40 +312,40 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
 #pragma unroll
                     for (int j = 0; j < 32; ++j) v[j] *= kx;
                 }
-                if (!rok) continue;
-                if (!last_bx) {
-#pragma unroll
-                    for (int q8 = 0; q8 < 4; ++q8)
-                        if (col0 + q8 * 8 < N)
-                            *reinterpret_cast<uint4*>(out + static_cast<size_t>(row) * N + col0 +
-                                                      q8 * 8) = pack8(v + 8 * q8);
-                } else {
-                    // O in W's orientation, then partial sums of O^2 and D^2.
-                    float ob[32];
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) ob[j] = __bfloat162float(__float2bfloat16_rn(v[j]));
-                    if (!md.trans) {
+                if (rok) {
+                    if (!last_bx) {
 #pragma unroll
                         for (int q8 = 0; q8 < 4; ++q8)
                             if (col0 + q8 * 8 < N)
-                                *reinterpret_cast<uint4*>(md.O + static_cast<size_t>(row) * N + col0 +
-                                                          q8 * 8) = pack8(v + 8 * q8);
+                                *reinterpret_cast<uint4*>(out + static_cast<size_t>(row) * N +
+                                                          col0 + q8 * 8) = pack8(v + 8 * q8);
                     } else {
+                        // O in W's orientation, then partial sums of O^2 and D^2.
+                        if (!md.trans) {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if (col0 + j < N)
-                                md.O[static_cast<size_t>(col0 + j) * M + row] = __float2bfloat16_rn(v[j]);
-                    }
+                            for (int q8 = 0; q8 < 4; ++q8)
+                                if (col0 + q8 * 8 < N)
+                                    *reinterpret_cast<uint4*>(md.O + static_cast<size_t>(row) * N +
+                                                              col0 + q8 * 8) = pack8(v + 8 * q8);
+                        } else {
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        if (col0 + j < N) {
-                            const float o = ob[j];
-                            const float dv = urow * o * vvec[col0 + j];
-                            sum_o = fmaf(o, o, sum_o);
-                            sum_d = fmaf(dv, dv, sum_d);
+                            for (int j = 0; j < 32; ++j)
+                                if (col0 + j < N)
+                                    md.O[static_cast<size_t>(col0 + j) * M + row] =
+                                        __float2bfloat16_rn(v[j]);
+                        }
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) {
+                            if (col0 + j < N) {
+                                const float o = __bfloat162float(__float2bfloat16_rn(v[j]));
+                                const float dv = urow * o * vvec[col0 + j];
+                                sum_o = fmaf(o, o, sum_o);
+                                sum_d = fmaf(dv, dv, sum_d);
+                            }
                         }
                     }
                 }
+                if (ch + 1 < nch) tmem_ld_wait(rv[cur ^ 1]);
             }
             tc_fence_before();
             mbar_arrive(&tempty_bar[acc]);
@@ -341,7 +356,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                     sum_d += __shfl_xor_sync(0xffffffffu, sum_d, o);
                 }
                 if (lane == 0) {
-                    float* dst = md.nspart + (static_cast<size_t>(t.local) * 4 + ew) * 2;
+                    float* dst = md.nspart + (static_cast<size_t>(t.local) * kEpiWarps + ew) * 2;
                     dst[0] = sum_o;
                     dst[1] = sum_d;
                 }

@@ -328,8 +328,8 @@ scalars_kernel(const MatDesc* __restrict__ mats, MatScalars* __restrict__ scal,
     const int g = blockIdx.x;
     const MatDesc& d = mats[g];
     float a = 0.f, b = 0.f;
-    // Four partials (one per epilogue warp) per GEMM tile of the last iteration.
-    for (int i = threadIdx.x; i < 4 * d.ns_tiles; i += blockDim.x) {
+    // One partial per epilogue warp per GEMM tile of the last iteration.
+    for (int i = threadIdx.x; i < kNsPartsPerTile * d.ns_tiles; i += blockDim.x) {
         a += d.nspart[2 * i];
         b += d.nspart[2 * i + 1];
     }

@@ -67,6 +67,13 @@ WORKLOADS = {
 }
 
 
+def first_layers(wl: Workload, layers: int, per_layer: int = 4) -> Workload:
+    """The first `layers` layers of a GPT-2 workload: same shapes, same seeds,
+    so matrix i draws the same inputs as in the full set."""
+    return dataclasses.replace(wl, name=f"{wl.name}_first{layers}l",
+                               shapes=wl.shapes[: layers * per_layer])
+
+
 def stress_workload(rows: int, cols: int, sigma: float, ns_steps: int) -> Workload:
     """One large matrix in bf16 with fp32 state, 3 MALT steps (stress sweep)."""
     wid = 5_000 + int(sigma * 10) * 10 + ns_steps
