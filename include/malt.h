@@ -172,6 +172,34 @@ int malt_debug_wait_timeout(int64_t budget_ns, void* stream);
 int malt_profile_enable(malt_state_t* st, int32_t enable);
 int malt_profile_read(malt_state_t* st, double* ms_out, int64_t* launches_out, int32_t nkinds);
 
+/* Statistics stage of ONE matrix without any device allocation.
+ * The paper has no counterpart: this exists for callers that cannot allocate
+ * device memory when they need the work done -- code inside a CUDA stream
+ * capture, code that must not trigger the device synchronisation an
+ * allocation may cause, code whose framework allocator owns all device
+ * memory.  It runs the momentum and statistics updates and writes the two
+ * diagonal preconditioners, exactly as a MALT step does for that matrix:
+ *   m <- mu1 m + (1 - mu1) g;  l, r <- EMAs of the row / column sums of g^2;
+ *   L_out = (l + eps)^(-1/8) (rows floats), R_out = (r + eps)^(-1/8) (cols floats).
+ * All pointers are caller-owned device buffers laid out as in malt_param_t
+ * (g rows x cols in g_dtype, m rows x cols fp32, l and L_out rows fp32, r and
+ * R_out cols fp32), 16-byte aligned; rows and cols positive multiples of 8.
+ * Its scratch (per-tile partial sums) lives in a fixed array inside the
+ * library, MALT_NOALLOC_SCRATCH_FLOATS floats (4 MiB) on every GPU that loads
+ * the library, held until the process exits.  A matrix that needs more --
+ * ceil(cols/256)*rows rounded up to 64, plus ceil(rows/64)*cols floats -- is
+ * rejected with MALT_ERR_UNSUPPORTED (and a message on stderr).
+ * The first call on a device looks up the array's device address (with that
+ * device current), so make that first call before any stream capture.  All
+ * calls share the one array: calls that overlap on the GPU (other streams,
+ * other threads) race and must be serialised by the caller.  Nothing in the
+ * array needs to start at zero; every partial sum is written before it is
+ * read.  Enqueued on `stream`; does not synchronise. */
+#define MALT_NOALLOC_SCRATCH_FLOATS 1048576
+int malt_stats_noalloc(const void* g, int32_t g_dtype, float* m, float* l, float* r,
+                       float* L_out, float* R_out, int64_t rows, int64_t cols,
+                       float mu1, float mu2, float eps, void* stream);
+
 /* Bytes of device workspace the state holds. */
 size_t malt_workspace_bytes(const malt_state_t* st);
 

@@ -30,7 +30,9 @@ SCALARS_PER_MAT = 8
 EXPORTS = ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
            "malt_set_scalars", "malt_check", "malt_debug_direction", "malt_debug_scalars",
            "malt_debug_wait_timeout", "malt_profile_enable", "malt_profile_read",
-           "malt_workspace_bytes", "malt_status_string", "malt_destroy_state")
+           "malt_workspace_bytes", "malt_status_string", "malt_destroy_state",
+           "malt_stats_noalloc")
+NOALLOC_SCRATCH_FLOATS = 1048576
 KIND_NAMES = ("bind", "stats", "finalize", "prescale", "norms", "ns_gram", "ns_poly", "ns_bx",
               "scalars", "apply")
 
@@ -92,6 +94,9 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.malt_status_string.restype = ctypes.c_char_p
     lib.malt_destroy_state.argtypes = [vp]
     lib.malt_destroy_state.restype = None
+    f32 = ctypes.c_float
+    lib.malt_stats_noalloc.argtypes = [vp, i32, vp, vp, vp, vp, vp, i64, i64, f32, f32, f32, vp]
+    lib.malt_stats_noalloc.restype = ctypes.c_int
     for name in ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
                  "malt_set_scalars", "malt_check", "malt_debug_direction",
                  "malt_debug_scalars", "malt_debug_wait_timeout", "malt_profile_enable",
@@ -210,6 +215,18 @@ def malt_profile_read(st):
     cnt = (ctypes.c_int64 * n)()
     _check(load().malt_profile_read(st, ms, cnt, n), "malt_profile_read")
     return {KIND_NAMES[k]: (float(ms[k]), int(cnt[k])) for k in range(n)}
+
+
+def malt_stats_noalloc(G, M, l, r, L_out, R_out, mu1=0.95, mu2=0.99, eps=1e-8, stream=None) -> int:
+    """Statistics stage of one matrix with no device allocation (see
+    include/malt.h).  Returns the status code; it does not raise, so callers
+    can see MALT_ERR_UNSUPPORTED for matrices past the scratch limit."""
+    rows, cols = M.shape
+    return load().malt_stats_noalloc(
+        ctypes.c_void_p(G.data_ptr()), _dtype_code(G), ctypes.c_void_p(M.data_ptr()),
+        ctypes.c_void_p(l.data_ptr()), ctypes.c_void_p(r.data_ptr()),
+        ctypes.c_void_p(L_out.data_ptr()), ctypes.c_void_p(R_out.data_ptr()),
+        rows, cols, mu1, mu2, eps, _stream_handle(stream))
 
 
 def malt_workspace_bytes(st) -> int:
