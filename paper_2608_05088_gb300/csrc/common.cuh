@@ -19,13 +19,17 @@ constexpr int kStatCols = 256;
 constexpr int kPreTile = 64;
 // Apply kernel: elements per block.
 constexpr int kApplyElems = 4096;
-// Newton-Schulz GEMM tile: BM x BN output, BK reduction slice (one 128-byte row).
+// Newton-Schulz GEMM: a CTA pair computes a kTileM x kBN output tile; each CTA
+// owns kBM rows of it, loads kBM rows of A and kBN/2 rows (N) of B per kBK
+// reduction slice (one 128-byte swizzle row of bf16).
 constexpr int kBM = 128;
+constexpr int kTileM = 2 * kBM;
 constexpr int kBN = 256;
 constexpr int kBK = 64;
-constexpr int kStages = 4;
-constexpr int kBMN = 64;           // MN extent of one 128-byte swizzle atom (bf16)
-constexpr int kNsPartsPerTile = 8; // graft partial pairs per GEMM tile (one per epilogue warp)
+constexpr int kStages = 6;
+constexpr int kBMN = 64;            // MN extent of one 128-byte swizzle atom (bf16)
+constexpr int kEpiWarpsPerCta = 8;  // two per TMEM lane quarter
+constexpr int kNsPartsPerTile = 2 * kEpiWarpsPerCta;  // graft partial pairs per tile
 constexpr int kMaxClasses = 8;     // shape classes per GEMM launch
 constexpr int kBindChunk = 128;    // parameters per pointer-binding launch
 constexpr int kScalarsPerMat = 8;  // debug scalars per matrix
@@ -83,7 +87,7 @@ enum GemmPhase : int32_t { kGram = 0, kPoly = 1, kBX = 2 };
 
 struct GemmClass {  // 64-byte aligned through its CUtensorMap members
     CUtensorMap tmA;              // operand A: rows of a K-major matrix (box kBK x kBM)
-    CUtensorMap tmB;              // operand B: K-major rows (box kBK x kBN), or for kBX
+    CUtensorMap tmB;              // operand B: K-major rows (box kBK x kBM), or for kBX
                                   // an MN-major [K][N] matrix (box kBMN x kBK)
     int32_t M, N, K;              // per-matrix product shape
     int32_t batch;

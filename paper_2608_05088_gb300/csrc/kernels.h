@@ -30,8 +30,10 @@ cudaError_t launch_apply(const MatDesc* mats, const UserPtrs* ptrs, const MatSca
                          cudaStream_t s);
 cudaError_t launch_wait_probe(int32_t* status, uint64_t budget_ns, cudaStream_t s);
 
-// Newton-Schulz GEMM phase over up to kMaxClasses shape classes.
-cudaError_t launch_ns_gemm(const GemmParams& P, int grid, cudaStream_t s);
+// Newton-Schulz GEMM phase over up to kMaxClasses shape classes, on
+// grid_pairs CTA pairs (clusters of two).
+cudaError_t launch_ns_gemm(const GemmParams& P, int grid_pairs, cudaStream_t s);
 size_t ns_gemm_smem_bytes();
+int ns_gemm_max_pairs();
 
 }  // namespace malt

@@ -65,7 +65,7 @@ struct ShapeClass {
     __nv_bfloat16* X[2] = {nullptr, nullptr};   // ping-pong NS iterates [batch][p][q]
     __nv_bfloat16* A = nullptr;                  // X X^T        [batch][p][p]
     __nv_bfloat16* B = nullptr;                  // aI + bA + cA^2 [batch][p][p]
-    CUtensorMap tmXa[2], tmXb[2], tmXmn[2], tmAa, tmAb, tmBa;
+    CUtensorMap tmX[2], tmXmn[2], tmA, tmB;    // 128-row K-major boxes; 64x64 MN boxes
 };
 
 struct Carver {
@@ -227,7 +227,7 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         d.stat_cb = (c + kStatCols - 1) / kStatCols;
         d.pre_tr = (m + kPreTile - 1) / kPreTile;
         d.pre_tc = (c + kPreTile - 1) / kPreTile;
-        d.ns_tiles = ((p + kBM - 1) / kBM) * ((q + kBN - 1) / kBN);
+        d.ns_tiles = ((p + kTileM - 1) / kTileM) * ((q + kBN - 1) / kBN);
     }
 
     // Workspace layout.
@@ -322,13 +322,11 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         ShapeClass& C = st->classes[k];
         bool ok = true;
         for (int b = 0; b < 2; ++b) {
-            ok &= encode_3d(&C.tmXa[b], C.X[b], C.q, C.p, C.batch, kBM);
-            ok &= encode_3d(&C.tmXb[b], C.X[b], C.q, C.p, C.batch, kBN);
+            ok &= encode_3d(&C.tmX[b], C.X[b], C.q, C.p, C.batch, kBM);
             ok &= encode_3d(&C.tmXmn[b], C.X[b], C.q, C.p, C.batch, kBK);
         }
-        ok &= encode_3d(&C.tmAa, C.A, C.p, C.p, C.batch, kBM);
-        ok &= encode_3d(&C.tmAb, C.A, C.p, C.p, C.batch, kBN);
-        ok &= encode_3d(&C.tmBa, C.B, C.p, C.p, C.batch, kBM);
+        ok &= encode_3d(&C.tmA, C.A, C.p, C.p, C.batch, kBM);
+        ok &= encode_3d(&C.tmB, C.B, C.p, C.p, C.batch, kBM);
         if (!ok) {
             std::fprintf(stderr, "malt: cuTensorMapEncodeTiled failed for class %d x %d\n", C.p, C.q);
             return MALT_ERR_CUDA;
@@ -394,25 +392,25 @@ int run_gemm_phase(malt_state* st, int phase, int it, int last, const malt_hpara
             G.batch = C.batch;
             G.mat_of = C.d_mat_of;
             if (phase == kGram) {
-                G.tmA = C.tmXa[cur];
-                G.tmB = C.tmXb[cur];
+                G.tmA = C.tmX[cur];
+                G.tmB = C.tmX[cur];
                 G.M = C.p; G.N = C.p; G.K = C.q;
                 G.ein = nullptr;
                 G.out = C.A;
             } else if (phase == kPoly) {
-                G.tmA = C.tmAa;
-                G.tmB = C.tmAb;
+                G.tmA = C.tmA;
+                G.tmB = C.tmA;
                 G.M = C.p; G.N = C.p; G.K = C.p;
                 G.ein = C.A;
                 G.out = C.B;
             } else {
-                G.tmA = C.tmBa;
+                G.tmA = C.tmB;
                 G.tmB = C.tmXmn[cur];
                 G.M = C.p; G.N = C.q; G.K = C.p;
                 G.ein = nullptr;
                 G.out = last ? nullptr : C.X[nxt];
             }
-            G.tiles_m = (G.M + kBM - 1) / kBM;
+            G.tiles_m = (G.M + kTileM - 1) / kTileM;
             G.tiles_n = (G.N + kBN - 1) / kBN;
             G.tile_begin = tiles;
             tiles += G.tiles_m * G.tiles_n * G.batch;
@@ -429,9 +427,9 @@ int run_gemm_phase(malt_state* st, int phase, int it, int last, const malt_hpara
         P.scal = st->d_scal;
         P.status = st->d_status;
         P.budget_ns = kWaitBudgetNs;
-        const int grid = std::max(1, std::min(tiles, st->num_sms));
+        const int pairs = std::max(1, std::min(tiles, ns_gemm_max_pairs()));
         LaunchScope ls(st, MALT_KIND_NS_GRAM + phase, s);
-        MALT_CUDA(launch_ns_gemm(P, grid, s), "ns_gemm_kernel");
+        MALT_CUDA(launch_ns_gemm(P, pairs, s), "ns_gemm_kernel");
     }
     return MALT_OK;
 }

@@ -1,6 +1,7 @@
 // ns_gemm.cu -- the Newton-Schulz engine: batched same-shape bf16 GEMMs on the
-// sm_103a tensor cores (tcgen05.mma, fp32 accumulators in TMEM, operands
-// staged into shared memory by TMA with 128-byte swizzle).
+// sm_103a tensor cores, two SMs per tile (tcgen05.mma.cta_group::2, fp32
+// accumulators in TMEM, operands staged into shared memory by TMA with
+// 128-byte swizzle).
 //
 // One Newton-Schulz iteration (the Orth step of Algorithm 1, run on the wide
 // orientation X of Mt, p x q) is three launches of this kernel:
@@ -15,16 +16,27 @@
 // in W's orientation and per-warp partial sums of O^2 and of D^2 with
 // D = L O R (Algorithm 1, D_t line) for the graft.
 //
-// Each launch is persistent (one CTA per SM) over a tile list that spans all
-// shape classes and all matrices of each class.  Per CTA: warp 0 issues TMA
-// loads into a kStages-deep ring, warp 1 issues tcgen05.mma into one of two
-// TMEM accumulators, warps 2-9 drain the other accumulator (tcgen05.ld; two
-// warps per 32-lane quarter, each taking half the columns) and run the
-// epilogue, so the epilogue of tile i overlaps the MMAs of tile i+1.
-// Every wait is bounded; a timeout sets the status word and the CTA winds down.
+// Work split.  A cluster of two CTAs (a CTA pair on two SMs) computes one
+// 256 x 256 output tile per turn: CTA r owns rows [128 r, 128 r + 128) of the
+// tile in its own TMEM.  Per 64-wide reduction slice each CTA loads its 128
+// rows of A and its half (128 N-rows or N-columns) of B, 32 KB, into a
+// kStages-deep ring; the MMA, issued by one thread of the even CTA, reads both
+// CTAs' shared memory.  Each SM therefore pulls 32 KB from L2 per
+// 128 x 256 x 64 of MMA work instead of 48 KB, and the 6-stage ring covers
+// half as much again of load latency.
+//
+// Roles per CTA: warp 0 issues TMA loads (the peer's loads complete on the
+// even CTA's full barrier), warp 1 owns TMEM (allocated for the pair) and, in
+// the even CTA, issues tcgen05.mma into one of two TMEM accumulators; warps
+// 2-9 drain the other accumulator (tcgen05.ld, pipelined per 32-column chunk)
+// and run the epilogue, so the epilogue of tile i overlaps the MMAs of tile
+// i+1.  MMA completion is multicast to both CTAs' barriers; both CTAs'
+// epilogue warps release an accumulator on the even CTA's barrier.  Every wait
+// is bounded; a timeout sets the status word and the CTA winds down.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <cstdint>
+#include <cstdio>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -34,23 +46,26 @@ namespace malt {
 
 namespace {
 
-constexpr int kEpiWarps = kNsPartsPerTile;           // two per TMEM lane quarter
+constexpr int kEpiWarps = kEpiWarpsPerCta;
 constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr int kEpiCols = kBN / (kEpiWarps / 4);        // accumulator columns per warp
 constexpr int kEpiChunks = kEpiCols / 32;
-constexpr uint32_t kABytes = kBM * kBK * 2;
-constexpr uint32_t kBBytes = kBN * kBK * 2;
+constexpr int kHalfN = kBN / 2;                        // B rows (or columns) per CTA
+constexpr uint32_t kABytes = kBM * kBK * 2;            // 16 KB
+constexpr uint32_t kBBytes = kHalfN * kBK * 2;         // 16 KB
 constexpr uint32_t kStageBytes = kABytes + kBBytes;
 constexpr uint32_t kTmemCols = 2 * kBN;
-constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, kBN);
-constexpr uint32_t kIdescBmn = idesc_bf16_f32(kBM, kBN, true);
-constexpr uint32_t kMnBoxBytes = kBMN * kBK * 2;        // one 64 x 64 MN-major box
-constexpr uint32_t kMnLbo = kMnBoxBytes;                // next 64 MN-elements
-static_assert(kBN % kBMN == 0, "N tile must be whole MN-major boxes");
+constexpr uint32_t kIdesc = idesc_bf16_f32(kTileM, kBN);
+constexpr uint32_t kIdescBmn = idesc_bf16_f32(kTileM, kBN, true);
+constexpr uint32_t kMnBoxBytes = kBMN * kBK * 2;       // one 64 x 64 MN-major box
+constexpr uint32_t kMnLbo = kMnBoxBytes;               // next 64 MN-elements
 constexpr size_t kSmemBytes = static_cast<size_t>(kStages) * kStageBytes + 1024;
+constexpr uint16_t kPairMask = 0x3;
 
 static_assert(kBK * 2 == 128, "one K slice must be one 128-byte swizzle row");
 static_assert(kTmemCols <= 512, "two accumulators must fit in TMEM");
+static_assert(kHalfN % kBMN == 0, "B half must be whole MN-major boxes");
+static_assert(kEpiWarps == 8, "epilogue layout assumes two warps per lane quarter");
 
 struct Tile {
     int cls, b, mt, nt, local;
@@ -66,6 +81,27 @@ __device__ __forceinline__ Tile decode_tile(const GemmParams& P, int tile) {
     const int rem = local - b * per;
     const int mt = rem / C.tiles_n;
     return Tile{c, b, mt, rem - mt * C.tiles_n, rem};
+}
+
+// Bytes CTA `rank` loads for one reduction slice of tile t.  Boxes that lie
+// wholly past M or N are skipped: they only feed accumulator rows / columns
+// that are never stored.
+__device__ __forceinline__ uint32_t slice_bytes(const GemmClass& C, const Tile& t, int rank,
+                                                bool b_mn, int* nbox_b) {
+    uint32_t bytes = 0;
+    if (t.mt * kTileM + rank * kBM < C.M) bytes += kABytes;
+    const int n0 = t.nt * kBN + rank * kHalfN;
+    int nb = 0;
+    if (b_mn) {
+        for (int j = 0; j < kHalfN / kBMN; ++j)
+            if (n0 + j * kBMN < C.N) ++nb;
+        bytes += nb * kMnBoxBytes;
+    } else if (n0 < C.N) {
+        nb = 1;
+        bytes += kBBytes;
+    }
+    *nbox_b = nb;
+    return bytes;
 }
 
 __device__ __forceinline__ void unpack8(const uint4& u, float* v) {
@@ -93,7 +129,7 @@ __device__ __forceinline__ void raise_timeout(const GemmParams& P, volatile int*
 
 }  // namespace
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 ns_gemm_kernel(const __grid_constant__ GemmParams P) {
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[kStages];
@@ -105,11 +141,16 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
     __shared__ int abort_sh;
     volatile int* abort_flag = &abort_sh;
 
+    // Same offset in both CTAs: the MMA addresses the peer's tiles through
+    // the even CTA's descriptors.
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint64_t budget = P.budget_ns;
     const bool b_mn = (P.phase == kBX);
+    const int rank = static_cast<int>(cluster_ctarank());
+    const bool leader = (rank == 0);
+    const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -118,7 +159,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull_bar[a], 1);
-            mbar_init(&tempty_bar[a], 32 * kEpiWarps);
+            mbar_init(&tempty_bar[a], 2 * kEpiWarps);
         }
         mbar_init(&drain_bar, 1);
         abort_sh = 0;
@@ -132,11 +173,11 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
         }
     }
     if (warp == 1) {
-        tmem_alloc(&tmem_slot, kTmemCols);
-        tmem_relinquish();
+        tmem_alloc_pair(&tmem_slot, kTmemCols);
+        tmem_relinquish_pair();
     }
     tc_fence_before();
-    __syncthreads();
+    cluster_sync();          // both CTAs' barriers initialised, TMEM allocated
     tc_fence_after();
     const uint32_t tmem_base = tmem_slot;
 
@@ -144,33 +185,33 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
         // ---------------------------------------------------- TMA producer
         if (lane == 0) {
             uint32_t stage = 0, phase = 0;
-            for (int tile = blockIdx.x; tile < P.total_tiles; tile += gridDim.x) {
+            for (int tile = pair; tile < P.total_tiles; tile += npairs) {
                 const Tile t = decode_tile(P, tile);
                 const GemmClass& C = P.cls[t.cls];
                 const int nkb = (C.K + kBK - 1) / kBK;
+                int nb_self = 0, nb_peer = 0;
+                const uint32_t bytes_self = slice_bytes(C, t, rank, b_mn, &nb_self);
+                const uint32_t bytes_pair = bytes_self + slice_bytes(C, t, rank ^ 1, b_mn, &nb_peer);
+                const bool load_a = t.mt * kTileM + rank * kBM < C.M;
+                const int a_row = t.mt * kTileM + rank * kBM;
+                const int n0 = t.nt * kBN + rank * kHalfN;
                 bool ok = true;
                 for (int kb = 0; kb < nkb; ++kb) {
-                    if (!mbar_wait_bounded(&empty_bar[stage], phase ^ 1u, budget, abort_flag)) {
+                    if (!mbar_wait_cluster_bounded(&empty_bar[stage], phase ^ 1u, budget, abort_flag)) {
                         raise_timeout(P, abort_flag);
                         ok = false;
                         break;
                     }
                     uint8_t* sa = smem + stage * kStageBytes;
+                    const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
+                    if (leader) mbar_arrive_expect_tx(&full_bar[stage], bytes_pair);
+                    if (load_a) tma_load_3d_pair(sa, &C.tmA, kb * kBK, a_row, t.b, fb);
                     if (b_mn) {
-                        // B = X as [K][N]: boxes of 64 N-elements x kBK K-rows.  Boxes
-                        // wholly past N only feed output columns that are never
-                        // stored, so they are not fetched.
-                        const int nbox = min(kBN / kBMN, (C.N - t.nt * kBN + kBMN - 1) / kBMN);
-                        mbar_arrive_expect_tx(&full_bar[stage], kABytes + nbox * kMnBoxBytes);
-                        tma_load_3d(sa, &C.tmA, kb * kBK, t.mt * kBM, t.b, &full_bar[stage]);
-                        for (int j = 0; j < nbox; ++j)
-                            tma_load_3d(sa + kABytes + j * kMnBoxBytes, &C.tmB,
-                                        t.nt * kBN + j * kBMN, kb * kBK, t.b, &full_bar[stage]);
-                    } else {
-                        mbar_arrive_expect_tx(&full_bar[stage], kStageBytes);
-                        tma_load_3d(sa, &C.tmA, kb * kBK, t.mt * kBM, t.b, &full_bar[stage]);
-                        tma_load_3d(sa + kABytes, &C.tmB, kb * kBK, t.nt * kBN, t.b,
-                                    &full_bar[stage]);
+                        for (int j = 0; j < nb_self; ++j)
+                            tma_load_3d_pair(sa + kABytes + j * kMnBoxBytes, &C.tmB,
+                                             n0 + j * kBMN, kb * kBK, t.b, fb);
+                    } else if (nb_self > 0) {
+                        tma_load_3d_pair(sa + kABytes, &C.tmB, kb * kBK, n0, t.b, fb);
                     }
                     if (++stage == kStages) { stage = 0; phase ^= 1u; }
                 }
@@ -178,16 +219,16 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
             }
         }
     } else if (warp == 1) {
-        // ------------------------------------------------------ MMA issuer
-        if (lane == 0) {
+        // ------------------------------------------- MMA issuer (even CTA)
+        if (lane == 0 && leader) {
             uint32_t stage = 0, phase = 0;
             int it = 0;
-            for (int tile = blockIdx.x; tile < P.total_tiles; tile += gridDim.x, ++it) {
+            for (int tile = pair; tile < P.total_tiles; tile += npairs, ++it) {
                 const Tile t = decode_tile(P, tile);
                 const GemmClass& C = P.cls[t.cls];
                 const int nkb = (C.K + kBK - 1) / kBK;
                 const uint32_t acc = it & 1, acc_phase = (it >> 1) & 1;
-                if (!mbar_wait_bounded(&tempty_bar[acc], acc_phase ^ 1u, budget, abort_flag)) {
+                if (!mbar_wait_cluster_bounded(&tempty_bar[acc], acc_phase ^ 1u, budget, abort_flag)) {
                     raise_timeout(P, abort_flag);
                     break;
                 }
@@ -195,7 +236,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                 const uint32_t d_tmem = tmem_base + acc * kBN;
                 bool ok = true;
                 for (int kb = 0; kb < nkb; ++kb) {
-                    if (!mbar_wait_bounded(&full_bar[stage], phase, budget, abort_flag)) {
+                    if (!mbar_wait_cluster_bounded(&full_bar[stage], phase, budget, abort_flag)) {
                         raise_timeout(P, abort_flag);
                         ok = false;
                         break;
@@ -208,45 +249,47 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
 #pragma unroll
                         for (int kk = 0; kk < kBK / 16; ++kk) {
                             // A: +32 bytes along K; B: +16 K-rows = two 1024-byte atoms.
-                            tc_mma_bf16(d_tmem, da + 2 * kk, db + (2048u >> 4) * kk, kIdescBmn,
-                                        (kb | kk) != 0 ? 1u : 0u);
+                            tc_mma_bf16_pair(d_tmem, da + 2 * kk, db + (2048u >> 4) * kk,
+                                             kIdescBmn, (kb | kk) != 0 ? 1u : 0u);
                         }
                     } else {
                         const uint64_t db = smem_desc_k_sw128(sa + kABytes);
 #pragma unroll
                         for (int kk = 0; kk < kBK / 16; ++kk) {
                             // +32 bytes along K per 16-element MMA slice (encoded >> 4).
-                            tc_mma_bf16(d_tmem, da + 2 * kk, db + 2 * kk, kIdesc,
-                                        (kb | kk) != 0 ? 1u : 0u);
+                            tc_mma_bf16_pair(d_tmem, da + 2 * kk, db + 2 * kk, kIdesc,
+                                             (kb | kk) != 0 ? 1u : 0u);
                         }
                     }
-                    tc_commit(&empty_bar[stage]);
+                    tc_commit_pair_multicast(&empty_bar[stage], kPairMask);
                     if (++stage == kStages) { stage = 0; phase ^= 1u; }
                 }
                 if (!ok) break;
-                tc_commit(&tfull_bar[acc]);
+                tc_commit_pair_multicast(&tfull_bar[acc], kPairMask);
             }
             // Do not release TMEM while MMAs may still be in flight.
-            tc_commit(&drain_bar);
-            if (!mbar_wait_bounded(&drain_bar, 0, budget, nullptr)) raise_timeout(P, abort_flag);
+            tc_commit_pair_multicast(&drain_bar, 0x1);
+            if (!mbar_wait_cluster_bounded(&drain_bar, 0, budget, nullptr)) raise_timeout(P, abort_flag);
         }
     } else {
         // -------------------------------------------------------- epilogue
         const int ew = warp - 2;                  // epilogue warp 0..kEpiWarps-1
         const int quarter = warp & 3;             // TMEM lanes this warp may read
         const int colw = (ew >> 2) * kEpiCols;    // first accumulator column of this warp
+        const uint32_t tempty_leader0 = mapa_shared(smem_u32(&tempty_bar[0]), 0);
+        const uint32_t tempty_leader1 = mapa_shared(smem_u32(&tempty_bar[1]), 0);
         int it = 0;
-        for (int tile = blockIdx.x; tile < P.total_tiles; tile += gridDim.x, ++it) {
+        for (int tile = pair; tile < P.total_tiles; tile += npairs, ++it) {
             const Tile t = decode_tile(P, tile);
             const GemmClass& C = P.cls[t.cls];
             const uint32_t acc = it & 1, acc_phase = (it >> 1) & 1;
-            if (!mbar_wait_bounded(&tfull_bar[acc], acc_phase, budget, abort_flag)) {
+            if (!mbar_wait_cluster_bounded(&tfull_bar[acc], acc_phase, budget, abort_flag)) {
                 raise_timeout(P, abort_flag);
                 break;
             }
             tc_fence_after();
             const int M = C.M, N = C.N;
-            const int row = t.mt * kBM + quarter * 32 + lane;
+            const int row = t.mt * kTileM + rank * kBM + quarter * 32 + lane;
             const bool rok = row < M;
             const int g = C.mat_of[t.b];
             const MatDesc& md = P.mats[g];
@@ -277,10 +320,9 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                         dst[q8] = make_uint4(0u, 0u, 0u, 0u);
                 }
             };
-            uint4 xin[2][4];
+            uint4 xin[4];
             uint32_t rv[2][32];
             if (nch > 0) {
-                if (need_ein) load_ein(0, xin[0]);
                 tmem_ld_issue(tbase, rv[0]);
                 tmem_ld_wait(rv[0]);
             }
@@ -288,11 +330,9 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
             for (int ch = 0; ch < kEpiChunks; ++ch) {
                 if (ch >= nch) break;
                 const int cur = ch & 1;
-                // Keep the next chunk's TMEM load (and epilogue input) in flight.
-                if (ch + 1 < nch) {
-                    if (need_ein) load_ein(ch + 1, xin[cur ^ 1]);
-                    tmem_ld_issue(tbase + (ch + 1) * 32, rv[cur ^ 1]);
-                }
+                if (need_ein) load_ein(ch, xin);
+                // Keep the next chunk's TMEM load in flight.
+                if (ch + 1 < nch) tmem_ld_issue(tbase + (ch + 1) * 32, rv[cur ^ 1]);
                 const int col0 = col_base + ch * 32;
                 float v[32];
 #pragma unroll
@@ -304,7 +344,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                 } else if (P.phase == kPoly) {
                     float x[32];
 #pragma unroll
-                    for (int q8 = 0; q8 < 4; ++q8) unpack8(xin[cur][q8], x + 8 * q8);
+                    for (int q8 = 0; q8 < 4; ++q8) unpack8(xin[q8], x + 8 * q8);
 #pragma unroll
                     for (int j = 0; j < 32; ++j)
                         v[j] = fmaf(P.b, x[j], P.c * v[j]) + (col0 + j == row ? P.a : 0.f);
@@ -348,7 +388,8 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                 if (ch + 1 < nch) tmem_ld_wait(rv[cur ^ 1]);
             }
             tc_fence_before();
-            mbar_arrive(&tempty_bar[acc]);
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(acc ? tempty_leader1 : tempty_leader0);
             if (last_bx) {
 #pragma unroll
                 for (int o = 16; o > 0; o >>= 1) {
@@ -356,7 +397,8 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                     sum_d += __shfl_xor_sync(0xffffffffu, sum_d, o);
                 }
                 if (lane == 0) {
-                    float* dst = md.nspart + (static_cast<size_t>(t.local) * kEpiWarps + ew) * 2;
+                    float* dst = md.nspart + (static_cast<size_t>(t.local) * kNsPartsPerTile +
+                                              rank * kEpiWarps + ew) * 2;
                     dst[0] = sum_o;
                     dst[1] = sum_d;
                 }
@@ -364,17 +406,41 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
         }
     }
 
+    // Neither CTA may leave (or free TMEM) while its pair partner can still
+    // signal its barriers or read its shared memory.
     tc_fence_before();
-    __syncthreads();
+    cluster_sync();
     if (warp == 1) {
         tc_fence_after();
-        tmem_dealloc(tmem_base, kTmemCols);
+        tmem_dealloc_pair(tmem_base, kTmemCols);
     }
 }
 
 size_t ns_gemm_smem_bytes() { return kSmemBytes; }
 
-cudaError_t launch_ns_gemm(const GemmParams& P, int grid, cudaStream_t s) {
+// Number of CTA pairs that can be resident at once (the persistent grid).
+int ns_gemm_max_pairs() {
+    static int cached = -1;
+    if (cached > 0) return cached;
+    int n = 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2, 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    if (cudaFuncSetAttribute(ns_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(kSmemBytes)) != cudaSuccess ||
+        cudaOccupancyMaxActiveClusters(&n, ns_gemm_kernel, &cfg) != cudaSuccess || n <= 0) {
+        cudaGetLastError();
+        int dev = 0, sms = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        n = sms / 2;
+    }
+    cached = n;
+    return cached;
+}
+
+cudaError_t launch_ns_gemm(const GemmParams& P, int grid_pairs, cudaStream_t s) {
     static bool configured = false;
     if (!configured) {
         const cudaError_t e = cudaFuncSetAttribute(
@@ -382,8 +448,20 @@ cudaError_t launch_ns_gemm(const GemmParams& P, int grid, cudaStream_t s) {
         if (e != cudaSuccess) return e;
         configured = true;
     }
-    ns_gemm_kernel<<<grid, kThreads, kSmemBytes, s>>>(P);
-    return cudaGetLastError();
+    ns_gemm_kernel<<<2 * grid_pairs, kThreads, kSmemBytes, s>>>(P);
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) {
+        cudaFuncAttributes fa{};
+        cudaFuncGetAttributes(&fa, ns_gemm_kernel);
+        std::fprintf(stderr,
+                     "malt: ns_gemm_kernel launch (%d CTAs x %d threads, %zu B dynamic smem) "
+                     "refused: %s; kernel uses %d registers, %zu B static smem, allows %d "
+                     "threads and %d B dynamic smem per block\n",
+                     2 * grid_pairs, kThreads, kSmemBytes, cudaGetErrorString(e), fa.numRegs,
+                     fa.sharedSizeBytes, fa.maxThreadsPerBlock, fa.maxDynamicSharedSizeBytes);
+        cudaGetLastError();
+    }
+    return e;
 }
 
 }  // namespace malt
