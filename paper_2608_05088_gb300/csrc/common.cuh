@@ -64,7 +64,7 @@ struct MatDesc {
     float* prepart;          // [pre_tiles][2]  sum Mt^2, sum (L G R)^2
     float* nspart;           // [ns_tiles][kNsPartsPerTile][2]: sum O^2, sum D^2
     __nv_bfloat16* X0;       // NS-frame Mt (p x q, bf16): Mt, or Mt^T when trans
-    __nv_bfloat16* O;        // [m][n] orthogonalised direction, W's orientation
+    __nv_bfloat16* O;        // [p][q] orthogonalised direction in the NS frame
 };
 
 // Per-matrix scalars kept on the device (index = matrix).
@@ -89,6 +89,8 @@ struct GemmClass {  // 64-byte aligned through its CUtensorMap members
     CUtensorMap tmA;              // operand A: rows of a K-major matrix (box kBK x kBM)
     CUtensorMap tmB;              // operand B: K-major rows (box kBK x kBM), or for kBX
                                   // an MN-major [K][N] matrix (box kBMN x kBK)
+    CUtensorMap tmOut;            // output [batch][M][N], store box 32 x 32, 64-byte swizzle
+                                  // (the last kBX stores O)
     int32_t M, N, K;              // per-matrix product shape
     int32_t batch;
     int32_t tiles_m, tiles_n;
@@ -96,7 +98,7 @@ struct GemmClass {  // 64-byte aligned through its CUtensorMap members
     int32_t pad_;
     const int32_t* mat_of;        // [batch] -> matrix index
     const __nv_bfloat16* ein;     // epilogue input (A for kPoly), [batch][M][N]
-    __nv_bfloat16* out;           // output [batch][M][N] (unused by the last kBX)
+
 };
 
 struct GemmParams {

@@ -43,19 +43,25 @@ bool get_encoder() {
     return true;
 }
 
-// 3-D bf16 tensor [batch][rows][cols], box kBK x box_rows x 1, 128-byte swizzle,
-// zero fill outside the tensor.
+// 3-D bf16 tensor [batch][rows][cols], box box_cols x box_rows x 1, zero fill
+// outside the tensor on loads (stores skip the outside).
 bool encode_3d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint64_t batch,
-               uint32_t box_rows) {
+               uint32_t box_rows, uint32_t box_cols = kBK,
+               CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
     const cuuint64_t dims[3] = {cols, rows, batch};
     const cuuint64_t strides[2] = {cols * 2, rows * cols * 2};
-    const cuuint32_t box[3] = {static_cast<cuuint32_t>(kBK), box_rows, 1};
+    const cuuint32_t box[3] = {box_cols, box_rows, 1};
     const cuuint32_t estr[3] = {1, 1, 1};
     const CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base),
                                 dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
+}
+
+// Store map of an epilogue output: 32 x 32 boxes with 64-byte swizzle.
+bool encode_store(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint64_t batch) {
+    return encode_3d(map, base, cols, rows, batch, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
 }
 
 struct ShapeClass {
@@ -65,7 +71,9 @@ struct ShapeClass {
     __nv_bfloat16* X[2] = {nullptr, nullptr};   // ping-pong NS iterates [batch][p][q]
     __nv_bfloat16* A = nullptr;                  // X X^T        [batch][p][p]
     __nv_bfloat16* B = nullptr;                  // aI + bA + cA^2 [batch][p][p]
+    __nv_bfloat16* O = nullptr;                  // last iterate   [batch][p][q]
     CUtensorMap tmX[2], tmXmn[2], tmA, tmB;    // 128-row K-major boxes; 64x64 MN boxes
+    CUtensorMap stX[2], stA, stB, stO;         // epilogue store maps
 };
 
 struct Carver {
@@ -232,7 +240,7 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
 
     // Workspace layout.
     Carver cv;
-    std::vector<size_t> o_row(n), o_col(n), o_L(n), o_R(n), o_pre(n), o_ns(n), o_O(n);
+    std::vector<size_t> o_row(n), o_col(n), o_L(n), o_R(n), o_pre(n), o_ns(n);
     for (int i = 0; i < n; ++i) {
         const MatDesc& d = st->hmats[i];
         o_row[i] = cv.take(sizeof(float) * static_cast<size_t>(d.stat_cb) * d.m);
@@ -241,10 +249,9 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         o_R[i] = cv.take(sizeof(float) * d.n);
         o_pre[i] = cv.take(sizeof(float) * 2 * static_cast<size_t>(d.pre_tr) * d.pre_tc);
         o_ns[i] = cv.take(sizeof(float) * 2 * kNsPartsPerTile * static_cast<size_t>(d.ns_tiles));
-        o_O[i] = cv.take(2 * static_cast<size_t>(d.m) * d.n);
     }
     const int nc = static_cast<int>(st->classes.size());
-    std::vector<size_t> o_X0(nc), o_X1(nc), o_A(nc), o_B(nc), o_matof(nc);
+    std::vector<size_t> o_X0(nc), o_X1(nc), o_A(nc), o_B(nc), o_O(nc), o_matof(nc);
     for (int k = 0; k < nc; ++k) {
         const ShapeClass& C = st->classes[k];
         const size_t pq = static_cast<size_t>(C.batch) * C.p * C.q * 2;
@@ -253,6 +260,7 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         o_X1[k] = cv.take(pq);
         o_A[k] = cv.take(pp);
         o_B[k] = cv.take(pp);
+        o_O[k] = cv.take(pq);
         o_matof[k] = cv.take(sizeof(int32_t) * C.batch);
     }
     const size_t o_mats = cv.take(sizeof(MatDesc) * std::max(n, 1));
@@ -278,6 +286,7 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         C.X[1] = H(o_X1[k]);
         C.A = H(o_A[k]);
         C.B = H(o_B[k]);
+        C.O = H(o_O[k]);
         C.d_mat_of = reinterpret_cast<int32_t*>(base + o_matof[k]);
     }
     for (int i = 0; i < n; ++i) {
@@ -289,9 +298,9 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         d.R = F(o_R[i]);
         d.prepart = F(o_pre[i]);
         d.nspart = F(o_ns[i]);
-        d.O = H(o_O[i]);
         const size_t slot = static_cast<size_t>(d.bidx) * C.p * C.q;
         d.X0 = C.X[0] + slot;
+        d.O = C.O + slot;
     }
     st->d_mats = reinterpret_cast<MatDesc*>(base + o_mats);
     st->d_ptrs = reinterpret_cast<UserPtrs*>(base + o_ptrs);
@@ -309,7 +318,12 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         pref[0][i + 1] = pref[0][i] + d.stat_rb * d.stat_cb;
         pref[1][i + 1] = pref[1][i] + d.m + d.n;
         pref[2][i + 1] = pref[2][i] + d.pre_tr * d.pre_tc;
-        pref[3][i + 1] = pref[3][i] + static_cast<int32_t>((elems + kApplyElems - 1) / kApplyElems);
+        // apply: contiguous runs of kApplyElems, or 64 x 64 tiles for a tall
+        // matrix whose O is read transposed from the NS frame
+        const int32_t apply_blocks =
+            d.trans ? ((d.m + 63) / 64) * ((d.n + 63) / 64)
+                    : static_cast<int32_t>((elems + kApplyElems - 1) / kApplyElems);
+        pref[3][i + 1] = pref[3][i] + apply_blocks;
     }
     st->blocks_stats = pref[0][n];
     st->total_fin = pref[1][n];
@@ -327,6 +341,10 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         }
         ok &= encode_3d(&C.tmA, C.A, C.p, C.p, C.batch, kBM);
         ok &= encode_3d(&C.tmB, C.B, C.p, C.p, C.batch, kBM);
+        for (int b = 0; b < 2; ++b) ok &= encode_store(&C.stX[b], C.X[b], C.q, C.p, C.batch);
+        ok &= encode_store(&C.stA, C.A, C.p, C.p, C.batch);
+        ok &= encode_store(&C.stB, C.B, C.p, C.p, C.batch);
+        ok &= encode_store(&C.stO, C.O, C.q, C.p, C.batch);
         if (!ok) {
             std::fprintf(stderr, "malt: cuTensorMapEncodeTiled failed for class %d x %d\n", C.p, C.q);
             return MALT_ERR_CUDA;
@@ -396,24 +414,26 @@ int run_gemm_phase(malt_state* st, int phase, int it, int last, const malt_hpara
                 G.tmB = C.tmX[cur];
                 G.M = C.p; G.N = C.p; G.K = C.q;
                 G.ein = nullptr;
-                G.out = C.A;
+                G.tmOut = C.stA;
             } else if (phase == kPoly) {
                 G.tmA = C.tmA;
                 G.tmB = C.tmA;
                 G.M = C.p; G.N = C.p; G.K = C.p;
                 G.ein = C.A;
-                G.out = C.B;
+                G.tmOut = C.stB;
             } else {
                 G.tmA = C.tmB;
                 G.tmB = C.tmXmn[cur];
                 G.M = C.p; G.N = C.q; G.K = C.p;
                 G.ein = nullptr;
-                G.out = last ? nullptr : C.X[nxt];
+                G.tmOut = last ? C.stO : C.stX[nxt];
             }
             G.tiles_m = (G.M + kTileM - 1) / kTileM;
             G.tiles_n = (G.N + kBN - 1) / kBN;
             G.tile_begin = tiles;
-            tiles += G.tiles_m * G.tiles_n * G.batch;
+            // Gram and Poly products are symmetric: upper-triangle tiles only.
+            const int per = phase == kBX ? G.tiles_m * G.tiles_n : G.tiles_m * (G.tiles_m + 1) / 2;
+            tiles += per * G.batch;
         }
         P.nclasses = static_cast<int32_t>(cnt);
         P.total_tiles = tiles;
@@ -600,9 +620,15 @@ int malt_set_scalars(malt_state_t* st, const float* nu_host, int32_t n, int64_t 
 int malt_debug_direction(malt_state_t* st, int32_t idx, void* out, void* stream) {
     if (st == nullptr || idx < 0 || idx >= st->nmat || out == nullptr) return MALT_ERR_INVALID_ARG;
     const MatDesc& d = st->hmats[idx];
-    MALT_CUDA(cudaMemcpyAsync(out, d.O, static_cast<size_t>(d.m) * d.n * 2, cudaMemcpyDeviceToDevice,
-                              static_cast<cudaStream_t>(stream)),
-              "cudaMemcpyAsync(O)");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (d.trans) {
+        // O is kept in the NS frame (n x m) for a tall matrix: transpose on the way out.
+        MALT_CUDA(launch_transpose_bf16(d.O, static_cast<__nv_bfloat16*>(out), d.n, d.m, s),
+                  "transpose_bf16_kernel");
+    } else {
+        MALT_CUDA(cudaMemcpyAsync(out, d.O, static_cast<size_t>(d.m) * d.n * 2,
+                                  cudaMemcpyDeviceToDevice, s), "cudaMemcpyAsync(O)");
+    }
     return MALT_OK;
 }
 

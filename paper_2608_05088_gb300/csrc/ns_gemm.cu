@@ -7,6 +7,9 @@
 // orientation X of Mt, p x q) is three launches of this kernel:
 //   kGram  A  = X X^T               (M = N = p, K = q)    operands: rows of X, rows of X
 //   kPoly  B' = a I + b A + c A A   (M = N = p, K = p)    operands: rows of A, rows of A (A = A^T)
+// A and B' are symmetric, so those two phases compute only the tiles on and
+// above the diagonal and store each off-diagonal tile twice (as is and
+// transposed); the products are then exactly symmetric.
 //   kBX    X' = B' X                (M = p, N = q, K = p) operands: rows of B', X read MN-major
 // so a X + (b A + c A A) X = B' X with the a X term folded into B' (its error
 // is that of the bf16 B it rides on).  The kBX B operand is X itself, read as
@@ -14,7 +17,8 @@
 // 1/(||Mt||_F + ns_eps) normalisation is folded into the first iteration's
 // epilogues (A scaled by k^2, X' by k).  The last iteration's epilogue writes O
 // in W's orientation and per-warp partial sums of O^2 and of D^2 with
-// D = L O R (Algorithm 1, D_t line) for the graft.
+// D = L O R (Algorithm 1, D_t line) for the graft; O stays in the NS frame
+// (the apply pass reads a tall matrix's O transposed).
 //
 // Work split.  A cluster of two CTAs (a CTA pair on two SMs) computes one
 // 256 x 256 output tile per turn: CTA r owns rows [128 r, 128 r + 128) of the
@@ -30,7 +34,9 @@
 // the even CTA, issues tcgen05.mma into one of two TMEM accumulators; warps
 // 2-9 drain the other accumulator (tcgen05.ld, pipelined per 32-column chunk)
 // and run the epilogue, so the epilogue of tile i overlaps the MMAs of tile
-// i+1.  MMA completion is multicast to both CTAs' barriers; both CTAs'
+// i+1.  Each epilogue warp converts its 32 x 32 chunk to bf16 in a
+// double-buffered shared-memory box (64-byte swizzle, bank-conflict free) and
+// writes it with one TMA bulk tensor store.  MMA completion is multicast to both CTAs' barriers; both CTAs'
 // epilogue warps release an accumulator on the even CTA's barrier.  Every wait
 // is bounded; a timeout sets the status word and the CTA winds down.
 #include <cuda_bf16.h>
@@ -59,28 +65,46 @@ constexpr uint32_t kIdesc = idesc_bf16_f32(kTileM, kBN);
 constexpr uint32_t kIdescBmn = idesc_bf16_f32(kTileM, kBN, true);
 constexpr uint32_t kMnBoxBytes = kBMN * kBK * 2;       // one 64 x 64 MN-major box
 constexpr uint32_t kMnLbo = kMnBoxBytes;               // next 64 MN-elements
-constexpr size_t kSmemBytes = static_cast<size_t>(kStages) * kStageBytes + 1024;
+constexpr uint32_t kStoreBoxBytes = 32 * 32 * 2;      // one 32 x 32 bf16 output box
+constexpr uint32_t kStageOutBytes = 2 * kStoreBoxBytes * kEpiWarps;  // double-buffered per warp
+constexpr size_t kSmemBytes =
+    static_cast<size_t>(kStages) * kStageBytes + kStageOutBytes + 1024;
 constexpr uint16_t kPairMask = 0x3;
 
 static_assert(kBK * 2 == 128, "one K slice must be one 128-byte swizzle row");
 static_assert(kTmemCols <= 512, "two accumulators must fit in TMEM");
 static_assert(kHalfN % kBMN == 0, "B half must be whole MN-major boxes");
 static_assert(kEpiWarps == 8, "epilogue layout assumes two warps per lane quarter");
+static_assert(kTileM == kBN, "symmetric products need square tiles");
 
 struct Tile {
     int cls, b, mt, nt, local;
 };
 
-__device__ __forceinline__ Tile decode_tile(const GemmParams& P, int tile) {
+// Tiles of one matrix: all tiles_m x tiles_n, or for the symmetric products
+// (Gram and Poly) only the upper triangle nt >= mt, row by row.
+__device__ __forceinline__ int tiles_per_matrix(const GemmClass& C, bool sym) {
+    return sym ? C.tiles_m * (C.tiles_m + 1) / 2 : C.tiles_m * C.tiles_n;
+}
+
+__device__ __forceinline__ Tile decode_tile(const GemmParams& P, int tile, bool sym) {
     int c = 0;
     while (c + 1 < P.nclasses && tile >= P.cls[c + 1].tile_begin) ++c;
     const GemmClass& C = P.cls[c];
     const int local = tile - C.tile_begin;
-    const int per = C.tiles_m * C.tiles_n;
+    const int per = tiles_per_matrix(C, sym);
     const int b = local / per;
     const int rem = local - b * per;
-    const int mt = rem / C.tiles_n;
-    return Tile{c, b, mt, rem - mt * C.tiles_n, rem};
+    if (!sym) {
+        const int mt = rem / C.tiles_n;
+        return Tile{c, b, mt, rem - mt * C.tiles_n, rem};
+    }
+    int mt = 0, u = rem;
+    while (u >= C.tiles_m - mt) {
+        u -= C.tiles_m - mt;
+        ++mt;
+    }
+    return Tile{c, b, mt, mt + u, rem};
 }
 
 // Bytes CTA `rank` loads for one reduction slice of tile t.  Boxes that lie
@@ -148,6 +172,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint64_t budget = P.budget_ns;
     const bool b_mn = (P.phase == kBX);
+    const bool sym = (P.phase != kBX);   // A and B' are symmetric: upper tiles only
     const int rank = static_cast<int>(cluster_ctarank());
     const bool leader = (rank == 0);
     const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
@@ -186,7 +211,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
         if (lane == 0) {
             uint32_t stage = 0, phase = 0;
             for (int tile = pair; tile < P.total_tiles; tile += npairs) {
-                const Tile t = decode_tile(P, tile);
+                const Tile t = decode_tile(P, tile, sym);
                 const GemmClass& C = P.cls[t.cls];
                 const int nkb = (C.K + kBK - 1) / kBK;
                 int nb_self = 0, nb_peer = 0;
@@ -224,7 +249,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
             uint32_t stage = 0, phase = 0;
             int it = 0;
             for (int tile = pair; tile < P.total_tiles; tile += npairs, ++it) {
-                const Tile t = decode_tile(P, tile);
+                const Tile t = decode_tile(P, tile, sym);
                 const GemmClass& C = P.cls[t.cls];
                 const int nkb = (C.K + kBK - 1) / kBK;
                 const uint32_t acc = it & 1, acc_phase = (it >> 1) & 1;
@@ -273,6 +298,8 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
         }
     } else {
         // -------------------------------------------------------- epilogue
+        uint8_t* stage_out = smem + kStages * kStageBytes;   // 1024-byte aligned
+        int obuf = 0;
         const int ew = warp - 2;                  // epilogue warp 0..kEpiWarps-1
         const int quarter = warp & 3;             // TMEM lanes this warp may read
         const int colw = (ew >> 2) * kEpiCols;    // first accumulator column of this warp
@@ -280,7 +307,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
         const uint32_t tempty_leader1 = mapa_shared(smem_u32(&tempty_bar[1]), 0);
         int it = 0;
         for (int tile = pair; tile < P.total_tiles; tile += npairs, ++it) {
-            const Tile t = decode_tile(P, tile);
+            const Tile t = decode_tile(P, tile, sym);
             const GemmClass& C = P.cls[t.cls];
             const uint32_t acc = it & 1, acc_phase = (it >> 1) & 1;
             if (!mbar_wait_cluster_bounded(&tfull_bar[acc], acc_phase, budget, abort_flag)) {
@@ -296,7 +323,6 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
             const float kx = P.first ? P.scal[g].k : 1.f;
             const size_t bs = static_cast<size_t>(M) * N;
             const __nv_bfloat16* ein = C.ein != nullptr ? C.ein + t.b * bs : nullptr;
-            __nv_bfloat16* out = C.out != nullptr ? C.out + t.b * bs : nullptr;
             const bool need_ein = (P.phase == kPoly);
             const bool last_bx = (P.phase == kBX) && P.last;
             // NS frame row / column scalings of D = L O R (swapped when transposed).
@@ -322,6 +348,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
             };
             uint4 xin[4];
             uint32_t rv[2][32];
+            const int row0 = t.mt * kTileM + rank * kBM + quarter * 32;   // warp's first row
             if (nch > 0) {
                 tmem_ld_issue(tbase, rv[0]);
                 tmem_ld_wait(rv[0]);
@@ -352,36 +379,64 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
 #pragma unroll
                     for (int j = 0; j < 32; ++j) v[j] *= kx;
                 }
-                if (rok) {
-                    if (!last_bx) {
+                {
+                    // Stage the 32 x 32 chunk (row = lane, 64 bytes) with the 64-byte
+                    // swizzle the store map expects, then one TMA store writes it
+                    // (A, B', the next X, or O in the NS frame on the last iteration).
+                    uint8_t* box = stage_out + (ew * 2 + obuf) * kStoreBoxBytes;
+                    if (lane == 0) bulk_wait_group_read<1>();   // this buffer's last store read it
+                    __syncwarp();
 #pragma unroll
-                        for (int q8 = 0; q8 < 4; ++q8)
-                            if (col0 + q8 * 8 < N)
-                                *reinterpret_cast<uint4*>(out + static_cast<size_t>(row) * N +
-                                                          col0 + q8 * 8) = pack8(v + 8 * q8);
-                    } else {
-                        // O in W's orientation, then partial sums of O^2 and D^2.
-                        if (!md.trans) {
+                    for (int c = 0; c < 4; ++c)
+                        *reinterpret_cast<uint4*>(box + lane * 64 + ((c ^ ((lane >> 1) & 3)) << 4)) =
+                            pack8(v + 8 * c);
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_3d(&C.tmOut, box, col0, row0, t.b);
+                        bulk_commit_group();
+                    }
+                    obuf ^= 1;
+                }
+                if (sym && t.nt != t.mt) {
+                    // Mirror an off-diagonal tile of the symmetric product: the
+                    // transposed chunk (box row = column j, 32 rows of this warp)
+                    // goes to rows [col0, col0+32) x columns [row0, row0+32).
+                    // Lane pairs swap one value per column pair so each lane
+                    // writes a 32-bit (two-row) word.
+                    uint8_t* box = stage_out + (ew * 2 + obuf) * kStoreBoxBytes;
+                    if (lane == 0) bulk_wait_group_read<1>();
+                    __syncwarp();
+                    const bool odd = lane & 1;
+                    const int r2 = lane & ~1;                 // first of the two rows
 #pragma unroll
-                            for (int q8 = 0; q8 < 4; ++q8)
-                                if (col0 + q8 * 8 < N)
-                                    *reinterpret_cast<uint4*>(md.O + static_cast<size_t>(row) * N +
-                                                              col0 + q8 * 8) = pack8(v + 8 * q8);
-                        } else {
+                    for (int j = 0; j < 32; j += 2) {
+                        // even lane keeps column j, odd lane keeps column j + 1
+                        const float send = odd ? v[j] : v[j + 1];
+                        const float recv = __shfl_xor_sync(0xffffffffu, send, 1);
+                        const float lo = odd ? recv : v[j];        // row r2
+                        const float hi = odd ? v[j + 1] : recv;    // row r2 + 1
+                        const int jc = j + (odd ? 1 : 0);          // box row
+                        const int off = jc * 64 + (((r2 >> 3) ^ ((jc >> 1) & 3)) << 4) + (r2 & 7) * 2;
+                        *reinterpret_cast<__nv_bfloat162*>(box + off) = __floats2bfloat162_rn(lo, hi);
+                    }
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_3d(&C.tmOut, box, row0, col0, t.b);
+                        bulk_commit_group();
+                    }
+                    obuf ^= 1;
+                }
+                if (last_bx && rok) {
+                    // Partial sums of O^2 and D^2 over the stored (bf16) O.
 #pragma unroll
-                            for (int j = 0; j < 32; ++j)
-                                if (col0 + j < N)
-                                    md.O[static_cast<size_t>(col0 + j) * M + row] =
-                                        __float2bfloat16_rn(v[j]);
-                        }
-#pragma unroll
-                        for (int j = 0; j < 32; ++j) {
-                            if (col0 + j < N) {
-                                const float o = __bfloat162float(__float2bfloat16_rn(v[j]));
-                                const float dv = urow * o * vvec[col0 + j];
-                                sum_o = fmaf(o, o, sum_o);
-                                sum_d = fmaf(dv, dv, sum_d);
-                            }
+                    for (int j = 0; j < 32; ++j) {
+                        if (col0 + j < N) {
+                            const float o = __bfloat162float(__float2bfloat16_rn(v[j]));
+                            const float dv = urow * o * vvec[col0 + j];
+                            sum_o = fmaf(o, o, sum_o);
+                            sum_d = fmaf(dv, dv, sum_d);
                         }
                     }
                 }
@@ -404,6 +459,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                 }
             }
         }
+        if (lane == 0) bulk_wait_group_all();     // every output store has landed
     }
 
     // Neither CTA may leave (or free TMEM) while its pair partner can still

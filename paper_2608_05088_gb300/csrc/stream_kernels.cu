@@ -359,18 +359,85 @@ scalars_kernel(const MatDesc* __restrict__ mats, MatScalars* __restrict__ scal,
 }
 
 // ------------------------------------------------------------------ apply
+__device__ __forceinline__ void apply8(const MatDesc& d, const UserPtrs& up, bool wbf, float s,
+                                       float decay, int i, int j, const float (&o)[8]) {
+    const size_t e = static_cast<size_t>(i) * d.n + j;
+    const float Li = d.L[i];
+    const float4 r0 = *reinterpret_cast<const float4*>(d.R + j);
+    const float4 r1 = *reinterpret_cast<const float4*>(d.R + j + 4);
+    const float rj[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
+    float w[8];
+    if (wbf) {
+        const uint4 u = *reinterpret_cast<const uint4*>(static_cast<__nv_bfloat16*>(up.w) + e);
+        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float2 f = __bfloat1622float2(h[k]);
+            w[2 * k] = f.x;
+            w[2 * k + 1] = f.y;
+        }
+    } else {
+        const float4* wp = reinterpret_cast<const float4*>(static_cast<float*>(up.w) + e);
+        const float4 a = wp[0], b = wp[1];
+        w[0] = a.x; w[1] = a.y; w[2] = a.z; w[3] = a.w;
+        w[4] = b.x; w[5] = b.y; w[6] = b.z; w[7] = b.w;
+    }
+    const float sl = s * Li;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) w[k] = fmaf(-sl * o[k], rj[k], decay * w[k]);
+    if (wbf) {
+        *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(up.w) + e) = pack8_bf16(w);
+    } else {
+        float4* wp = reinterpret_cast<float4*>(static_cast<float*>(up.w) + e);
+        wp[0] = make_float4(w[0], w[1], w[2], w[3]);
+        wp[1] = make_float4(w[4], w[5], w[6], w[7]);
+    }
+}
+
 __global__ void __launch_bounds__(256)
 apply_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
              const MatScalars* __restrict__ scal, const int32_t* __restrict__ pref, int nmat,
              float decay) {
+    __shared__ float tile[64][65];
     const int g = find_mat(pref, nmat, blockIdx.x);
     const MatDesc& d = mats[g];
-    const int n = d.n;
-    const int32_t total = d.m * n;
-    const int32_t e0 = (blockIdx.x - __ldg(pref + g)) * kApplyElems;
+    const int m = d.m, n = d.n;
+    const int local = blockIdx.x - __ldg(pref + g);
     const float s = scal[g].scale;
     const UserPtrs up = ptrs[g];
     const bool wbf = d.w_bf16 != 0;
+    if (d.trans) {
+        // Tall matrix: O is stored n x m (NS frame).  Stage the 64 x 64 tile of
+        // O^T covering W rows [i0, i0+64) x cols [j0, j0+64) through shared memory.
+        const int tiles_c = (n + 63) / 64;
+        const int i0 = (local / tiles_c) * 64, j0 = (local % tiles_c) * 64;
+        const int t = threadIdx.x;
+#pragma unroll
+        for (int pass = 0; pass < 2; ++pass) {
+            const int jj = pass * 32 + (t >> 3);          // row of O_ns = column of W
+            const int ii = (t & 7) * 8;                   // 8 consecutive rows of W
+            float o[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+            if (j0 + jj < n && i0 + ii < m)
+                load8(d.O, true, static_cast<size_t>(j0 + jj) * m + i0 + ii, o);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) tile[ii + k][jj] = o[k];
+        }
+        __syncthreads();
+#pragma unroll
+        for (int pass = 0; pass < 2; ++pass) {
+            const int ii = pass * 32 + (t >> 3);          // row of W
+            const int jj = (t & 7) * 8;                   // 8 consecutive columns of W
+            if (i0 + ii < m && j0 + jj < n) {
+                float o[8];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) o[k] = tile[ii][jj + k];
+                apply8(d, up, wbf, s, decay, i0 + ii, j0 + jj, o);
+            }
+        }
+        return;
+    }
+    const int32_t total = m * n;
+    const int32_t e0 = local * kApplyElems;
 #pragma unroll
     for (int v = 0; v < kApplyElems / (256 * 8); ++v) {
         const int32_t e = e0 + (v * 256 + threadIdx.x) * 8;
@@ -378,35 +445,37 @@ apply_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs
         const int i = e / n, j = e - i * n;
         float o[8];
         load8(d.O, true, static_cast<size_t>(e), o);
-        const float Li = d.L[i];
-        const float4 r0 = *reinterpret_cast<const float4*>(d.R + j);
-        const float4 r1 = *reinterpret_cast<const float4*>(d.R + j + 4);
-        const float rj[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
-        float w[8];
-        if (wbf) {
-            const uint4 u = *reinterpret_cast<const uint4*>(static_cast<__nv_bfloat16*>(up.w) + e);
-            const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+        apply8(d, up, wbf, s, decay, i, j, o);
+    }
+}
+
+// dst (cols x rows) = src^T through 64 x 64 shared-memory tiles (debug copy of O).
+__global__ void __launch_bounds__(256)
+transpose_bf16_kernel(const __nv_bfloat16* __restrict__ src, __nv_bfloat16* __restrict__ dst,
+                      int rows, int cols) {
+    __shared__ float tile[64][65];
+    const int tiles_c = (cols + 63) / 64;
+    const int r0 = (blockIdx.x / tiles_c) * 64, c0 = (blockIdx.x % tiles_c) * 64;
+    const int t = threadIdx.x;
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const float2 f = __bfloat1622float2(h[k]);
-                w[2 * k] = f.x;
-                w[2 * k + 1] = f.y;
-            }
-        } else {
-            const float4* wp = reinterpret_cast<const float4*>(static_cast<float*>(up.w) + e);
-            const float4 a = wp[0], b = wp[1];
-            w[0] = a.x; w[1] = a.y; w[2] = a.z; w[3] = a.w;
-            w[4] = b.x; w[5] = b.y; w[6] = b.z; w[7] = b.w;
-        }
-        const float sl = s * Li;
+    for (int pass = 0; pass < 2; ++pass) {
+        const int rr = pass * 32 + (t >> 3), cc = (t & 7) * 8;
+        float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        if (r0 + rr < rows && c0 + cc < cols)
+            load8(src, true, static_cast<size_t>(r0 + rr) * cols + c0 + cc, v);
 #pragma unroll
-        for (int k = 0; k < 8; ++k) w[k] = fmaf(-sl * o[k], rj[k], decay * w[k]);
-        if (wbf) {
-            *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(up.w) + e) = pack8_bf16(w);
-        } else {
-            float4* wp = reinterpret_cast<float4*>(static_cast<float*>(up.w) + e);
-            wp[0] = make_float4(w[0], w[1], w[2], w[3]);
-            wp[1] = make_float4(w[4], w[5], w[6], w[7]);
+        for (int k = 0; k < 8; ++k) tile[rr][cc + k] = v[k];
+    }
+    __syncthreads();
+#pragma unroll
+    for (int pass = 0; pass < 2; ++pass) {
+        const int cc = pass * 32 + (t >> 3), rr = (t & 7) * 8;
+        if (c0 + cc < cols && r0 + rr < rows) {
+            float v[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) v[k] = tile[rr + k][cc];
+            *reinterpret_cast<uint4*>(dst + static_cast<size_t>(c0 + cc) * rows + r0 + rr) =
+                pack8_bf16(v);
         }
     }
 }
@@ -469,6 +538,13 @@ cudaError_t launch_apply(const MatDesc* mats, const UserPtrs* ptrs, const MatSca
                          const int32_t* pref, int nmat, int32_t blocks, float decay,
                          cudaStream_t s) {
     apply_kernel<<<blocks, 256, 0, s>>>(mats, ptrs, scal, pref, nmat, decay);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_transpose_bf16(const __nv_bfloat16* src, __nv_bfloat16* dst, int rows, int cols,
+                                  cudaStream_t s) {
+    const int blocks = ((rows + 63) / 64) * ((cols + 63) / 64);
+    transpose_bf16_kernel<<<blocks, 256, 0, s>>>(src, dst, rows, cols);
     return cudaGetLastError();
 }
 

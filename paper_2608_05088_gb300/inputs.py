@@ -43,6 +43,16 @@ class Workload:
     def elements(self) -> int:
         return int(sum(m * n for m, n in self.shapes))
 
+    def ns_flops_min(self) -> float:
+        """Newton-Schulz flops of one step when the symmetry of A = X X^T and
+        of the polynomial in A is used: per matrix and iteration p^2 q (Gram,
+        one triangle) + p^3 (A A, one triangle) + 2 p^2 q (B X)."""
+        tot = 0.0
+        for m, n in self.shapes:
+            p, q = min(m, n), max(m, n)
+            tot += 3.0 * p * p * q + p ** 3
+        return tot * self.ns_steps
+
     def ns_flops_dense(self) -> float:
         """Dense Newton-Schulz flops of one step: per matrix and iteration
         4 p^2 q + 2 p^3 with p = min(m, n), q = max(m, n)."""
