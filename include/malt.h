@@ -123,6 +123,27 @@ int malt_step(malt_state_t* st, const malt_param_t* params, int32_t n,
 int malter_step(malt_state_t* st, const malt_param_t* params, int32_t n,
                 const malt_hparams_t* hp, void* stream);
 
+/* One MALT (malter = 0) or MALTER (malter != 0) step whose gradients arrive
+ * in HOST memory and whose updated weights are copied back to HOST memory.
+ * g_host[i] holds rows*cols elements of params[i].g_dtype and is copied into
+ * the device buffer params[i].g (which the library overwrites); after the
+ * update, params[i].w is copied to w_host[i] (rows*cols elements of
+ * params[i].w_dtype).  Host buffers should be page-locked (cudaHostAlloc /
+ * pinned) for the copies to overlap.  The copies run on two library-owned
+ * streams ordered by events against `stream`: the next call's gradient copy
+ * waits only until the last step that read the same device G buffers (same
+ * params[0].g) has consumed them -- so a caller that alternates two device
+ * gradient sets gets the copy-in of step i+1 fully overlapped with step i,
+ * and a caller with one set still overlaps it with step i's Newton-Schulz
+ * work -- and this step's weight copy overlaps the next step, whose weight
+ * update waits for it.  Returns immediately; w_host is valid
+ * once malt_check (which waits for all three streams) returns.  The host
+ * buffers must stay untouched until then.  Same validation and errors as
+ * malt_step, plus MALT_ERR_INVALID_ARG for a null host pointer. */
+int malt_step_host(malt_state_t* st, const malt_param_t* params, int32_t n,
+                   const malt_hparams_t* hp, int32_t malter, const void* const* g_host,
+                   void* const* w_host, void* stream);
+
 /* Checkpoint support: copy the n per-matrix nu values and the step counter t
  * to host memory (get) or from host memory (set).  Both synchronise with the
  * stream of the state's last call.  M, l, r and W are caller-owned and are
@@ -130,7 +151,8 @@ int malter_step(malt_state_t* st, const malt_param_t* params, int32_t n,
 int malt_get_scalars(malt_state_t* st, float* nu_host, int32_t n, int64_t* t_host);
 int malt_set_scalars(malt_state_t* st, const float* nu_host, int32_t n, int64_t t_host);
 
-/* Wait for the stream of the state's last call, then return (and clear) the
+/* Wait for the stream of the state's last call (and the copy streams of
+ * malt_step_host), then return (and clear) the
  * device-side status word: MALT_OK, or MALT_ERR_TIMEOUT when a kernel gave up
  * on a bounded wait, or MALT_ERR_CUDA when the stream reported an error. */
 int malt_check(malt_state_t* st);

@@ -124,6 +124,26 @@ struct malt_state {
     std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> ev_pending;
     double prof_ms[MALT_NUM_KINDS] = {};
     int64_t prof_launches[MALT_NUM_KINDS] = {};
+    // Host-buffer steps: copy streams and the events that order them against
+    // the compute stream (created on first use).
+    cudaStream_t h2d = nullptr, d2h = nullptr;
+    cudaEvent_t ev_h2d = nullptr, ev_applied = nullptr, ev_d2h = nullptr;
+    // "G consumed" events per device gradient buffer set (keyed by the first
+    // parameter's G pointer), so callers that alternate two sets let the next
+    // copy-in run while the current step still reads the other set.
+    static constexpr int kGSlots = 2;
+    const void* g_key[kGSlots] = {nullptr, nullptr};
+    cudaEvent_t ev_g_consumed[kGSlots] = {nullptr, nullptr};
+    bool g_recorded[kGSlots] = {false, false};
+    int g_next_slot = 0;
+    bool pipe_primed = false;
+};
+
+// Ordering hooks of a host-buffer step inside run_step.
+struct PipeHooks {
+    cudaEvent_t record_g_consumed;   // after the last kernel that reads G
+    cudaEvent_t wait_before_apply;   // the previous step's weight read-back (or null)
+    cudaEvent_t record_applied;      // after the apply kernel
 };
 
 namespace {
@@ -155,6 +175,11 @@ int validate_hparams(const malt_hparams_t* hp) {
 
 void free_state(malt_state* st) {
     if (st == nullptr) return;
+    for (cudaEvent_t e : {st->ev_g_consumed[0], st->ev_g_consumed[1], st->ev_h2d, st->ev_applied,
+                          st->ev_d2h})
+        if (e != nullptr) cudaEventDestroy(e);
+    for (cudaStream_t q : {st->h2d, st->d2h})
+        if (q != nullptr) cudaStreamDestroy(q);
     for (auto& p : st->ev_pending) {
         cudaEventDestroy(p.second.first);
         cudaEventDestroy(p.second.second);
@@ -454,8 +479,8 @@ int run_gemm_phase(malt_state* st, int phase, int it, int last, const malt_hpara
     return MALT_OK;
 }
 
-int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_hparams_t* hp,
-             void* stream, int malter) {
+int validate_step(malt_state* st, const malt_param_t* params, int32_t n,
+                  const malt_hparams_t* hp) {
     if (st == nullptr || (n > 0 && params == nullptr)) return MALT_ERR_INVALID_ARG;
     int rc = validate_hparams(hp);
     if (rc != MALT_OK) return rc;
@@ -468,6 +493,13 @@ int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_h
             a.w_dtype != params[i].w_dtype || a.g_dtype != params[i].g_dtype)
             return MALT_ERR_SHAPE_CHANGED;
     }
+    return MALT_OK;
+}
+
+int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_hparams_t* hp,
+             void* stream, int malter, const PipeHooks* hooks = nullptr) {
+    int rc = validate_step(st, params, n, hp);
+    if (rc != MALT_OK) return rc;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     st->last_stream = s;
     if (n == 0) return MALT_OK;
@@ -490,6 +522,8 @@ int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_h
         MALT_CUDA(launch_prescale(st->d_mats, st->d_ptrs, st->d_pref[2], nm, st->blocks_pre,
                                   malter, s), "prescale_kernel");
     }
+    if (hooks != nullptr)   // stats and prescale are the only readers of G
+        MALT_CUDA(cudaEventRecord(hooks->record_g_consumed, s), "cudaEventRecord(G consumed)");
     {
         LaunchScope ls(st, MALT_KIND_NORMS, s);
         MALT_CUDA(launch_norms(st->d_mats, st->d_scal, nm, hp->ns_eps, malter, s), "norms_kernel");
@@ -516,12 +550,85 @@ int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_h
         LaunchScope ls(st, MALT_KIND_SCALARS, s);
         MALT_CUDA(launch_scalars(st->d_mats, st->d_scal, st->d_t, nm, sh, s), "scalars_kernel");
     }
+    if (hooks != nullptr && hooks->wait_before_apply != nullptr)
+        MALT_CUDA(cudaStreamWaitEvent(s, hooks->wait_before_apply, 0), "cudaStreamWaitEvent(W read)");
     {
         LaunchScope ls(st, MALT_KIND_APPLY, s);
         MALT_CUDA(launch_apply(st->d_mats, st->d_ptrs, st->d_scal, st->d_pref[3], nm,
                                st->blocks_apply, 1.f - hp->lr * hp->weight_decay, s),
                   "apply_kernel");
     }
+    if (hooks != nullptr)
+        MALT_CUDA(cudaEventRecord(hooks->record_applied, s), "cudaEventRecord(applied)");
+    return MALT_OK;
+}
+
+size_t elem_bytes(int32_t dtype) { return dtype == MALT_BF16 ? 2 : 4; }
+
+int ensure_pipe(malt_state* st) {
+    if (st->h2d != nullptr) return MALT_OK;
+    MALT_CUDA(cudaStreamCreateWithFlags(&st->h2d, cudaStreamNonBlocking), "cudaStreamCreate(h2d)");
+    MALT_CUDA(cudaStreamCreateWithFlags(&st->d2h, cudaStreamNonBlocking), "cudaStreamCreate(d2h)");
+    for (cudaEvent_t* e : {&st->ev_g_consumed[0], &st->ev_g_consumed[1], &st->ev_h2d,
+                           &st->ev_applied, &st->ev_d2h})
+        MALT_CUDA(cudaEventCreateWithFlags(e, cudaEventDisableTiming), "cudaEventCreate");
+    return MALT_OK;
+}
+
+// Slot of the "G consumed" event for this device gradient buffer set.
+int g_slot(malt_state* st, const void* key) {
+    for (int k = 0; k < malt_state::kGSlots; ++k)
+        if (st->g_key[k] == key) return k;
+    const int k = st->g_next_slot;
+    st->g_next_slot = (k + 1) % malt_state::kGSlots;
+    st->g_key[k] = key;
+    st->g_recorded[k] = false;
+    return k;
+}
+
+int run_host_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_hparams_t* hp,
+                  int malter, const void* const* g_host, void* const* w_host, void* stream) {
+    int rc = validate_step(st, params, n, hp);
+    if (rc != MALT_OK) return rc;
+    if (n > 0 && (g_host == nullptr || w_host == nullptr)) return MALT_ERR_INVALID_ARG;
+    for (int i = 0; i < n; ++i)
+        if (g_host[i] == nullptr || w_host[i] == nullptr) return MALT_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (n == 0) {
+        st->last_stream = s;
+        return MALT_OK;
+    }
+    MALT_CUDA(cudaSetDevice(st->device), "cudaSetDevice");
+    rc = ensure_pipe(st);
+    if (rc != MALT_OK) return rc;
+    // Gradients in: wait until the last step that read this device G set has
+    // consumed it.  (A step whose set differs may still be running.)
+    const int slot = g_slot(st, params[0].g);
+    if (st->g_recorded[slot])
+        MALT_CUDA(cudaStreamWaitEvent(st->h2d, st->ev_g_consumed[slot], 0), "cudaStreamWaitEvent(G)");
+    for (int i = 0; i < n; ++i) {
+        const size_t bytes = static_cast<size_t>(params[i].rows) * params[i].cols *
+                             elem_bytes(params[i].g_dtype);
+        MALT_CUDA(cudaMemcpyAsync(const_cast<void*>(params[i].g), g_host[i], bytes,
+                                  cudaMemcpyHostToDevice, st->h2d), "cudaMemcpyAsync(G in)");
+    }
+    MALT_CUDA(cudaEventRecord(st->ev_h2d, st->h2d), "cudaEventRecord(h2d)");
+    MALT_CUDA(cudaStreamWaitEvent(s, st->ev_h2d, 0), "cudaStreamWaitEvent(h2d)");
+    const PipeHooks hooks{st->ev_g_consumed[slot], st->pipe_primed ? st->ev_d2h : nullptr,
+                          st->ev_applied};
+    rc = run_step(st, params, n, hp, stream, malter, &hooks);
+    if (rc != MALT_OK) return rc;
+    st->g_recorded[slot] = true;
+    // Weights out, overlapping the next step's statistics and Newton-Schulz work.
+    MALT_CUDA(cudaStreamWaitEvent(st->d2h, st->ev_applied, 0), "cudaStreamWaitEvent(applied)");
+    for (int i = 0; i < n; ++i) {
+        const size_t bytes = static_cast<size_t>(params[i].rows) * params[i].cols *
+                             elem_bytes(params[i].w_dtype);
+        MALT_CUDA(cudaMemcpyAsync(w_host[i], params[i].w, bytes, cudaMemcpyDeviceToHost, st->d2h),
+                  "cudaMemcpyAsync(W out)");
+    }
+    MALT_CUDA(cudaEventRecord(st->ev_d2h, st->d2h), "cudaEventRecord(d2h)");
+    st->pipe_primed = true;
     return MALT_OK;
 }
 
@@ -570,9 +677,19 @@ int malter_step(malt_state_t* st, const malt_param_t* params, int32_t n, const m
     return run_step(st, params, n, hp, stream, 1);
 }
 
+int malt_step_host(malt_state_t* st, const malt_param_t* params, int32_t n,
+                   const malt_hparams_t* hp, int32_t malter, const void* const* g_host,
+                   void* const* w_host, void* stream) {
+    return run_host_step(st, params, n, hp, malter != 0, g_host, w_host, stream);
+}
+
 int malt_check(malt_state_t* st) {
     if (st == nullptr) return MALT_ERR_INVALID_ARG;
     MALT_CUDA(cudaStreamSynchronize(st->last_stream), "cudaStreamSynchronize");
+    if (st->d2h != nullptr) {
+        MALT_CUDA(cudaStreamSynchronize(st->h2d), "cudaStreamSynchronize(h2d)");
+        MALT_CUDA(cudaStreamSynchronize(st->d2h), "cudaStreamSynchronize(d2h)");
+    }
     if (st->ws == nullptr) return MALT_OK;
     int32_t status = 0;
     MALT_CUDA(cudaMemcpy(&status, st->d_status, sizeof(status), cudaMemcpyDeviceToHost),
@@ -717,6 +834,10 @@ const char* malt_status_string(int code) {
 void malt_destroy_state(malt_state_t* st) {
     if (st == nullptr) return;
     cudaStreamSynchronize(st->last_stream);
+    if (st->d2h != nullptr) {
+        cudaStreamSynchronize(st->h2d);
+        cudaStreamSynchronize(st->d2h);
+    }
     free_state(st);
 }
 

@@ -31,7 +31,7 @@ EXPORTS = ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
            "malt_set_scalars", "malt_check", "malt_debug_direction", "malt_debug_scalars",
            "malt_debug_wait_timeout", "malt_profile_enable", "malt_profile_read",
            "malt_workspace_bytes", "malt_status_string", "malt_destroy_state",
-           "malt_stats_noalloc")
+           "malt_stats_noalloc", "malt_step_host")
 NOALLOC_SCRATCH_FLOATS = 1048576
 KIND_NAMES = ("bind", "stats", "finalize", "prescale", "norms", "ns_gram", "ns_poly", "ns_bx",
               "scalars", "apply")
@@ -94,6 +94,9 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.malt_status_string.restype = ctypes.c_char_p
     lib.malt_destroy_state.argtypes = [vp]
     lib.malt_destroy_state.restype = None
+    lib.malt_step_host.argtypes = [vp, P(malt_param_t), i32, P(malt_hparams_t), i32,
+                                   P(vp), P(vp), vp]
+    lib.malt_step_host.restype = ctypes.c_int
     f32 = ctypes.c_float
     lib.malt_stats_noalloc.argtypes = [vp, i32, vp, vp, vp, vp, vp, i64, i64, f32, f32, f32, vp]
     lib.malt_stats_noalloc.restype = ctypes.c_int
@@ -170,6 +173,18 @@ def malter_step(st, params, hp: malt_hparams_t, stream=None):
     arr = params_array(params)
     _check(load().malter_step(st, arr, len(params), ctypes.byref(hp), _stream_handle(stream)),
            "malter_step")
+
+
+def malt_step_host(st, params, hp: malt_hparams_t, g_host, w_host, malter=False, stream=None):
+    """Step with gradients from host tensors g_host[i] (pinned) into the device
+    buffers of params, and updated weights copied back into host tensors
+    w_host[i]; valid after malt_check."""
+    arr = params_array(params)
+    n = len(params)
+    gp = (ctypes.c_void_p * max(n, 1))(*[t.data_ptr() for t in g_host])
+    wp = (ctypes.c_void_p * max(n, 1))(*[t.data_ptr() for t in w_host])
+    _check(load().malt_step_host(st, arr, n, ctypes.byref(hp), 1 if malter else 0, gp, wp,
+                                 _stream_handle(stream)), "malt_step_host")
 
 
 def malt_check(st) -> int:
@@ -251,6 +266,11 @@ class MaltOptimizer:
     def step(self, hp: malt_hparams_t, malter: bool = False, stream=None, params=None):
         ps = self.params if params is None else params
         (malter_step if malter else malt_step)(self.state, ps, hp, stream)
+
+    def step_host(self, hp: malt_hparams_t, g_host, w_host, malter: bool = False, stream=None,
+                  params=None):
+        ps = self.params if params is None else params
+        malt_step_host(self.state, ps, hp, g_host, w_host, malter, stream)
 
     def check(self) -> int:
         return malt_check(self.state)

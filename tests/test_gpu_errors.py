@@ -51,3 +51,33 @@ def test_empty_parameter_list():
     opt.step(malt.hparams())
     assert opt.check() == malt.MALT_OK
     opt.close()
+
+
+def test_host_buffer_step_matches_device_step():
+    """malt_step_host (gradients from pinned host memory, weights copied back)
+    gives bitwise the same W, M, l, r as malt_step on the same gradients, and
+    the host copies of W equal the device W after every step."""
+    import numpy as np
+    import torch
+    wl = inputs.Workload("hoststep", 42, ((256, 512), (392, 136), (520, 1544)), "bf16", 1.5, 0.02,
+                         "malter", 3)
+    a = Run(wl, check=[])
+    b = Run(wl, check=[])
+    g_host = [torch.empty(s, dtype=torch.float32).pin_memory() for s in wl.shapes]
+    w_host = [torch.empty(s, dtype=torch.bfloat16).pin_memory() for s in wl.shapes]
+    # alternate two device gradient sets, as a pipelining caller does
+    G2 = [torch.empty_like(g) for g in b.G]
+    sets = [b.params, list(zip(b.W, G2, b.M, b.l, b.r))]
+    for step in range(wl.steps):
+        for i in range(len(wl.shapes)):
+            g_host[i].copy_(torch.from_numpy(inputs.gradient(wl, i, step)))
+        a.step(oracle=False)
+        b.opt.step_host(b.hp, g_host, w_host, malter=True, params=sets[step % 2])
+        assert a.status() == malt.MALT_OK and b.opt.check() == malt.MALT_OK
+        for i in range(len(wl.shapes)):
+            assert torch.equal(a.W[i], b.W[i])
+            assert torch.equal(w_host[i], b.W[i].cpu())
+            for x, y in ((a.M[i], b.M[i]), (a.l[i], b.l[i]), (a.r[i], b.r[i])):
+                assert torch.equal(x, y)
+    a.close()
+    b.close()

@@ -3,8 +3,10 @@
 Bars: momentum / statistics / ||Mt|| within 1e-5 relative (fp32 arithmetic);
 orthogonalised direction O and the grafting norms within 2e-2 relative
 Frobenius (bf16 Newton-Schulz operands with fp32 accumulation); final weights
-within 5e-3 relative Frobenius and the update W_0 - W_t within 2e-2; bf16
-weights within one bf16 ulp of the oracle's round-to-nearest-even result.
+within 5e-3 relative Frobenius and the update within 2e-2; bf16 weights
+within |x_gpu - x_oracle| + 1 ulp of the oracle's round-to-nearest-even
+result (x the pre-rounding values) and equal to the rounding of the GPU's own
+pre-rounding value.
 """
 import numpy as np
 import pytest
@@ -144,4 +146,49 @@ def test_gpt2_medium_malter_sampled():
     assert run.status() == 0
     for i in check:
         run.assert_close(i)
+    run.close()
+
+
+def test_gpt2_large_bench_configuration():
+    """The benchmark's own configuration: all 144 GPT-2 Large matrices in one
+    grouped step (bf16 W, fp32 state, 5 NS iterations), 2 MALT steps.  One
+    matrix of each shape is checked in full against the oracle; every
+    matrix's statistics l, r against fp64 row / column sums of its
+    gradients (a property that holds at any size)."""
+    wl = inputs.WORKLOADS["gpt2_large"]
+    check = [0, 1, 2, 3]
+    run = Run(wl, check=check)
+    sq_rows = {}
+    sq_cols = {}
+    mu2 = run.hp_ref.mu2
+    for s in range(2):
+        grads = inputs.gradients_for_step(wl, s)
+        for i, G in enumerate(grads):
+            G64 = G.astype(np.float64)
+            r_, c_ = np.sum(G64 * G64, axis=1), np.sum(G64 * G64, axis=0)
+            sq_rows[i] = mu2 * sq_rows.get(i, 0.0) + (1 - mu2) * r_
+            sq_cols[i] = mu2 * sq_cols.get(i, 0.0) + (1 - mu2) * c_
+        run.step(grads=grads)
+    assert run.status() == 0
+    for i in check:
+        run.assert_close(i)
+    for i in range(len(wl.shapes)):
+        l_gpu = run.host(run.l[i])
+        r_gpu = run.host(run.r[i])
+        assert np.max(np.abs(l_gpu - sq_rows[i]) / sq_rows[i]) < 1e-5, i
+        assert np.max(np.abs(r_gpu - sq_cols[i]) / sq_cols[i]) < 1e-5, i
+        assert np.all(np.isfinite(run.host(run.W[i])))
+    run.close()
+
+
+@pytest.mark.parametrize("rows,cols,sigma,ns_steps", [(4096, 4096, 3.0, 8), (4096, 16384, 1.0, 5),
+                                                      (16384, 4096, 0.0, 5)])
+def test_stress_shapes(rows, cols, sigma, ns_steps):
+    """Largest single matrices of the stress set (bf16 W, fp32 state), one
+    MALT step each, checked in full against the oracle."""
+    wl = inputs.stress_workload(rows, cols, sigma, ns_steps)
+    run = Run(wl)
+    run.step()
+    assert run.status() == 0
+    run.assert_close(0, f"stress {rows}x{cols} sigma={sigma} k={ns_steps}")
     run.close()
