@@ -428,16 +428,18 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                     }
                     obuf ^= 1;
                 }
-                if (last_bx && rok) {
-                    // Partial sums of O^2 and D^2 over the stored (bf16) O.
+                if (last_bx) {
+                    // Partial sums of O^2 and (O v)^2 over the stored (bf16) O of this
+                    // row; D^2 = u_row^2 (O v)^2 is formed once per tile.  Lane j holds
+                    // v[col0 + j] and broadcasts it (columns past N contribute 0).
+                    const float vl = (col0 + lane < N) ? vvec[col0 + lane] : 0.f;
 #pragma unroll
                     for (int j = 0; j < 32; ++j) {
-                        if (col0 + j < N) {
-                            const float o = __bfloat162float(__float2bfloat16_rn(v[j]));
-                            const float dv = urow * o * vvec[col0 + j];
-                            sum_o = fmaf(o, o, sum_o);
-                            sum_d = fmaf(dv, dv, sum_d);
-                        }
+                        const float vj = __shfl_sync(0xffffffffu, vl, j);
+                        const float o = __bfloat162float(__float2bfloat16_rn(v[j]));
+                        const float ov = o * vj;
+                        sum_o = fmaf(o, (col0 + j < N) ? o : 0.f, sum_o);
+                        sum_d = fmaf(ov, ov, sum_d);
                     }
                 }
                 if (ch + 1 < nch) tmem_ld_wait(rv[cur ^ 1]);
@@ -446,6 +448,8 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(acc ? tempty_leader1 : tempty_leader0);
             if (last_bx) {
+                if (!rok) sum_o = 0.f;
+                sum_d = rok ? urow * urow * sum_d : 0.f;
 #pragma unroll
                 for (int o = 16; o > 0; o >>= 1) {
                     sum_o += __shfl_xor_sync(0xffffffffu, sum_o, o);
