@@ -15,10 +15,12 @@ namespace malt {
 // Statistics kernel tile (rows x cols of W per block).
 constexpr int kStatRows = 64;
 constexpr int kStatCols = 256;
-// Prescale kernel tile.
-constexpr int kPreTile = 64;
-// Apply kernel: elements per block.
-constexpr int kApplyElems = 4096;
+// Prescale block (rows x cols of Mt); the apply pass of a tall matrix uses
+// the same block shape.
+constexpr int kPreRows = 64;
+constexpr int kPreCols = 256;
+// Apply kernel (wide matrices): contiguous elements per block.
+constexpr int kApplyElems = 16384;
 // Newton-Schulz GEMM: a CTA pair computes a kTileM x kBN output tile; each CTA
 // owns kBM rows of it, loads kBM rows of A and kBN/2 rows (N) of B per kBK
 // reduction slice (one 128-byte swizzle row of bf16).
@@ -54,7 +56,7 @@ struct MatDesc {
     int32_t w_bf16, g_bf16;  // element types of W and G
     int32_t cls, bidx;       // shape class and index within its batch
     int32_t stat_rb, stat_cb;       // statistics row bands / column chunks
-    int32_t pre_tr, pre_tc;         // prescale tiles (rows, cols)
+    int32_t pre_tr, pre_tc;         // prescale blocks (kPreRows x kPreCols), rows and cols
     int32_t ns_tiles;               // GEMM tiles of one p x q product
     int32_t pad_;
     float* rowpart;          // [stat_cb][m] partial row sums of G^2

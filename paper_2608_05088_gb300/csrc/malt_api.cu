@@ -258,8 +258,8 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         st->classes[k].mats.push_back(i);
         d.stat_rb = (m + kStatRows - 1) / kStatRows;
         d.stat_cb = (c + kStatCols - 1) / kStatCols;
-        d.pre_tr = (m + kPreTile - 1) / kPreTile;
-        d.pre_tc = (c + kPreTile - 1) / kPreTile;
+        d.pre_tr = (m + kPreRows - 1) / kPreRows;
+        d.pre_tc = (c + kPreCols - 1) / kPreCols;
         d.ns_tiles = ((p + kTileM - 1) / kTileM) * ((q + kBN - 1) / kBN);
     }
 
@@ -343,10 +343,10 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         pref[0][i + 1] = pref[0][i] + d.stat_rb * d.stat_cb;
         pref[1][i + 1] = pref[1][i] + d.m + d.n;
         pref[2][i + 1] = pref[2][i] + d.pre_tr * d.pre_tc;
-        // apply: contiguous runs of kApplyElems, or 64 x 64 tiles for a tall
-        // matrix whose O is read transposed from the NS frame
+        // apply: contiguous runs of kApplyElems, or 64 x kPreCols blocks for a
+        // tall matrix whose O is read transposed from the NS frame
         const int32_t apply_blocks =
-            d.trans ? ((d.m + 63) / 64) * ((d.n + 63) / 64)
+            d.trans ? ((d.m + 63) / 64) * ((d.n + kPreCols - 1) / kPreCols)
                     : static_cast<int32_t>((elems + kApplyElems - 1) / kApplyElems);
         pref[3][i + 1] = pref[3][i] + apply_blocks;
     }

@@ -213,85 +213,156 @@ finalize_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ p
 }
 
 // --------------------------------------------------------------- prescale
+// One block = kPreRows x kPreCols of Mt.  A wide matrix is streamed like the
+// statistics pass (warp w owns 8 rows, lane 8 consecutive columns, four rows
+// of loads in flight) and written as bf16 in place of its NS frame; a tall
+// matrix's NS frame is Mt^T, so its block walks four 64 x 64 sub-tiles
+// through shared memory and writes each transposed.
 __global__ void __launch_bounds__(256)
 prescale_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
                 const int32_t* __restrict__ pref, int nmat, int malter) {
-    __shared__ float tile[kPreTile][kPreTile + 1];
-    __shared__ float red[32];
+    __shared__ float tile[64][65];
+    __shared__ float2 red[8];
     const int g = find_mat(pref, nmat, blockIdx.x);
     const MatDesc& d = mats[g];
     const int m = d.m, n = d.n;
     const int local = blockIdx.x - __ldg(pref + g);
     const int tr = local / d.pre_tc, tc = local - tr * d.pre_tc;
-    const int r0 = tr * kPreTile, c0 = tc * kPreTile;
-    const int t = threadIdx.x;
+    const int r0 = tr * kPreRows, c0 = tc * kPreCols;
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
     const UserPtrs up = ptrs[g];
     const float* __restrict__ Lv = d.L;
     const float* __restrict__ Rv = d.R;
-    const bool trans = d.trans != 0;
-
+    const float* __restrict__ Mp = up.m;
+    const bool gbf = d.g_bf16 != 0;
     float s_mt = 0.f, s_lgr = 0.f;
-    const int cc = (t & 15) * 4;
-    const int col = c0 + cc;
-    float4 R4 = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (col < n) R4 = *reinterpret_cast<const float4*>(Rv + col);
+
+    if (!d.trans) {
+        const int col = c0 + lane * 8;
+        const bool colok = col < n;
+        float rj[8];
+        if (colok) {
+            const float4 a = *reinterpret_cast<const float4*>(Rv + col);
+            const float4 b = *reinterpret_cast<const float4*>(Rv + col + 4);
+            rj[0] = a.x; rj[1] = a.y; rj[2] = a.z; rj[3] = a.w;
+            rj[4] = b.x; rj[5] = b.y; rj[6] = b.z; rj[7] = b.w;
+        }
+        const int row0 = r0 + warp * 8;
 #pragma unroll
-    for (int pass = 0; pass < 4; ++pass) {
-        const int rr = pass * 16 + (t >> 4);
-        const int row = r0 + rr;
-        float v0 = 0.f, v1 = 0.f, v2 = 0.f, v3 = 0.f;
-        if (row < m && col < n) {
-            const size_t off = static_cast<size_t>(row) * n + col;
-            const float Li = Lv[row];
-            const float4 mv = *reinterpret_cast<const float4*>(up.m + off);
-            v0 = Li * mv.x * R4.x; v1 = Li * mv.y * R4.y;
-            v2 = Li * mv.z * R4.z; v3 = Li * mv.w * R4.w;
-            s_mt += v0 * v0 + v1 * v1 + v2 * v2 + v3 * v3;
-            if (!trans) {
-                uint2 pk;
-                *reinterpret_cast<__nv_bfloat162*>(&pk.x) = __floats2bfloat162_rn(v0, v1);
-                *reinterpret_cast<__nv_bfloat162*>(&pk.y) = __floats2bfloat162_rn(v2, v3);
-                *reinterpret_cast<uint2*>(d.X0 + off) = pk;
-            }
-            if (malter) {
-                float gq[4];
-                if (d.g_bf16) {
-                    const uint2 u = *reinterpret_cast<const uint2*>(
-                        static_cast<const __nv_bfloat16*>(up.g) + off);
-                    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
-                    const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
-                    gq[0] = a.x; gq[1] = a.y; gq[2] = b.x; gq[3] = b.y;
-                } else {
-                    const float4 gf = *reinterpret_cast<const float4*>(
-                        static_cast<const float*>(up.g) + off);
-                    gq[0] = gf.x; gq[1] = gf.y; gq[2] = gf.z; gq[3] = gf.w;
+        for (int rb = 0; rb < 8; rb += 4) {
+            float mv[4][8], li[4];
+            bool ok[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int row = row0 + rb + u;
+                ok[u] = colok && row < m;
+                li[u] = 0.f;
+                if (ok[u]) {
+                    const size_t off = static_cast<size_t>(row) * n + col;
+                    const float4 a = *reinterpret_cast<const float4*>(Mp + off);
+                    const float4 b = *reinterpret_cast<const float4*>(Mp + off + 4);
+                    mv[u][0] = a.x; mv[u][1] = a.y; mv[u][2] = a.z; mv[u][3] = a.w;
+                    mv[u][4] = b.x; mv[u][5] = b.y; mv[u][6] = b.z; mv[u][7] = b.w;
+                    li[u] = Lv[row];
                 }
-                const float a0 = Li * gq[0] * R4.x, a1 = Li * gq[1] * R4.y;
-                const float a2 = Li * gq[2] * R4.z, a3 = Li * gq[3] * R4.w;
-                s_lgr += a0 * a0 + a1 * a1 + a2 * a2 + a3 * a3;
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                if (!ok[u]) continue;
+                const int row = row0 + rb + u;
+                const size_t off = static_cast<size_t>(row) * n + col;
+                float v[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    v[j] = li[u] * mv[u][j] * rj[j];
+                    s_mt = fmaf(v[j], v[j], s_mt);
+                }
+                *reinterpret_cast<uint4*>(d.X0 + off) = pack8_bf16(v);
+                if (malter) {
+                    float gv[8];
+                    load8(up.g, gbf, off, gv);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        const float a = li[u] * gv[j] * rj[j];
+                        s_lgr = fmaf(a, a, s_lgr);
+                    }
+                }
             }
         }
-        tile[rr][cc + 0] = v0; tile[rr][cc + 1] = v1;
-        tile[rr][cc + 2] = v2; tile[rr][cc + 3] = v3;
-    }
-    __syncthreads();
-    // NS frame of a tall matrix is Mt^T: output row = column of Mt, 8
-    // consecutive rows of Mt per thread.
+    } else {
+        const int cc = (t & 15) * 4;
+        for (int sub = 0; sub < kPreCols / 64; ++sub) {
+            const int cs = c0 + sub * 64;
+            if (cs >= n) break;                          // uniform across the block
+            const int col = cs + cc;
+            float4 R4 = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (col < n) R4 = *reinterpret_cast<const float4*>(Rv + col);
 #pragma unroll
-    for (int pass = 0; pass < 2 && trans; ++pass) {
-        const int oc = pass * 32 + (t >> 3);
-        const int seg = (t & 7) * 8;
-        const int gcol = c0 + oc, grow = r0 + seg;
-        if (gcol < n && grow < m) {
-            float v[8];
+            for (int pass = 0; pass < 4; ++pass) {
+                const int rr = pass * 16 + (t >> 4);
+                const int row = r0 + rr;
+                float v0 = 0.f, v1 = 0.f, v2 = 0.f, v3 = 0.f;
+                if (row < m && col < n) {
+                    const size_t off = static_cast<size_t>(row) * n + col;
+                    const float Li = Lv[row];
+                    const float4 mq = *reinterpret_cast<const float4*>(Mp + off);
+                    v0 = Li * mq.x * R4.x; v1 = Li * mq.y * R4.y;
+                    v2 = Li * mq.z * R4.z; v3 = Li * mq.w * R4.w;
+                    s_mt += v0 * v0 + v1 * v1 + v2 * v2 + v3 * v3;
+                    if (malter) {
+                        float gq[4];
+                        if (gbf) {
+                            const uint2 u = *reinterpret_cast<const uint2*>(
+                                static_cast<const __nv_bfloat16*>(up.g) + off);
+                            const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+                            const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+                            gq[0] = a.x; gq[1] = a.y; gq[2] = b.x; gq[3] = b.y;
+                        } else {
+                            const float4 gf = *reinterpret_cast<const float4*>(
+                                static_cast<const float*>(up.g) + off);
+                            gq[0] = gf.x; gq[1] = gf.y; gq[2] = gf.z; gq[3] = gf.w;
+                        }
+                        const float a0 = Li * gq[0] * R4.x, a1 = Li * gq[1] * R4.y;
+                        const float a2 = Li * gq[2] * R4.z, a3 = Li * gq[3] * R4.w;
+                        s_lgr += a0 * a0 + a1 * a1 + a2 * a2 + a3 * a3;
+                    }
+                }
+                tile[rr][cc + 0] = v0; tile[rr][cc + 1] = v1;
+                tile[rr][cc + 2] = v2; tile[rr][cc + 3] = v3;
+            }
+            __syncthreads();
+            // Output row = column of Mt, 8 consecutive rows of Mt per thread.
 #pragma unroll
-            for (int j = 0; j < 8; ++j) v[j] = tile[seg + j][oc];
-            *reinterpret_cast<uint4*>(d.X0 + static_cast<size_t>(gcol) * m + grow) = pack8_bf16(v);
+            for (int pass = 0; pass < 2; ++pass) {
+                const int oc = pass * 32 + (t >> 3);
+                const int seg = (t & 7) * 8;
+                const int gcol = cs + oc, grow = r0 + seg;
+                if (gcol < n && grow < m) {
+                    float v[8];
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) v[j] = tile[seg + j][oc];
+                    *reinterpret_cast<uint4*>(d.X0 + static_cast<size_t>(gcol) * m + grow) =
+                        pack8_bf16(v);
+                }
+            }
+            __syncthreads();                              // tile is reused by the next sub-tile
         }
     }
-    const float a = block_sum(s_mt, red);
-    const float b = block_sum(s_lgr, red);
+    // One fixed-order reduction of both partial sums.
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        s_mt += __shfl_xor_sync(0xffffffffu, s_mt, o);
+        s_lgr += __shfl_xor_sync(0xffffffffu, s_lgr, o);
+    }
+    if (lane == 0) red[warp] = make_float2(s_mt, s_lgr);
+    __syncthreads();
     if (t == 0) {
+        float a = 0.f, b = 0.f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) {
+            a += red[w].x;
+            b += red[w].y;
+        }
         d.prepart[2 * local + 0] = a;
         d.prepart[2 * local + 1] = b;
     }
@@ -407,38 +478,44 @@ apply_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs
     const UserPtrs up = ptrs[g];
     const bool wbf = d.w_bf16 != 0;
     if (d.trans) {
-        // Tall matrix: O is stored n x m (NS frame).  Stage the 64 x 64 tile of
-        // O^T covering W rows [i0, i0+64) x cols [j0, j0+64) through shared memory.
-        const int tiles_c = (n + 63) / 64;
-        const int i0 = (local / tiles_c) * 64, j0 = (local % tiles_c) * 64;
+        // Tall matrix: O is stored n x m (NS frame).  The block covers W rows
+        // [i0, i0+64) x cols [c0, c0+kPreCols) as four 64 x 64 tiles of O^T
+        // staged through shared memory.
+        const int tiles_c = (n + kPreCols - 1) / kPreCols;
+        const int i0 = (local / tiles_c) * 64, c0 = (local % tiles_c) * kPreCols;
         const int t = threadIdx.x;
+        for (int sub = 0; sub < kPreCols / 64; ++sub) {
+            const int j0 = c0 + sub * 64;
+            if (j0 >= n) break;                           // uniform across the block
 #pragma unroll
-        for (int pass = 0; pass < 2; ++pass) {
-            const int jj = pass * 32 + (t >> 3);          // row of O_ns = column of W
-            const int ii = (t & 7) * 8;                   // 8 consecutive rows of W
-            float o[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-            if (j0 + jj < n && i0 + ii < m)
-                load8(d.O, true, static_cast<size_t>(j0 + jj) * m + i0 + ii, o);
+            for (int pass = 0; pass < 2; ++pass) {
+                const int jj = pass * 32 + (t >> 3);      // row of O_ns = column of W
+                const int ii = (t & 7) * 8;               // 8 consecutive rows of W
+                float o[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+                if (j0 + jj < n && i0 + ii < m)
+                    load8(d.O, true, static_cast<size_t>(j0 + jj) * m + i0 + ii, o);
 #pragma unroll
-            for (int k = 0; k < 8; ++k) tile[ii + k][jj] = o[k];
-        }
-        __syncthreads();
-#pragma unroll
-        for (int pass = 0; pass < 2; ++pass) {
-            const int ii = pass * 32 + (t >> 3);          // row of W
-            const int jj = (t & 7) * 8;                   // 8 consecutive columns of W
-            if (i0 + ii < m && j0 + jj < n) {
-                float o[8];
-#pragma unroll
-                for (int k = 0; k < 8; ++k) o[k] = tile[ii][jj + k];
-                apply8(d, up, wbf, s, decay, i0 + ii, j0 + jj, o);
+                for (int k = 0; k < 8; ++k) tile[ii + k][jj] = o[k];
             }
+            __syncthreads();
+#pragma unroll
+            for (int pass = 0; pass < 2; ++pass) {
+                const int ii = pass * 32 + (t >> 3);      // row of W
+                const int jj = (t & 7) * 8;               // 8 consecutive columns of W
+                if (i0 + ii < m && j0 + jj < n) {
+                    float o[8];
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) o[k] = tile[ii][jj + k];
+                    apply8(d, up, wbf, s, decay, i0 + ii, j0 + jj, o);
+                }
+            }
+            __syncthreads();                              // tile is reused by the next sub-tile
         }
         return;
     }
     const int32_t total = m * n;
     const int32_t e0 = local * kApplyElems;
-#pragma unroll
+#pragma unroll 4
     for (int v = 0; v < kApplyElems / (256 * 8); ++v) {
         const int32_t e = e0 + (v * 256 + threadIdx.x) * 8;
         if (e >= total) break;
