@@ -299,6 +299,27 @@ def run_malt(args):
     t_ms = max_over_ranks(e0.elapsed_time(e1), dev)
     value = world * args.steps / (t_ms / 1e3)
 
+    # ---- the same engine as Muon (identity preconditioners, no statistics):
+    # the optimizer-only counterpart of the paper's MALT-vs-Muon overhead table.
+    muon = None
+    if not args.no_muon:
+        for _ in range(2):
+            opt.step(hp, muon=True)
+        torch.cuda.synchronize()
+        barrier()
+        m0 = torch.cuda.Event(enable_timing=True)
+        m1 = torch.cuda.Event(enable_timing=True)
+        m0.record(stream)
+        for _ in range(args.steps):
+            opt.step(hp, muon=True)
+        m1.record(stream)
+        torch.cuda.synchronize()
+        tm = max_over_ranks(m0.elapsed_time(m1), dev) / args.steps
+        muon = {"ms_per_step": tm, "malt_ms_per_step": t_ms / args.steps,
+                "malt_overhead_vs_muon": (t_ms / args.steps) / tm - 1.0}
+        if opt.check() != malt.MALT_OK:
+            raise SystemExit("muon step failed")
+
     # ---- end to end through the C ABI with host buffers (malt_step_host):
     # every step copies all gradients in from pinned host memory and all
     # updated weights back out; the library overlaps those copies with the
@@ -383,7 +404,8 @@ def run_malt(args):
            "dtype": "bf16", "data": "synthetic", "config": workload_config(wl),
            "clocks": clk, "e2e": e2e, "gpu_launches": launches, "roofline": roofline,
            "hbm_kernels": mem, "ms_per_step_by_kernel": breakdown,
-           "cpu_baseline": cpu, "workspace_bytes": opt.workspace_bytes()}
+           "cpu_baseline": cpu, "muon_same_engine": muon,
+           "workspace_bytes": opt.workspace_bytes()}
     print(json.dumps(out), flush=True)
     opt.close()
 
@@ -397,6 +419,7 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-muon", action="store_true")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling only: the first N layers of the workload")
     args = ap.parse_args()

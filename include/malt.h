@@ -123,6 +123,16 @@ int malt_step(malt_state_t* st, const malt_param_t* params, int32_t n,
 int malter_step(malt_state_t* st, const malt_param_t* params, int32_t n,
                 const malt_hparams_t* hp, void* stream);
 
+/* One Muon step through the same engine, for comparison with MALT: the
+ * update of Section 3.1 (eq. muon-update) with the momentum of Algorithm 1,
+ *   M <- mu1 M + (1 - mu1) G,  O = NS_k(M),  W <- W - lr ||O||/(||O|| + eps) O,
+ * i.e. MALT with L = R = I (the graft then only rescales by ||O||/(||O||+eps)).
+ * The row / column statistics l, r are neither read nor updated (their
+ * pointers must still be valid); t advances.  Same arguments and errors as
+ * malt_step. */
+int muon_step(malt_state_t* st, const malt_param_t* params, int32_t n,
+              const malt_hparams_t* hp, void* stream);
+
 /* One MALT (malter = 0) or MALTER (malter != 0) step whose gradients arrive
  * in HOST memory and whose updated weights are copied back to HOST memory.
  * g_host[i] holds rows*cols elements of params[i].g_dtype and is copied into

@@ -15,10 +15,10 @@ struct BindParams {
 
 cudaError_t launch_bind(const BindParams& P, UserPtrs* table, cudaStream_t s);
 cudaError_t launch_stats(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* pref,
-                         int nmat, int32_t blocks, float mu1, cudaStream_t s);
+                         int nmat, int32_t blocks, float mu1, int with_stats, cudaStream_t s);
 cudaError_t launch_finalize(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* pref,
                             int nmat, int32_t total, float mu2, float eps, long long* tcount,
-                            cudaStream_t s);
+                            int identity, cudaStream_t s);
 cudaError_t launch_prescale(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* pref,
                             int nmat, int32_t blocks, int malter, cudaStream_t s);
 cudaError_t launch_norms(const MatDesc* mats, MatScalars* scal, int nmat, float ns_eps,

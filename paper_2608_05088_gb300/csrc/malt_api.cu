@@ -496,8 +496,14 @@ int validate_step(malt_state* st, const malt_param_t* params, int32_t n,
     return MALT_OK;
 }
 
+// Update flavours sharing the engine: MALT (Algorithm 1), MALTER (Algorithm 2),
+// and Muon with the same EMA momentum (identity preconditioners, no statistics).
+enum Flavour { kMalt = 0, kMalter = 1, kMuon = 2 };
+
 int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_hparams_t* hp,
-             void* stream, int malter, const PipeHooks* hooks = nullptr) {
+             void* stream, int flavour, const PipeHooks* hooks = nullptr) {
+    const int malter = flavour == kMalter ? 1 : 0;
+    const int muon = flavour == kMuon ? 1 : 0;
     int rc = validate_step(st, params, n, hp);
     if (rc != MALT_OK) return rc;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -510,12 +516,12 @@ int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_h
     {
         LaunchScope ls(st, MALT_KIND_STATS, s);
         MALT_CUDA(launch_stats(st->d_mats, st->d_ptrs, st->d_pref[0], nm, st->blocks_stats,
-                               hp->mu1, s), "stats_kernel");
+                               hp->mu1, !muon, s), "stats_kernel");
     }
     {
         LaunchScope ls(st, MALT_KIND_FINALIZE, s);
         MALT_CUDA(launch_finalize(st->d_mats, st->d_ptrs, st->d_pref[1], nm, st->total_fin,
-                                  hp->mu2, hp->eps, st->d_t, s), "finalize_kernel");
+                                  hp->mu2, hp->eps, st->d_t, muon, s), "finalize_kernel");
     }
     {
         LaunchScope ls(st, MALT_KIND_PRESCALE, s);
@@ -587,7 +593,7 @@ int g_slot(malt_state* st, const void* key) {
 }
 
 int run_host_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_hparams_t* hp,
-                  int malter, const void* const* g_host, void* const* w_host, void* stream) {
+                  int flavour, const void* const* g_host, void* const* w_host, void* stream) {
     int rc = validate_step(st, params, n, hp);
     if (rc != MALT_OK) return rc;
     if (n > 0 && (g_host == nullptr || w_host == nullptr)) return MALT_ERR_INVALID_ARG;
@@ -616,7 +622,7 @@ int run_host_step(malt_state* st, const malt_param_t* params, int32_t n, const m
     MALT_CUDA(cudaStreamWaitEvent(s, st->ev_h2d, 0), "cudaStreamWaitEvent(h2d)");
     const PipeHooks hooks{st->ev_g_consumed[slot], st->pipe_primed ? st->ev_d2h : nullptr,
                           st->ev_applied};
-    rc = run_step(st, params, n, hp, stream, malter, &hooks);
+    rc = run_step(st, params, n, hp, stream, flavour, &hooks);
     if (rc != MALT_OK) return rc;
     st->g_recorded[slot] = true;
     // Weights out, overlapping the next step's statistics and Newton-Schulz work.
@@ -669,18 +675,23 @@ int malt_init_state(malt_state_t** out, const malt_param_t* params, int32_t n, v
 
 int malt_step(malt_state_t* st, const malt_param_t* params, int32_t n, const malt_hparams_t* hp,
               void* stream) {
-    return run_step(st, params, n, hp, stream, 0);
+    return run_step(st, params, n, hp, stream, kMalt);
 }
 
 int malter_step(malt_state_t* st, const malt_param_t* params, int32_t n, const malt_hparams_t* hp,
                 void* stream) {
-    return run_step(st, params, n, hp, stream, 1);
+    return run_step(st, params, n, hp, stream, kMalter);
+}
+
+int muon_step(malt_state_t* st, const malt_param_t* params, int32_t n, const malt_hparams_t* hp,
+              void* stream) {
+    return run_step(st, params, n, hp, stream, kMuon);
 }
 
 int malt_step_host(malt_state_t* st, const malt_param_t* params, int32_t n,
                    const malt_hparams_t* hp, int32_t malter, const void* const* g_host,
                    void* const* w_host, void* stream) {
-    return run_host_step(st, params, n, hp, malter != 0, g_host, w_host, stream);
+    return run_host_step(st, params, n, hp, malter != 0 ? kMalter : kMalt, g_host, w_host, stream);
 }
 
 int malt_check(malt_state_t* st) {

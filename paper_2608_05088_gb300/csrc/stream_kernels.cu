@@ -101,6 +101,8 @@ __global__ void bind_kernel(const __grid_constant__ BindParams P, UserPtrs* __re
 constexpr int kStatRowsPerWarp = kStatRows / 8;
 constexpr int kStatBatch = 4;
 
+// kStats = false (Muon through the same engine): momentum only.
+template <bool kStats>
 __global__ void __launch_bounds__(256)
 stats_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
              const int32_t* __restrict__ pref, int nmat, float mu1) {
@@ -162,10 +164,13 @@ stats_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs
                 mp[0] = make_float4(nm[0], nm[1], nm[2], nm[3]);
                 mp[1] = make_float4(nm[4], nm[5], nm[6], nm[7]);
             }
-            rs = warp_sum(rs);
-            if (lane == rb4 + u) myrow = rs;
+            if (kStats) {
+                rs = warp_sum(rs);
+                if (lane == rb4 + u) myrow = rs;
+            }
         }
     }
+    if (!kStats) return;
     if (lane < kStatRowsPerWarp && row0 + lane < m)
         d.rowpart[static_cast<size_t>(cb) * m + row0 + lane] = myrow;
 
@@ -187,13 +192,17 @@ stats_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs
 __global__ void __launch_bounds__(256)
 finalize_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
                 const int32_t* __restrict__ pref, int nmat, int32_t total,
-                float mu2, float eps, long long* tcount) {
+                float mu2, float eps, long long* tcount, int identity) {
     const int32_t x = blockIdx.x * blockDim.x + threadIdx.x;
     if (x == 0) *tcount += 1;                 // 1-based step count
     if (x >= total) return;
     const int g = find_mat(pref, nmat, x);
     const MatDesc& d = mats[g];
     const int local = x - __ldg(pref + g);
+    if (identity) {                           // Muon: L = R = I, statistics untouched
+        if (local < d.m) d.L[local] = 1.f; else d.R[local - d.m] = 1.f;
+        return;
+    }
     const UserPtrs up = ptrs[g];
     if (local < d.m) {
         const int i = local;
@@ -580,16 +589,20 @@ cudaError_t launch_bind(const BindParams& P, UserPtrs* table, cudaStream_t s) {
 }
 
 cudaError_t launch_stats(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* pref,
-                         int nmat, int32_t blocks, float mu1, cudaStream_t s) {
-    stats_kernel<<<blocks, 256, 0, s>>>(mats, ptrs, pref, nmat, mu1);
+                         int nmat, int32_t blocks, float mu1, int with_stats, cudaStream_t s) {
+    if (with_stats)
+        stats_kernel<true><<<blocks, 256, 0, s>>>(mats, ptrs, pref, nmat, mu1);
+    else
+        stats_kernel<false><<<blocks, 256, 0, s>>>(mats, ptrs, pref, nmat, mu1);
     return cudaGetLastError();
 }
 
 cudaError_t launch_finalize(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* pref,
                             int nmat, int32_t total, float mu2, float eps, long long* tcount,
-                            cudaStream_t s) {
+                            int identity, cudaStream_t s) {
     const int blocks = (total + 255) / 256 > 0 ? (total + 255) / 256 : 1;
-    finalize_kernel<<<blocks, 256, 0, s>>>(mats, ptrs, pref, nmat, total, mu2, eps, tcount);
+    finalize_kernel<<<blocks, 256, 0, s>>>(mats, ptrs, pref, nmat, total, mu2, eps, tcount,
+                                          identity);
     return cudaGetLastError();
 }
 

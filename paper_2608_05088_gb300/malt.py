@@ -31,7 +31,7 @@ EXPORTS = ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
            "malt_set_scalars", "malt_check", "malt_debug_direction", "malt_debug_scalars",
            "malt_debug_wait_timeout", "malt_profile_enable", "malt_profile_read",
            "malt_workspace_bytes", "malt_status_string", "malt_destroy_state",
-           "malt_stats_noalloc", "malt_step_host")
+           "malt_stats_noalloc", "malt_step_host", "muon_step")
 NOALLOC_SCRATCH_FLOATS = 1048576
 KIND_NAMES = ("bind", "stats", "finalize", "prescale", "norms", "ns_gram", "ns_poly", "ns_bx",
               "scalars", "apply")
@@ -94,6 +94,8 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.malt_status_string.restype = ctypes.c_char_p
     lib.malt_destroy_state.argtypes = [vp]
     lib.malt_destroy_state.restype = None
+    lib.muon_step.argtypes = [vp, P(malt_param_t), i32, P(malt_hparams_t), vp]
+    lib.muon_step.restype = ctypes.c_int
     lib.malt_step_host.argtypes = [vp, P(malt_param_t), i32, P(malt_hparams_t), i32,
                                    P(vp), P(vp), vp]
     lib.malt_step_host.restype = ctypes.c_int
@@ -173,6 +175,12 @@ def malter_step(st, params, hp: malt_hparams_t, stream=None):
     arr = params_array(params)
     _check(load().malter_step(st, arr, len(params), ctypes.byref(hp), _stream_handle(stream)),
            "malter_step")
+
+
+def muon_step(st, params, hp: malt_hparams_t, stream=None):
+    arr = params_array(params)
+    _check(load().muon_step(st, arr, len(params), ctypes.byref(hp), _stream_handle(stream)),
+           "muon_step")
 
 
 def malt_step_host(st, params, hp: malt_hparams_t, g_host, w_host, malter=False, stream=None):
@@ -263,9 +271,13 @@ class MaltOptimizer:
         self.n = len(self.params)
         self.state = malt_init_state(self.params, stream)
 
-    def step(self, hp: malt_hparams_t, malter: bool = False, stream=None, params=None):
+    def step(self, hp: malt_hparams_t, malter: bool = False, stream=None, params=None,
+             muon: bool = False):
         ps = self.params if params is None else params
-        (malter_step if malter else malt_step)(self.state, ps, hp, stream)
+        if muon:
+            muon_step(self.state, ps, hp, stream)
+        else:
+            (malter_step if malter else malt_step)(self.state, ps, hp, stream)
 
     def step_host(self, hp: malt_hparams_t, g_host, w_host, malter: bool = False, stream=None,
                   params=None):

@@ -80,10 +80,12 @@ class Run:
             G = grads[i] if grads is not None else self.gradient(i, s)
             self.G[i].copy_(self.torch.from_numpy(np.ascontiguousarray(G)))
             if oracle and i in self.check:
+                # Muon through the same engine = MALT with identity preconditioners
                 self.W_ref[i], self.info[i] = ref.malt_step_ref(
                     self.W_ref[i], G.astype(np.float64), self.st_ref[i], self.hp_ref,
-                    variant=self.variant, weight_dtype=self.w_dtypes[i])
-        self.opt.step(self.hp, malter=(self.variant == "malter"))
+                    variant="malt" if self.variant == "muon" else self.variant,
+                    weight_dtype=self.w_dtypes[i], force_identity=(self.variant == "muon"))
+        self.opt.step(self.hp, malter=(self.variant == "malter"), muon=(self.variant == "muon"))
         self.steps_done += 1
 
     def status(self):
@@ -103,8 +105,11 @@ class Run:
             # bf16 rounding decides most entries of W_0 - W_t, so compare the
             # pre-rounding update rebuilt from the GPU's own l, r, O and scale.
             eps = self.hp_ref.eps
-            Lg = (self.host(self.l[i]) + eps) ** -0.125
-            Rg = (self.host(self.r[i]) + eps) ** -0.125
+            if self.variant == "muon":
+                Lg, Rg = np.ones(W.shape[0]), np.ones(W.shape[1])
+            else:
+                Lg = (self.host(self.l[i]) + eps) ** -0.125
+                Rg = (self.host(self.r[i]) + eps) ** -0.125
             dW = float(sc[6]) * Lg[:, None] * O * Rg[None, :]
             dW_ref = info["delta"]
             W_pre = self.W_prev[i] - dW        # the GPU's own pre-rounding value
@@ -112,10 +117,13 @@ class Run:
         else:
             dW = self.W0[i] - W
             dW_ref = self.W0[i] - self.W_ref[i]
+        stats_used = self.variant != "muon"      # Muon leaves l and r untouched
         return dict(
             M=rel(self.host(self.M[i]), st.M),
-            l=float(np.max(np.abs(self.host(self.l[i]) - st.l) / np.maximum(st.l, 1e-30))),
-            r=float(np.max(np.abs(self.host(self.r[i]) - st.r) / np.maximum(st.r, 1e-30))),
+            l=float(np.max(np.abs(self.host(self.l[i]) - st.l) / np.maximum(st.l, 1e-30)))
+            if stats_used else 0.0,
+            r=float(np.max(np.abs(self.host(self.r[i]) - st.r) / np.maximum(st.r, 1e-30)))
+            if stats_used else 0.0,
             O=rel(O, info["O"]),
             W=rel(W, self.W_ref[i]),
             dW=rel(dW, dW_ref),

@@ -19,7 +19,8 @@ def header_functions():
         if fn.endswith(".h"):
             src = open(os.path.join(ROOT, "include", fn)).read()
             src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-            for m in re.finditer(r"^\s*[A-Za-z_][\w\s\*]*?\b(malt\w*)\s*\(", src, flags=re.M):
+            decl = r"^\s*(?:const\s+)?(?:int|void|size_t|char)\s*\**\s*(\w+)\s*\("
+            for m in re.finditer(decl, src, flags=re.M):
                 names.add(m.group(1))
     return names
 

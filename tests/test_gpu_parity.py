@@ -192,3 +192,18 @@ def test_stress_shapes(rows, cols, sigma, ns_steps):
     assert run.status() == 0
     run.assert_close(0, f"stress {rows}x{cols} sigma={sigma} k={ns_steps}")
     run.close()
+
+
+def test_muon_through_the_same_engine():
+    """muon_step = the engine with identity preconditioners, against the
+    oracle's identity-preconditioner MALT step (plain Muon with the EMA
+    momentum, Section 3.1); l and r stay untouched."""
+    wl = inputs.Workload("muon", 36, RAGGED[:6], "f32", 1.5, 0.02, "muon", 3)
+    run = Run(wl, w_dtypes=["f32", "bf16"] * 3)
+    for s in range(wl.steps):
+        run.step()
+        assert run.status() == 0
+        for i in range(len(wl.shapes)):
+            run.assert_close(i, f"muon step {s}")
+            assert not np.any(run.host(run.l[i])) and not np.any(run.host(run.r[i]))
+    run.close()
