@@ -38,5 +38,7 @@ cudaError_t launch_transpose_bf16(const __nv_bfloat16* src, __nv_bfloat16* dst, 
 cudaError_t launch_ns_gemm(const GemmParams& P, int grid_pairs, cudaStream_t s);
 size_t ns_gemm_smem_bytes();
 int ns_gemm_max_pairs();
+// Opt the GEMM kernel into its shared memory and cache the resident pair count.
+cudaError_t ns_gemm_configure();
 
 }  // namespace malt

@@ -656,6 +656,10 @@ int malt_init_state(malt_state_t** out, const malt_param_t* params, int32_t n, v
         rc = cuda_fail(cudaDeviceGetAttribute(&st->num_sms, cudaDevAttrMultiProcessorCount, st->device),
                        "cudaDeviceGetAttribute");
     if (rc == MALT_OK) rc = plan_and_allocate(st, params, n);
+    // One-time kernel configuration (shared-memory opt-in, resident CTA pairs)
+    // happens here, so a first step taken inside a stream capture makes no
+    // such calls.
+    if (rc == MALT_OK && n > 0) rc = cuda_fail(ns_gemm_configure(), "ns_gemm_configure");
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     for (int i = 0; rc == MALT_OK && i < n; ++i) {
         const malt_param_t& p = params[i];

@@ -500,7 +500,7 @@ int ns_gemm_max_pairs() {
     return cached;
 }
 
-cudaError_t launch_ns_gemm(const GemmParams& P, int grid_pairs, cudaStream_t s) {
+cudaError_t ns_gemm_configure() {
     static bool configured = false;
     if (!configured) {
         const cudaError_t e = cudaFuncSetAttribute(
@@ -508,6 +508,13 @@ cudaError_t launch_ns_gemm(const GemmParams& P, int grid_pairs, cudaStream_t s) 
         if (e != cudaSuccess) return e;
         configured = true;
     }
+    ns_gemm_max_pairs();
+    return cudaSuccess;
+}
+
+cudaError_t launch_ns_gemm(const GemmParams& P, int grid_pairs, cudaStream_t s) {
+    const cudaError_t ce = ns_gemm_configure();
+    if (ce != cudaSuccess) return ce;
     ns_gemm_kernel<<<2 * grid_pairs, kThreads, kSmemBytes, s>>>(P);
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) {

@@ -2,6 +2,7 @@
 that runs out reports MALT_ERR_TIMEOUT and leaves the context usable."""
 import ctypes
 
+import numpy as np
 import pytest
 
 import paper_2608_05088_gb300.malt as malt
@@ -79,5 +80,42 @@ def test_host_buffer_step_matches_device_step():
             assert torch.equal(w_host[i], b.W[i].cpu())
             for x, y in ((a.M[i], b.M[i]), (a.l[i], b.l[i]), (a.r[i], b.r[i])):
                 assert torch.equal(x, y)
+    a.close()
+    b.close()
+
+
+def test_step_replays_from_a_cuda_graph():
+    """A step enqueues no host synchronisation and no allocation, so it can
+    be captured into a CUDA graph; replays advance the device-side step
+    counter and give bitwise the same state as eager steps."""
+    import torch
+    wl = inputs.Workload("graph", 43, ((256, 512), (392, 136)), "f32", 1.5, 0.02, "malter", 3)
+    a = Run(wl, check=[])
+    b = Run(wl, check=[])
+    grads = [inputs.gradient(wl, i, 0) for i in range(2)]
+    for run in (a, b):
+        for i in range(2):
+            run.G[i].copy_(torch.from_numpy(grads[i]))
+    torch.cuda.synchronize()
+    for _ in range(3):
+        a.opt.step(a.hp, malter=True)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(graph, stream=s):
+            b.opt.step(b.hp, malter=True, stream=s)
+    torch.cuda.synchronize()
+    # Capturing records the work without running it; replay three steps.
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize()
+    assert a.opt.check() == malt.MALT_OK and b.opt.check() == malt.MALT_OK
+    for i in range(2):
+        for x, y in ((a.W[i], b.W[i]), (a.M[i], b.M[i]), (a.l[i], b.l[i]), (a.r[i], b.r[i])):
+            assert torch.equal(x, y)
+    nu_a, t_a = a.opt.scalars()
+    nu_b, t_b = b.opt.scalars()
+    assert t_a == t_b == 3 and np.array_equal(nu_a, nu_b)
     a.close()
     b.close()
