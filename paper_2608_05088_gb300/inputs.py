@@ -144,3 +144,25 @@ def initial_weights(wl: Workload, indices=None, workers: int = 8):
     idxs = list(range(len(wl.shapes))) if indices is None else list(indices)
     with ThreadPoolExecutor(max_workers=workers) as ex:
         return list(ex.map(lambda i: initial_weight(wl, i), idxs))
+
+
+def toy_quadratic_problem(kappa: float, n: int = 50, r: int = 5, seed: int = 0):
+    """(A, B, C) of the matrix quadratic regression min_X 1/2 ||A X B^T - C||_F^2
+    (Appendix B): C = U* S* V*^T of rank r with orthonormal U*, V* (n x r) and a
+    random core S* of unit Frobenius norm; A = U* R1, B = V* R2 with r x r
+    factors R1, R2 of condition number kappa^(1/4) each, so the Hessian
+    (B^T B) kron (A^T A) has condition number cond(R1)^2 cond(R2)^2 = kappa."""
+    rng = _rng(9_000, int(round(np.log10(kappa) * 100)), seed, 4)
+    U, _ = np.linalg.qr(rng.standard_normal((n, r)))
+    V, _ = np.linalg.qr(rng.standard_normal((n, r)))
+    S = rng.standard_normal((r, r))
+    S /= np.linalg.norm(S)
+
+    def with_condition(c):
+        Q1, _ = np.linalg.qr(rng.standard_normal((r, r)))
+        Q2, _ = np.linalg.qr(rng.standard_normal((r, r)))
+        return Q1 @ np.diag(np.geomspace(1.0, c, r)) @ Q2.T
+
+    c = kappa ** 0.25
+    R1, R2 = with_condition(c), with_condition(c)
+    return U @ R1, V @ R2, U @ S @ V.T
