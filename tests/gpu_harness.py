@@ -31,7 +31,7 @@ class Run:
     """One optimizer state on the GPU plus oracle states for `check` matrices."""
 
     def __init__(self, wl: inputs.Workload, check=None, g_dtype="f32", w_dtypes=None,
-                 variant=None, device="cuda:0", ns_coeffs=ref.DEFAULT_NS_COEFFS):
+                 variant=None, device="cuda:0", ns_coeffs=ref.DEFAULT_NS_COEFFS, **hyper):
         import torch
         import paper_2608_05088_gb300.malt as malt
         self.torch, self.malt = torch, malt
@@ -58,8 +58,17 @@ class Run:
             self.r.append(torch.empty(c, dtype=torch.float32, device=self.dev))
         self.params = list(zip(self.W, self.G, self.M, self.l, self.r))
         self.opt = malt.MaltOptimizer(self.params)
-        self.hp_ref = ref.Hyper(lr=wl.lr, ns_steps=wl.ns_steps, ns_coeffs=tuple(ns_coeffs))
-        self.hp = malt.hparams(lr=wl.lr, ns_steps=wl.ns_steps, ns_coeffs=tuple(ns_coeffs))
+        # Extra hyperparameters (mu1, mu2, eps, weight_decay, ns_eps) go to both
+        # sides.  The library takes its hyperparameters as fp32, so the oracle
+        # gets the same fp32 values (1 - 0.999f differs from 1 - 0.999 by 1.3e-5
+        # relative, more than the statistics bar).
+        f32 = lambda v: float(np.float32(v))
+        self.hp_ref = ref.Hyper(lr=f32(wl.lr), ns_steps=wl.ns_steps,
+                                ns_coeffs=tuple(f32(c) for c in ns_coeffs),
+                                **{k: f32(v) for k, v in hyper.items()})
+        self.hp = malt.hparams(lr=wl.lr, ns_steps=wl.ns_steps, ns_coeffs=tuple(ns_coeffs), **hyper)
+        # the apply kernel's decay factor, 1 - lr * wd evaluated in fp32
+        self.decay_gpu = float(np.float32(1) - np.float32(wl.lr) * np.float32(self.hp_ref.weight_decay))
         self.W_ref = dict(self.W0)
         self.st_ref = {i: ref.State.zeros(*wl.shapes[i]) for i in self.check}
         self.info = {}
@@ -112,8 +121,10 @@ class Run:
                 Rg = (self.host(self.r[i]) + eps) ** -0.125
             dW = float(sc[6]) * Lg[:, None] * O * Rg[None, :]
             dW_ref = info["delta"]
-            W_pre = self.W_prev[i] - dW        # the GPU's own pre-rounding value
-            W_pre_ref = self.W_prev_ref[i] - dW_ref
+            # the GPU's own pre-rounding value, decoupled decay included
+            W_pre = self.decay_gpu * self.W_prev[i] - dW
+            hp = self.hp_ref
+            W_pre_ref = (1.0 - hp.lr * hp.weight_decay) * self.W_prev_ref[i] - dW_ref
         else:
             dW = self.W0[i] - W
             dW_ref = self.W0[i] - self.W_ref[i]

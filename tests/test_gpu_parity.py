@@ -207,3 +207,39 @@ def test_muon_through_the_same_engine():
             run.assert_close(i, f"muon step {s}")
             assert not np.any(run.host(run.l[i])) and not np.any(run.host(run.r[i]))
     run.close()
+
+
+@pytest.mark.parametrize("variant", ["malt", "malter"])
+@pytest.mark.parametrize("hyper", [
+    dict(weight_decay=0.1),                       # decoupled weight decay (reading 7)
+    dict(mu1=0.0, mu2=0.0),                       # no momentum, statistics of this G only
+    dict(eps=1e-3),                               # damping that dominates small rows
+    dict(mu1=0.9, mu2=0.999, ns_eps=1e-5),
+], ids=["wd0.1", "mu0", "eps1e-3", "mu0.9_0.999"])
+def test_hyperparameter_variants(variant, hyper):
+    """Non-default hyperparameters reach every kernel the same way they reach
+    the oracle (f32 and bf16 weights, 3 steps)."""
+    wl = inputs.Workload("hyper", 37, ((256, 512), (392, 136)), "f32", 1.5, 0.05, variant, 3)
+    run = Run(wl, w_dtypes=["f32", "bf16"], **hyper)
+    for s in range(wl.steps):
+        run.step()
+        assert run.status() == 0
+        for i in range(2):
+            run.assert_close(i, f"{hyper} step {s}")
+    run.close()
+
+
+@pytest.mark.parametrize("ns_steps,coeffs", [(1, (3.4445, -4.7750, 2.0315)),
+                                             (12, (1.5, -0.5, 0.0))])
+def test_newton_schulz_settings(ns_steps, coeffs):
+    """One quintic iteration, and twelve iterations of the cubic polynomial
+    (1.5, -0.5, 0), through the whole step."""
+    wl = inputs.Workload("nsset", 38, ((256, 512), (392, 136)), "f32", 1.0, 0.02, "malt", 2,
+                         ns_steps=ns_steps)
+    run = Run(wl, ns_coeffs=coeffs)
+    for _ in range(wl.steps):
+        run.step()
+    assert run.status() == 0
+    for i in range(2):
+        run.assert_close(i)
+    run.close()
