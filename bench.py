@@ -299,6 +299,28 @@ def run_malt(args):
     t_ms = max_over_ranks(e0.elapsed_time(e1), dev)
     value = world * args.steps / (t_ms / 1e3)
 
+    # ---- the same step with the phased Newton-Schulz schedule (one launch
+    # per product) for comparison with the persistent default.
+    sched = None
+    if not args.no_muon:
+        opt.set_ns_schedule(malt.MALT_NS_PHASED)
+        for _ in range(2):
+            opt.step(hp, malter=malter)
+        torch.cuda.synchronize()
+        barrier()
+        p0 = torch.cuda.Event(enable_timing=True)
+        p1 = torch.cuda.Event(enable_timing=True)
+        p0.record(stream)
+        for _ in range(args.steps):
+            opt.step(hp, malter=malter)
+        p1.record(stream)
+        torch.cuda.synchronize()
+        tp = max_over_ranks(p0.elapsed_time(p1), dev) / args.steps
+        opt.set_ns_schedule(malt.MALT_NS_PERSISTENT)
+        if opt.check() != malt.MALT_OK:
+            raise SystemExit("phased-schedule step failed")
+        sched = {"persistent_ms_per_step": t_ms / args.steps, "phased_ms_per_step": tp}
+
     # ---- the same engine as Muon (identity preconditioners, no statistics):
     # the optimizer-only counterpart of the paper's MALT-vs-Muon overhead table.
     muon = None
@@ -357,8 +379,8 @@ def run_malt(args):
 
     # ---- roofline of the dominant kernel (the Newton-Schulz GEMMs)
     pk, pk_src = peaks()
-    ns_ms = sum(prof[k][0] for k in ("ns_gram", "ns_poly", "ns_bx"))
-    ns_launches = sum(prof[k][1] for k in ("ns_gram", "ns_poly", "ns_bx"))
+    ns_ms = sum(prof[k][0] for k in malt.NS_KINDS)
+    ns_launches = sum(prof[k][1] for k in malt.NS_KINDS)
     # Algorithmic work: the Newton-Schulz flops with the symmetry of the Gram
     # matrix and of the polynomial used (3 p^2 q + p^3 per matrix and iteration),
     # which is what the kernels compute (upper-triangle tiles only).
@@ -369,7 +391,8 @@ def run_malt(args):
     traffic = ncu_traffic_per_launch()
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "traffic": traffic,
-                "kernel": "ns_gemm_kernel (Gram, Poly, BX launches)",
+                "kernel": "ns_gemm_kernel<persistent> (every Gram, Poly and BX product "
+                          "of the k iterations in one launch)",
                 "peak_source": f"{pk_src}: bf16_tflops_sustained",
                 "flops_per_step": wl.ns_flops_min(),
                 "flops_counted": "3p^2q + p^3 per matrix and NS iteration (symmetric Gram and polynomial)",
@@ -404,7 +427,7 @@ def run_malt(args):
            "dtype": "bf16", "data": "synthetic", "config": workload_config(wl),
            "clocks": clk, "e2e": e2e, "gpu_launches": launches, "roofline": roofline,
            "hbm_kernels": mem, "ms_per_step_by_kernel": breakdown,
-           "cpu_baseline": cpu, "muon_same_engine": muon,
+           "cpu_baseline": cpu, "muon_same_engine": muon, "ns_schedules": sched,
            "workspace_bytes": opt.workspace_bytes()}
     print(json.dumps(out), flush=True)
     opt.close()

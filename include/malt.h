@@ -176,6 +176,15 @@ int malt_check(malt_state_t* st);
  *   nu, alpha (1 on MALT steps), the applied scale lr*alpha*||O||/(||D||+eps),
  *   and 1/(||Mt||_F + ns_eps). */
 int malt_debug_direction(malt_state_t* st, int32_t idx, void* out, void* stream);
+/* malt_debug_timeout_site: where the first device-side wait gave up in the
+ *   work that the last MALT_ERR_TIMEOUT from malt_check covered, 5 int32 to
+ *   out5 (host memory): site code (1 claim a ring slot, 2 producer waits for
+ *   the previous product, 3 free operand stage, 4 / 20 / 36 next item in the
+ *   ring (odd producer / MMA / epilogue), 5 free accumulator, 6 stage
+ *   operands, 7 finished accumulator, 8 epilogue waits for the Gram product,
+ *   9 MMA drain; 0 when nothing timed out), work item, sequence number or
+ *   reduction slice, block and thread index. */
+int malt_debug_timeout_site(const malt_state_t* st, int32_t* out5);
 int malt_debug_scalars(malt_state_t* st, float* out_host, int32_t n);
 
 /* Exercise the bounded device-side wait used by the kernels: launch one
@@ -200,9 +209,42 @@ int malt_debug_wait_timeout(int64_t budget_ns, void* stream);
 #define MALT_KIND_NS_BX     7
 #define MALT_KIND_SCALARS   8
 #define MALT_KIND_APPLY     9
-#define MALT_NUM_KINDS     10
+#define MALT_KIND_NS_PERSISTENT 10   /* all Newton-Schulz products, persistent schedule */
+#define MALT_NUM_KINDS     11
 int malt_profile_enable(malt_state_t* st, int32_t enable);
 int malt_profile_read(malt_state_t* st, double* ms_out, int64_t* launches_out, int32_t nkinds);
+
+/* Newton-Schulz schedule of a state (the Orth step of Algorithm 1: k
+ * iterations of A = X X^T, B' = aI + bA + cA^2, X <- B' X per matrix).
+ *   MALT_NS_PERSISTENT (default): one persistent launch per group of up to 8
+ *     shape classes runs every product of every iteration.  Tiles are claimed
+ *     dynamically in product order; a tile of matrix j waits on the device
+ *     (bounded) only until the previous product of matrix j is stored, so
+ *     one matrix's next product overlaps another matrix's current one and
+ *     there is no launch gap or wave tail between products.
+ *   MALT_NS_PHASED: one launch per product (3 k launches per group), each
+ *     product over all matrices finished before the next starts.
+ * Both compute every tile with the same arithmetic: results are bitwise
+ * identical.  Takes effect at the next step.  MALT_ERR_INVALID_ARG for a
+ * null state or an unknown schedule. */
+#define MALT_NS_PHASED     0
+#define MALT_NS_PERSISTENT 1
+int malt_set_ns_schedule(malt_state_t* st, int32_t schedule);
+
+/* Host only (no GPU, no CUDA call): the persistent schedule's work list for
+ * these parameter shapes (only rows and cols are read) and ns_steps
+ * iterations, in claim order, 8 int32 per item: launch group, product index
+ * s = 3 * iteration + (0 Gram, 1 Poly, 2 BX), matrix index, tile row, tile
+ * column (256 x 256 tiles of the NS frame; Gram and Poly list the upper
+ * triangle only), the index of the counter the tile waits for ((s - 1) *
+ * n + matrix, or -1), the count that counter must reach (16 signals per
+ * tile of product s - 1), and the number of tiles of product s of this
+ * matrix.  Writes min(capacity, total) items to out (capacity * 8 int32,
+ * caller-owned) and the total to *count; call with capacity 0 to size out.
+ * MALT_ERR_INVALID_ARG for bad arguments or ns_steps outside [1, 64],
+ * MALT_ERR_UNSUPPORTED for a shape malt_init_state would reject. */
+int malt_ns_schedule(const malt_param_t* params, int32_t n, int32_t ns_steps, int32_t* out,
+                     int64_t capacity, int64_t* count);
 
 /* Statistics stage of ONE matrix without any device allocation.
  * The paper has no counterpart: this exists for callers that cannot allocate

@@ -84,37 +84,114 @@ struct StepHyper {
     int32_t malter;
 };
 
-// --------------------------------------------------------------- GEMM launch
+// ------------------------------------------------------ Newton-Schulz engine
 enum GemmPhase : int32_t { kGram = 0, kPoly = 1, kBX = 2 };
 
-struct GemmClass {  // 64-byte aligned through its CUtensorMap members
-    CUtensorMap tmA;              // operand A: rows of a K-major matrix (box kBK x kBM)
-    CUtensorMap tmB;              // operand B: K-major rows (box kBK x kBM), or for kBX
-                                  // an MN-major [K][N] matrix (box kBMN x kBK)
-    CUtensorMap tmOut;            // output [batch][M][N], store box 32 x 32, 64-byte swizzle
-                                  // (the last kBX stores O)
-    int32_t M, N, K;              // per-matrix product shape
-    int32_t batch;
-    int32_t tiles_m, tiles_n;
-    int32_t tile_begin;           // first global tile of this class in the launch
+// Epilogue warps of a CTA pair; each one signals a finished tile once.
+constexpr uint32_t kNsSignalsPerTile = 2 * kEpiWarpsPerCta;
+
+// One shape class (every matrix whose NS frame is p x q, stored batched) with
+// all the tensor maps of the three products of an NS iteration.
+struct NsClass {  // 64-byte aligned through its CUtensorMap members
+    CUtensorMap tmX[2];           // the ping-pong iterates X as K-major rows (box kBK x kBM)
+    CUtensorMap tmXmn[2];         // the same buffers as an MN-major [K][N] operand (box kBMN x kBK)
+    CUtensorMap tmA, tmB;         // A = X X^T and B' = aI + bA + cA^2, K-major rows
+    CUtensorMap stX[2], stA, stB, stO;   // epilogue stores: box 32 x 32, 64-byte swizzle
+    int32_t p, q, batch;
+    int32_t tiles_p, tiles_q;     // 256-wide tiles along p and along q
+    int32_t sym_begin;            // first item of this class within a Gram or Poly phase
+    int32_t full_begin;           // first item of this class within a BX phase
     int32_t pad_;
     const int32_t* mat_of;        // [batch] -> matrix index
-    const __nv_bfloat16* ein;     // epilogue input (A for kPoly), [batch][M][N]
-
+    const __nv_bfloat16* A;       // the A buffer [batch][p][p] (read by the Poly epilogue)
 };
 
-struct GemmParams {
-    GemmClass cls[kMaxClasses];
+// Work list of one launch: for each NS iteration i, the Gram tiles of every
+// class (sym_items), then the Poly tiles (sym_items), then the BX tiles
+// (full_items); item s-phase index = 3 i + kind.  A launch runs the items
+// [item_begin, item_end): one phase (phased schedule, static round-robin) or
+// the whole list (persistent schedule, claimed through *queue, each tile
+// waiting for its matrix's previous phase in done[]).
+struct NsParams {
+    NsClass cls[kMaxClasses];
     int32_t nclasses;
-    int32_t total_tiles;
-    int32_t phase;
-    int32_t first;                // first NS iteration: apply the 1/||Mt|| scale
-    int32_t last;                 // last NS iteration: write O and norm partials
+    int32_t nmat;                 // size of one row of done[]
+    int32_t ns_steps;
+    int32_t sym_items, full_items;
+    int32_t item_begin, item_end;
     float a, b, c;
     const MatDesc* mats;
     const MatScalars* scal;
     int32_t* status;
+    uint32_t* queue;              // next unclaimed item (persistent schedule)
+    uint32_t* done;               // [3 ns_steps][nmat] finished-tile signals (persistent)
     uint64_t budget_ns;
 };
+
+// One decoded work item: a 256 x 256 output tile of one product.
+struct NsWork {
+    int32_t s;                    // 3 * iter + kind
+    int32_t iter, kind;
+    int32_t cls, b;               // class and batch slot (matrix = cls.mat_of[b])
+    int32_t mt, nt;               // tile row / column
+    int32_t local;                // tile index within the matrix's product
+};
+
+// Tiles of one matrix in a product of this kind: all of them for B X, the
+// upper triangle (nt >= mt) for the symmetric Gram and polynomial products.
+__host__ __device__ __forceinline__ int32_t ns_phase_tiles(const NsClass& C, int32_t kind) {
+    return kind == kBX ? C.tiles_p * C.tiles_q : C.tiles_p * (C.tiles_p + 1) / 2;
+}
+
+__host__ __device__ __forceinline__ NsWork ns_decode(const NsParams& P, int32_t item) {
+    NsWork w;
+    const int32_t per_iter = 2 * P.sym_items + P.full_items;
+    w.iter = item / per_iter;
+    int32_t r = item - w.iter * per_iter;
+    if (r < P.sym_items) {
+        w.kind = kGram;
+    } else if (r < 2 * P.sym_items) {
+        w.kind = kPoly;
+        r -= P.sym_items;
+    } else {
+        w.kind = kBX;
+        r -= 2 * P.sym_items;
+    }
+    w.s = 3 * w.iter + w.kind;
+    const bool sym = w.kind != kBX;
+    int32_t c = 0;
+    while (c + 1 < P.nclasses && r >= (sym ? P.cls[c + 1].sym_begin : P.cls[c + 1].full_begin)) ++c;
+    const NsClass& C = P.cls[c];
+    const int32_t local = r - (sym ? C.sym_begin : C.full_begin);
+    const int32_t per = ns_phase_tiles(C, w.kind);
+    w.cls = c;
+    w.b = local / per;
+    const int32_t rem = local - w.b * per;
+    w.local = rem;
+    if (!sym) {
+        w.mt = rem / C.tiles_q;
+        w.nt = rem - w.mt * C.tiles_q;
+    } else {
+        int32_t mt = 0, u = rem;
+        while (u >= C.tiles_p - mt) {
+            u -= C.tiles_p - mt;
+            ++mt;
+        }
+        w.mt = mt;
+        w.nt = mt + u;
+    }
+    return w;
+}
+
+// The counter a work item of matrix g waits for under the persistent
+// schedule -- its matrix's previous product, s - 1 -- and the number of
+// signals that means "every tile stored".  -1 for the first product.
+__host__ __device__ __forceinline__ int32_t ns_dependency(const NsParams& P, const NsWork& w,
+                                                          int32_t g, uint32_t* target) {
+    if (w.s == 0) return -1;
+    const int32_t prev_kind = (w.kind + 2) % 3;
+    *target = kNsSignalsPerTile * static_cast<uint32_t>(ns_phase_tiles(P.cls[w.cls], prev_kind));
+    return (w.s - 1) * P.nmat + g;
+}
 
 }  // namespace malt

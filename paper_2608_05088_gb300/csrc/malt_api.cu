@@ -7,7 +7,10 @@
 // launch gets a block-prefix table.  A step then enqueues, on the caller's
 // stream and without any host synchronisation:
 //   bind (caller pointers) -> stats -> finalize -> prescale -> norms
-//   -> k x (Gram, Poly, BX) over all classes -> scalars -> apply.
+//   -> Newton-Schulz -> scalars -> apply,
+// where Newton-Schulz is one persistent launch per group of up to kMaxClasses
+// classes running all k x (Gram, Poly, BX) products (the default), or one
+// launch per product (the phased schedule).
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
@@ -117,6 +120,14 @@ struct malt_state {
     int32_t* d_status = nullptr;
     int32_t* d_pref[4] = {nullptr, nullptr, nullptr, nullptr};  // stats, fin, pre, apply
     int32_t blocks_stats = 0, total_fin = 0, blocks_pre = 0, blocks_apply = 0;
+    // Newton-Schulz work lists, one per group of up to kMaxClasses classes,
+    // and the persistent schedule's counters: [groups_pad] claim counters,
+    // then [3 * kMaxNsSteps][nmat] finished-tile signals.
+    std::vector<NsParams> ns_groups;
+    uint32_t* d_sched = nullptr;
+    int sched_groups_pad = 0;
+    int ns_schedule = MALT_NS_PERSISTENT;
+    int32_t last_timeout[5] = {};   // site record of the last timeout malt_check reported
     cudaStream_t last_stream = nullptr;
     // Profiling: event pairs recorded around launches, folded in on read.
     bool profiling = false;
@@ -224,11 +235,14 @@ struct LaunchScope {
     }
 };
 
-int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
-    st->nmat = n;
-    st->shape0.assign(params, params + n);
-    st->hmats.resize(n);
-    // Shape classes by NS frame.
+constexpr int kMaxNsSteps = 64;
+constexpr int kStatusWords = 8;
+
+// Per-matrix descriptions and shape classes (one per NS frame p x q, in order
+// of first appearance).  Host only.
+void build_classes(const malt_param_t* params, int n, std::vector<MatDesc>& hmats,
+                   std::vector<ShapeClass>& classes) {
+    hmats.resize(n);
     std::map<std::pair<int, int>, int> cls_of;
     for (int i = 0; i < n; ++i) {
         const int m = static_cast<int>(params[i].rows), c = static_cast<int>(params[i].cols);
@@ -236,15 +250,15 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         auto it = cls_of.find({p, q});
         int k;
         if (it == cls_of.end()) {
-            k = static_cast<int>(st->classes.size());
+            k = static_cast<int>(classes.size());
             cls_of[{p, q}] = k;
-            st->classes.emplace_back();
-            st->classes.back().p = p;
-            st->classes.back().q = q;
+            classes.emplace_back();
+            classes.back().p = p;
+            classes.back().q = q;
         } else {
             k = it->second;
         }
-        MatDesc& d = st->hmats[i];
+        MatDesc& d = hmats[i];
         std::memset(&d, 0, sizeof(d));
         d.m = m;
         d.n = c;
@@ -254,14 +268,75 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         d.w_bf16 = params[i].w_dtype == MALT_BF16;
         d.g_bf16 = params[i].g_dtype == MALT_BF16;
         d.cls = k;
-        d.bidx = st->classes[k].batch++;
-        st->classes[k].mats.push_back(i);
+        d.bidx = classes[k].batch++;
+        classes[k].mats.push_back(i);
         d.stat_rb = (m + kStatRows - 1) / kStatRows;
         d.stat_cb = (c + kStatCols - 1) / kStatCols;
         d.pre_tr = (m + kPreRows - 1) / kPreRows;
         d.pre_tc = (c + kPreCols - 1) / kPreCols;
         d.ns_tiles = ((p + kTileM - 1) / kTileM) * ((q + kBN - 1) / kBN);
     }
+}
+
+// Newton-Schulz work lists: classes ordered by Gram reduction length (q, then
+// p; the heaviest tiles are claimed first), in groups of up to kMaxClasses
+// per launch.  Tensor maps and device pointers are copied from the classes
+// as they stand (host-only callers leave them empty).  Host only.
+void plan_ns_groups(const std::vector<ShapeClass>& classes, int nmat, std::vector<NsParams>& groups,
+                    std::vector<std::vector<int>>* slot_class = nullptr) {
+    std::vector<int> order(classes.size());
+    for (size_t k = 0; k < order.size(); ++k) order[k] = static_cast<int>(k);
+    std::stable_sort(order.begin(), order.end(), [&](int x, int y) {
+        const ShapeClass& a = classes[x];
+        const ShapeClass& b = classes[y];
+        return a.q != b.q ? a.q > b.q : a.p > b.p;
+    });
+    groups.clear();
+    if (slot_class != nullptr) slot_class->clear();
+    for (size_t start = 0; start < order.size(); start += kMaxClasses) {
+        groups.emplace_back();
+        if (slot_class != nullptr) slot_class->emplace_back();
+        NsParams& P = groups.back();
+        std::memset(&P, 0, sizeof(P));
+        const size_t cnt = std::min(order.size() - start, static_cast<size_t>(kMaxClasses));
+        int32_t sym = 0, full = 0;
+        for (size_t j = 0; j < cnt; ++j) {
+            const ShapeClass& S = classes[order[start + j]];
+            if (slot_class != nullptr) slot_class->back().push_back(order[start + j]);
+            NsClass& C = P.cls[j];
+            for (int b = 0; b < 2; ++b) {
+                C.tmX[b] = S.tmX[b];
+                C.tmXmn[b] = S.tmXmn[b];
+                C.stX[b] = S.stX[b];
+            }
+            C.tmA = S.tmA;
+            C.tmB = S.tmB;
+            C.stA = S.stA;
+            C.stB = S.stB;
+            C.stO = S.stO;
+            C.p = S.p;
+            C.q = S.q;
+            C.batch = S.batch;
+            C.tiles_p = (S.p + kTileM - 1) / kTileM;
+            C.tiles_q = (S.q + kBN - 1) / kBN;
+            C.sym_begin = sym;
+            C.full_begin = full;
+            C.mat_of = S.d_mat_of;
+            C.A = S.A;
+            sym += ns_phase_tiles(C, kGram) * S.batch;
+            full += ns_phase_tiles(C, kBX) * S.batch;
+        }
+        P.nclasses = static_cast<int32_t>(cnt);
+        P.nmat = nmat;
+        P.sym_items = sym;
+        P.full_items = full;
+    }
+}
+
+int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
+    st->nmat = n;
+    st->shape0.assign(params, params + n);
+    build_classes(params, n, st->hmats, st->classes);
 
     // Workspace layout.
     Carver cv;
@@ -292,9 +367,14 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
     const size_t o_ptrs = cv.take(sizeof(UserPtrs) * std::max(n, 1));
     const size_t o_scal = cv.take(sizeof(MatScalars) * std::max(n, 1));
     const size_t o_t = cv.take(sizeof(long long));
-    const size_t o_status = cv.take(sizeof(int32_t));
+    // status word, then the first timeout's site record (site, item, seq, block, thread)
+    const size_t o_status = cv.take(sizeof(int32_t) * kStatusWords);
     size_t o_pref[4];
     for (int j = 0; j < 4; ++j) o_pref[j] = cv.take(sizeof(int32_t) * (n + 1));
+    const int ngroups = (nc + kMaxClasses - 1) / kMaxClasses;
+    st->sched_groups_pad = ((ngroups + 63) / 64) * 64;
+    const size_t o_sched = cv.take(sizeof(uint32_t) * (st->sched_groups_pad +
+                                                       static_cast<size_t>(3 * kMaxNsSteps) * n));
 
     st->ws_bytes = cv.off;
     if (cudaMalloc(&st->ws, st->ws_bytes) != cudaSuccess) {
@@ -333,6 +413,7 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
     st->d_t = reinterpret_cast<long long*>(base + o_t);
     st->d_status = reinterpret_cast<int32_t*>(base + o_status);
     for (int j = 0; j < 4; ++j) st->d_pref[j] = reinterpret_cast<int32_t*>(base + o_pref[j]);
+    st->d_sched = reinterpret_cast<uint32_t*>(base + o_sched);
 
     // Block-prefix tables.
     std::vector<int32_t> pref[4];
@@ -375,6 +456,16 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
             return MALT_ERR_CUDA;
         }
     }
+    plan_ns_groups(st->classes, n, st->ns_groups);
+    for (size_t gi = 0; gi < st->ns_groups.size(); ++gi) {
+        NsParams& P = st->ns_groups[gi];
+        P.mats = st->d_mats;
+        P.scal = st->d_scal;
+        P.status = st->d_status;
+        P.queue = st->d_sched + gi;
+        P.done = st->d_sched + st->sched_groups_pad;
+        P.budget_ns = kWaitBudgetNs;
+    }
 
     // Upload the static tables (init is allowed to synchronise).
     MALT_CUDA(cudaMemset(st->ws, 0, st->ws_bytes), "cudaMemset(workspace)");
@@ -410,71 +501,50 @@ int bind_pointers(malt_state* st, const malt_param_t* params, cudaStream_t s) {
     return MALT_OK;
 }
 
-// One GEMM phase of NS iteration `it` over every class, in launches of at
-// most kMaxClasses classes, heaviest K first.
-int run_gemm_phase(malt_state* st, int phase, int it, int last, const malt_hparams_t* hp,
-                   cudaStream_t s) {
-    const int cur = it & 1, nxt = cur ^ 1;
-    std::vector<int> order(st->classes.size());
-    for (size_t k = 0; k < order.size(); ++k) order[k] = static_cast<int>(k);
-    std::stable_sort(order.begin(), order.end(), [&](int x, int y) {
-        const ShapeClass& a = st->classes[x];
-        const ShapeClass& b = st->classes[y];
-        const int ka = phase == kGram ? a.q : a.p;
-        const int kb = phase == kGram ? b.q : b.p;
-        return ka > kb;
-    });
-    static GemmParams P;  // large (kMaxClasses tensor-map pairs): keep off the stack
-    for (size_t start = 0; start < order.size(); start += kMaxClasses) {
-        std::memset(&P, 0, sizeof(P));
-        const size_t cnt = std::min(order.size() - start, static_cast<size_t>(kMaxClasses));
-        int tiles = 0;
-        for (size_t j = 0; j < cnt; ++j) {
-            const ShapeClass& C = st->classes[order[start + j]];
-            GemmClass& G = P.cls[j];
-            G.batch = C.batch;
-            G.mat_of = C.d_mat_of;
-            if (phase == kGram) {
-                G.tmA = C.tmX[cur];
-                G.tmB = C.tmX[cur];
-                G.M = C.p; G.N = C.p; G.K = C.q;
-                G.ein = nullptr;
-                G.tmOut = C.stA;
-            } else if (phase == kPoly) {
-                G.tmA = C.tmA;
-                G.tmB = C.tmA;
-                G.M = C.p; G.N = C.p; G.K = C.p;
-                G.ein = C.A;
-                G.tmOut = C.stB;
-            } else {
-                G.tmA = C.tmB;
-                G.tmB = C.tmXmn[cur];
-                G.M = C.p; G.N = C.q; G.K = C.p;
-                G.ein = nullptr;
-                G.tmOut = last ? C.stO : C.stX[nxt];
-            }
-            G.tiles_m = (G.M + kTileM - 1) / kTileM;
-            G.tiles_n = (G.N + kBN - 1) / kBN;
-            G.tile_begin = tiles;
-            // Gram and Poly products are symmetric: upper-triangle tiles only.
-            const int per = phase == kBX ? G.tiles_m * G.tiles_n : G.tiles_m * (G.tiles_m + 1) / 2;
-            tiles += per * G.batch;
-        }
-        P.nclasses = static_cast<int32_t>(cnt);
-        P.total_tiles = tiles;
-        P.phase = phase;
-        P.first = it == 0;
-        P.last = last;
+// The k Newton-Schulz iterations over every class (after the norms kernel
+// has set 1 / (||Mt|| + ns_eps)).
+int run_newton_schulz(malt_state* st, const malt_hparams_t* hp, cudaStream_t s) {
+    thread_local NsParams P;  // ~12 KB of tensor maps: keep off the stack
+    const int k = hp->ns_steps;
+    const int max_pairs = ns_gemm_max_pairs();
+    auto prepare = [&](const NsParams& G) {
+        P = G;
+        P.ns_steps = k;
         P.a = hp->ns_a;
         P.b = hp->ns_b;
         P.c = hp->ns_c;
-        P.mats = st->d_mats;
-        P.scal = st->d_scal;
-        P.status = st->d_status;
-        P.budget_ns = kWaitBudgetNs;
-        const int pairs = std::max(1, std::min(tiles, ns_gemm_max_pairs()));
-        LaunchScope ls(st, MALT_KIND_NS_GRAM + phase, s);
-        MALT_CUDA(launch_ns_gemm(P, pairs, s), "ns_gemm_kernel");
+    };
+    if (st->ns_schedule == MALT_NS_PERSISTENT) {
+        LaunchScope ls(st, MALT_KIND_NS_PERSISTENT, s, static_cast<int>(st->ns_groups.size()));
+        const size_t counters = st->sched_groups_pad + static_cast<size_t>(3 * k) * st->nmat;
+        MALT_CUDA(cudaMemsetAsync(st->d_sched, 0, counters * sizeof(uint32_t), s),
+                  "cudaMemsetAsync(schedule counters)");
+        for (const NsParams& G : st->ns_groups) {
+            prepare(G);
+            const int items = k * (2 * G.sym_items + G.full_items);
+            P.item_begin = 0;
+            P.item_end = items;
+            const int pairs = std::max(1, std::min(items, max_pairs));
+            MALT_CUDA(launch_ns_gemm(P, true, pairs, s), "ns_gemm_kernel (persistent)");
+        }
+        return MALT_OK;
+    }
+    for (int it = 0; it < k; ++it) {
+        for (int phase = kGram; phase <= kBX; ++phase) {
+            for (const NsParams& G : st->ns_groups) {
+                prepare(G);
+                const int per_iter = 2 * G.sym_items + G.full_items;
+                const int begin = it * per_iter + (phase == kGram ? 0
+                                                   : phase == kPoly ? G.sym_items
+                                                                    : 2 * G.sym_items);
+                const int items = phase == kBX ? G.full_items : G.sym_items;
+                P.item_begin = begin;
+                P.item_end = begin + items;
+                const int pairs = std::max(1, std::min(items, max_pairs));
+                LaunchScope ls(st, MALT_KIND_NS_GRAM + phase, s);
+                MALT_CUDA(launch_ns_gemm(P, false, pairs, s), "ns_gemm_kernel");
+            }
+        }
     }
     return MALT_OK;
 }
@@ -534,13 +604,8 @@ int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_h
         LaunchScope ls(st, MALT_KIND_NORMS, s);
         MALT_CUDA(launch_norms(st->d_mats, st->d_scal, nm, hp->ns_eps, malter, s), "norms_kernel");
     }
-    for (int it = 0; it < hp->ns_steps; ++it) {
-        const int last = it == hp->ns_steps - 1;
-        for (int phase = kGram; phase <= kBX; ++phase) {
-            rc = run_gemm_phase(st, phase, it, last, hp, s);
-            if (rc != MALT_OK) return rc;
-        }
-    }
+    rc = run_newton_schulz(st, hp, s);
+    if (rc != MALT_OK) return rc;
     StepHyper sh;
     sh.lr = hp->lr;
     sh.mu1 = hp->mu1;
@@ -706,11 +771,12 @@ int malt_check(malt_state_t* st) {
         MALT_CUDA(cudaStreamSynchronize(st->d2h), "cudaStreamSynchronize(d2h)");
     }
     if (st->ws == nullptr) return MALT_OK;
-    int32_t status = 0;
-    MALT_CUDA(cudaMemcpy(&status, st->d_status, sizeof(status), cudaMemcpyDeviceToHost),
+    int32_t status[kStatusWords] = {};
+    MALT_CUDA(cudaMemcpy(status, st->d_status, sizeof(status), cudaMemcpyDeviceToHost),
               "cudaMemcpy(status)");
-    if (status != 0) {
-        MALT_CUDA(cudaMemset(st->d_status, 0, sizeof(int32_t)), "cudaMemset(status)");
+    if (status[0] != 0) {
+        std::memcpy(st->last_timeout, status + 1, sizeof(st->last_timeout));
+        MALT_CUDA(cudaMemset(st->d_status, 0, sizeof(status)), "cudaMemset(status)");
         return MALT_ERR_TIMEOUT;
     }
     return MALT_OK;
@@ -831,6 +897,60 @@ int malt_profile_read(malt_state_t* st, double* ms_out, int64_t* launches_out, i
 }
 
 size_t malt_workspace_bytes(const malt_state_t* st) { return st == nullptr ? 0 : st->ws_bytes; }
+
+int malt_debug_timeout_site(const malt_state_t* st, int32_t* out5) {
+    if (st == nullptr || out5 == nullptr) return MALT_ERR_INVALID_ARG;
+    std::memcpy(out5, st->last_timeout, sizeof(st->last_timeout));
+    return MALT_OK;
+}
+
+int malt_set_ns_schedule(malt_state_t* st, int32_t schedule) {
+    if (st == nullptr || (schedule != MALT_NS_PHASED && schedule != MALT_NS_PERSISTENT))
+        return MALT_ERR_INVALID_ARG;
+    st->ns_schedule = schedule;
+    return MALT_OK;
+}
+
+int malt_ns_schedule(const malt_param_t* params, int32_t n, int32_t ns_steps, int32_t* out,
+                     int64_t capacity, int64_t* count) {
+    if (count == nullptr || n < 0 || (n > 0 && params == nullptr) || ns_steps < 1 ||
+        ns_steps > kMaxNsSteps || capacity < 0 || (capacity > 0 && out == nullptr))
+        return MALT_ERR_INVALID_ARG;
+    for (int i = 0; i < n; ++i)
+        if (params[i].rows <= 0 || params[i].cols <= 0 || params[i].rows % 8 != 0 ||
+            params[i].cols % 8 != 0 || params[i].rows * params[i].cols >= (int64_t{1} << 31))
+            return MALT_ERR_UNSUPPORTED;
+    std::vector<MatDesc> hmats;
+    std::vector<ShapeClass> classes;
+    build_classes(params, n, hmats, classes);
+    std::vector<NsParams> groups;
+    std::vector<std::vector<int>> slot_class;
+    plan_ns_groups(classes, n, groups, &slot_class);
+    int64_t total = 0;
+    for (size_t gi = 0; gi < groups.size(); ++gi) {
+        NsParams& P = groups[gi];
+        P.ns_steps = ns_steps;
+        const int32_t items = ns_steps * (2 * P.sym_items + P.full_items);
+        for (int32_t item = 0; item < items; ++item, ++total) {
+            if (total >= capacity) continue;
+            const NsWork w = ns_decode(P, item);
+            const int32_t mat = classes[slot_class[gi][w.cls]].mats[w.b];
+            uint32_t target = 0;
+            const int32_t dep = ns_dependency(P, w, mat, &target);
+            int32_t* o = out + total * 8;
+            o[0] = static_cast<int32_t>(gi);
+            o[1] = w.s;
+            o[2] = mat;
+            o[3] = w.mt;
+            o[4] = w.nt;
+            o[5] = dep;
+            o[6] = static_cast<int32_t>(target);
+            o[7] = ns_phase_tiles(P.cls[w.cls], w.kind);
+        }
+    }
+    *count = total;
+    return MALT_OK;
+}
 
 const char* malt_status_string(int code) {
     switch (code) {

@@ -30,15 +30,38 @@
 // half as much again of load latency.
 //
 // Roles per CTA: warp 0 issues TMA loads (the peer's loads complete on the
-// even CTA's full barrier), warp 1 owns TMEM (allocated for the pair) and, in
-// the even CTA, issues tcgen05.mma into one of two TMEM accumulators; warps
-// 2-9 drain the other accumulator (tcgen05.ld, pipelined per 32-column chunk)
-// and run the epilogue, so the epilogue of tile i overlaps the MMAs of tile
-// i+1.  Each epilogue warp converts its 32 x 32 chunk to bf16 in a
-// double-buffered shared-memory box (64-byte swizzle, bank-conflict free) and
-// writes it with one TMA bulk tensor store.  MMA completion is multicast to both CTAs' barriers; both CTAs'
-// epilogue warps release an accumulator on the even CTA's barrier.  Every wait
-// is bounded; a timeout sets the status word and the CTA winds down.
+// even CTA's full barrier, and both producers arrive on it), warp 1 owns
+// TMEM (allocated for the pair) and, in the even CTA, issues tcgen05.mma into
+// one of two TMEM accumulators; warps 2-9 drain the other accumulator
+// (tcgen05.ld, pipelined per 32-column chunk) and run the epilogue, so the
+// epilogue of tile i overlaps the MMAs of tile i+1.  Each epilogue warp
+// converts its 32 x 32 chunk to bf16 in a double-buffered shared-memory box
+// (64-byte swizzle, bank-conflict free) and writes it with one TMA bulk
+// tensor store.  MMA completion is multicast to both CTAs' barriers; both
+// CTAs' epilogue warps release an accumulator on the even CTA's barrier.
+// Every wait is bounded; a timeout sets the status word (and records where,
+// for malt_debug_timeout_site) and the CTA winds down.
+//
+// Schedules.  A launch runs a range of the work list (NsParams): every tile
+// of every product of every NS iteration, product by product.
+//  * Phased: one launch per product (Gram, Poly, BX of one iteration); pair
+//    j takes items j, j + npairs, ...  The stream orders the products.
+//  * Persistent: one launch for all k iterations.  The even CTA's producer
+//    claims the next item with an atomic on a global counter and hands it to
+//    the other roles of both CTAs through an 8-slot ring in shared memory
+//    (mbarrier-guarded; the peer's copy written through shared::cluster).
+//    Each product of a matrix depends only on the previous product of the
+//    same matrix, so a tile waits (bounded, acquire) until every epilogue
+//    warp of every tile of that product has signalled done[] after its TMA
+//    stores completed.  Tiles of the next product of one matrix start while
+//    the current product of another matrix is still running: no grid-wide
+//    barrier between products, no launch gaps, no wave tails except the
+//    last.  Items are claimed in list order by running CTAs only, so every
+//    item a tile waits for is held by a CTA that is running and whose own
+//    dependencies come earlier still: the schedule cannot deadlock, whatever
+//    number of CTA pairs is resident.
+//  Both schedules run the same per-tile arithmetic, so their results are
+//  bitwise identical.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <cstdint>
@@ -70,6 +93,13 @@ constexpr uint32_t kStageOutBytes = 2 * kStoreBoxBytes * kEpiWarps;  // double-b
 constexpr size_t kSmemBytes =
     static_cast<size_t>(kStages) * kStageBytes + kStageOutBytes + 1024;
 constexpr uint16_t kPairMask = 0x3;
+// Persistent schedule: slots of the item ring, and the readers of each slot
+// besides the even CTA's producer that fills it (the even CTA's MMA thread,
+// the odd CTA's producer, every epilogue warp of both CTAs).
+constexpr int kItemSlots = 8;
+constexpr uint32_t kItemReaders = 2 + 2 * kEpiWarps;
+static_assert(2 * kEpiWarps == static_cast<int>(kNsSignalsPerTile),
+              "every epilogue warp of the pair signals a finished tile once");
 
 static_assert(kBK * 2 == 128, "one K slice must be one 128-byte swizzle row");
 static_assert(kTmemCols <= 512, "two accumulators must fit in TMEM");
@@ -77,50 +107,37 @@ static_assert(kHalfN % kBMN == 0, "B half must be whole MN-major boxes");
 static_assert(kEpiWarps == 8, "epilogue layout assumes two warps per lane quarter");
 static_assert(kTileM == kBN, "symmetric products need square tiles");
 
-struct Tile {
-    int cls, b, mt, nt, local;
+// Operands and output of one work item.
+struct Ops {
+    const CUtensorMap* a;
+    const CUtensorMap* b;
+    const CUtensorMap* out;
+    int M, N, K;
 };
 
-// Tiles of one matrix: all tiles_m x tiles_n, or for the symmetric products
-// (Gram and Poly) only the upper triangle nt >= mt, row by row.
-__device__ __forceinline__ int tiles_per_matrix(const GemmClass& C, bool sym) {
-    return sym ? C.tiles_m * (C.tiles_m + 1) / 2 : C.tiles_m * C.tiles_n;
+__device__ __forceinline__ Ops item_operands(const NsParams& P, const NsWork& w) {
+    const NsClass& C = P.cls[w.cls];
+    const int cur = w.iter & 1;
+    if (w.kind == kGram) return Ops{&C.tmX[cur], &C.tmX[cur], &C.stA, C.p, C.p, C.q};
+    if (w.kind == kPoly) return Ops{&C.tmA, &C.tmA, &C.stB, C.p, C.p, C.p};
+    const bool last = w.iter == P.ns_steps - 1;
+    return Ops{&C.tmB, &C.tmXmn[cur], last ? &C.stO : &C.stX[cur ^ 1], C.p, C.q, C.p};
 }
 
-__device__ __forceinline__ Tile decode_tile(const GemmParams& P, int tile, bool sym) {
-    int c = 0;
-    while (c + 1 < P.nclasses && tile >= P.cls[c + 1].tile_begin) ++c;
-    const GemmClass& C = P.cls[c];
-    const int local = tile - C.tile_begin;
-    const int per = tiles_per_matrix(C, sym);
-    const int b = local / per;
-    const int rem = local - b * per;
-    if (!sym) {
-        const int mt = rem / C.tiles_n;
-        return Tile{c, b, mt, rem - mt * C.tiles_n, rem};
-    }
-    int mt = 0, u = rem;
-    while (u >= C.tiles_m - mt) {
-        u -= C.tiles_m - mt;
-        ++mt;
-    }
-    return Tile{c, b, mt, mt + u, rem};
-}
-
-// Bytes CTA `rank` loads for one reduction slice of tile t.  Boxes that lie
+// Bytes CTA `rank` loads for one reduction slice of a tile.  Boxes that lie
 // wholly past M or N are skipped: they only feed accumulator rows / columns
 // that are never stored.
-__device__ __forceinline__ uint32_t slice_bytes(const GemmClass& C, const Tile& t, int rank,
+__device__ __forceinline__ uint32_t slice_bytes(const Ops& op, const NsWork& w, int rank,
                                                 bool b_mn, int* nbox_b) {
     uint32_t bytes = 0;
-    if (t.mt * kTileM + rank * kBM < C.M) bytes += kABytes;
-    const int n0 = t.nt * kBN + rank * kHalfN;
+    if (w.mt * kTileM + rank * kBM < op.M) bytes += kABytes;
+    const int n0 = w.nt * kBN + rank * kHalfN;
     int nb = 0;
     if (b_mn) {
         for (int j = 0; j < kHalfN / kBMN; ++j)
-            if (n0 + j * kBMN < C.N) ++nb;
+            if (n0 + j * kBMN < op.N) ++nb;
         bytes += nb * kMnBoxBytes;
-    } else if (n0 < C.N) {
+    } else if (n0 < op.N) {
         nb = 1;
         bytes += kBBytes;
     }
@@ -146,21 +163,57 @@ __device__ __forceinline__ uint4 pack8(const float* v) {
     return u;
 }
 
-__device__ __forceinline__ void raise_timeout(const GemmParams& P, volatile int* abort_flag) {
+// Where a wait gave up (recorded once per status word, for malt_debug_timeout_site).
+enum WaitSite : int32_t {
+    kSiteClaim = 1,      // even producer: a ring slot to become free
+    kSiteDepLoad = 2,    // producer: the previous product of the matrix
+    kSiteStage = 3,      // producer: a free operand stage
+    kSiteItem = 4,       // ring reader: the next item (+ 16 * role)
+    kSiteAccFree = 5,    // MMA: a free accumulator
+    kSiteStageFull = 6,  // MMA: operands of a stage
+    kSiteAccFull = 7,    // epilogue: a finished accumulator
+    kSiteDepEpi = 8,     // epilogue: the Gram product (polynomial epilogue)
+    kSiteDrain = 9,      // MMA: the last MMAs before TMEM is freed
+};
+
+__device__ __forceinline__ void raise_timeout(const NsParams& P, volatile int* abort_flag,
+                                              int site = 0, int item = -1, int seq = -1) {
+    if (atomicCAS(P.status + 1, 0, site == 0 ? -1 : site) == 0) {
+        P.status[2] = item;
+        P.status[3] = seq;
+        P.status[4] = static_cast<int32_t>(blockIdx.x);
+        P.status[5] = static_cast<int32_t>(threadIdx.x);
+    }
     atomicOr(P.status, kStatusTimeout);
     *abort_flag = 1;
 }
 
+// Persistent schedule: wait until the product this item reads from is
+// complete for its matrix.
+__device__ __forceinline__ bool wait_dependency(const NsParams& P, const NsWork& w,
+                                                volatile int* abort_flag) {
+    uint32_t target = 0;
+    const int g = P.cls[w.cls].mat_of[w.b];
+    const int idx = ns_dependency(P, w, g, &target);
+    if (idx < 0) return true;
+    return counter_wait_bounded(P.done + idx, target, P.budget_ns, P.status, kStatusTimeout,
+                                abort_flag);
+}
+
 }  // namespace
 
+template <bool kPersistent>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
-ns_gemm_kernel(const __grid_constant__ GemmParams P) {
+ns_gemm_kernel(const __grid_constant__ NsParams P) {
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[kStages];
     __shared__ __align__(8) uint64_t empty_bar[kStages];
     __shared__ __align__(8) uint64_t tfull_bar[2];
     __shared__ __align__(8) uint64_t tempty_bar[2];
     __shared__ __align__(8) uint64_t drain_bar;
+    __shared__ __align__(8) uint64_t item_full[kItemSlots];
+    __shared__ __align__(8) uint64_t item_empty[kItemSlots];
+    __shared__ int32_t item_ring[kItemSlots];
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_sh;
     volatile int* abort_flag = &abort_sh;
@@ -171,15 +224,19 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint64_t budget = P.budget_ns;
-    const bool b_mn = (P.phase == kBX);
-    const bool sym = (P.phase != kBX);   // A and B' are symmetric: upper tiles only
     const int rank = static_cast<int>(cluster_ctarank());
     const bool leader = (rank == 0);
     const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
-            mbar_init(&full_bar[s], 1);
+            // Both producers arrive on the even CTA's full barrier for every
+            // slice (the even one with the pair's transaction bytes), so the
+            // MMA never consumes a slice the odd producer has not reached --
+            // even when the odd CTA loads nothing (M or N within its partner's
+            // half) -- and the odd producer can never fall a whole parity
+            // cycle behind the empty barriers it waits on.
+            mbar_init(&full_bar[s], 2);
             mbar_init(&empty_bar[s], 1);
         }
         for (int a = 0; a < 2; ++a) {
@@ -187,14 +244,25 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
             mbar_init(&tempty_bar[a], 2 * kEpiWarps);
         }
         mbar_init(&drain_bar, 1);
+        if (kPersistent) {
+            for (int s = 0; s < kItemSlots; ++s) {
+                mbar_init(&item_full[s], 1);
+                mbar_init(&item_empty[s], kItemReaders);
+            }
+        }
         abort_sh = 0;
         fence_barrier_init();
         fence_proxy_async_smem();
     }
     if (warp == 0 && lane == 0) {
         for (int c = 0; c < P.nclasses; ++c) {
-            tma_prefetch_desc(&P.cls[c].tmA);
-            tma_prefetch_desc(&P.cls[c].tmB);
+            const NsClass& C = P.cls[c];
+            for (int j = 0; j < 2; ++j) {
+                tma_prefetch_desc(&C.tmX[j]);
+                tma_prefetch_desc(&C.tmXmn[j]);
+            }
+            tma_prefetch_desc(&C.tmA);
+            tma_prefetch_desc(&C.tmB);
         }
     }
     if (warp == 1) {
@@ -206,38 +274,85 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
     tc_fence_after();
     const uint32_t tmem_base = tmem_slot;
 
+    // Item number `seq` of this pair.  Phased: static round-robin.  Persistent:
+    // read from the ring (-2 when the wait gave up); only the even CTA's
+    // producer claims items (claim_item).
+    auto static_item = [&](int seq) -> int {
+        const long long it = static_cast<long long>(P.item_begin) + pair +
+                             static_cast<long long>(seq) * npairs;
+        return it < P.item_end ? static_cast<int>(it) : -1;
+    };
+    auto read_item = [&](int seq) -> int {
+        const int slot = seq % kItemSlots;
+        const uint32_t par = static_cast<uint32_t>(seq / kItemSlots) & 1u;
+        if (!mbar_wait_cluster_bounded(&item_full[slot], par, budget, abort_flag)) return -2;
+        const int item = *reinterpret_cast<volatile int32_t*>(&item_ring[slot]);
+        mbar_arrive_cluster(mapa_shared(smem_u32(&item_empty[slot]), 0));
+        return item;
+    };
+    auto claim_item = [&](int seq) -> int {
+        const int slot = seq % kItemSlots;
+        const uint32_t par = static_cast<uint32_t>(seq / kItemSlots) & 1u;
+        if (!mbar_wait_cluster_bounded(&item_empty[slot], par ^ 1u, budget, abort_flag)) return -2;
+        const uint32_t claimed = atomicAdd(P.queue, 1u);
+        const int item = claimed < static_cast<uint32_t>(P.item_end - P.item_begin)
+                             ? P.item_begin + static_cast<int>(claimed) : -1;
+        *reinterpret_cast<volatile int32_t*>(&item_ring[slot]) = item;
+        st_cluster_u32(mapa_shared(smem_u32(&item_ring[slot]), 1), static_cast<uint32_t>(item));
+        mbar_arrive_cluster(mapa_shared(smem_u32(&item_full[slot]), 0));
+        mbar_arrive_cluster(mapa_shared(smem_u32(&item_full[slot]), 1));
+        return item;
+    };
+
     if (warp == 0) {
         // ---------------------------------------------------- TMA producer
         if (lane == 0) {
             uint32_t stage = 0, phase = 0;
-            for (int tile = pair; tile < P.total_tiles; tile += npairs) {
-                const Tile t = decode_tile(P, tile, sym);
-                const GemmClass& C = P.cls[t.cls];
-                const int nkb = (C.K + kBK - 1) / kBK;
+            for (int seq = 0;; ++seq) {
+                const int item = !kPersistent ? static_item(seq)
+                                 : leader     ? claim_item(seq)
+                                              : read_item(seq);
+                if (item == -2) {
+                    raise_timeout(P, abort_flag, leader ? kSiteClaim : kSiteItem, -2, seq);
+                    break;
+                }
+                if (item < 0) break;
+                const NsWork w = ns_decode(P, item);
+                if (kPersistent) {
+                    if (!wait_dependency(P, w, abort_flag)) {
+                        raise_timeout(P, abort_flag, kSiteDepLoad, item, seq);
+                        break;
+                    }
+                    fence_proxy_async_global();   // the loads below read what other CTAs stored
+                }
+                const Ops op = item_operands(P, w);
+                const bool b_mn = w.kind == kBX;
+                const int nkb = (op.K + kBK - 1) / kBK;
                 int nb_self = 0, nb_peer = 0;
-                const uint32_t bytes_self = slice_bytes(C, t, rank, b_mn, &nb_self);
-                const uint32_t bytes_pair = bytes_self + slice_bytes(C, t, rank ^ 1, b_mn, &nb_peer);
-                const bool load_a = t.mt * kTileM + rank * kBM < C.M;
-                const int a_row = t.mt * kTileM + rank * kBM;
-                const int n0 = t.nt * kBN + rank * kHalfN;
+                const uint32_t bytes_self = slice_bytes(op, w, rank, b_mn, &nb_self);
+                const uint32_t bytes_pair = bytes_self + slice_bytes(op, w, rank ^ 1, b_mn, &nb_peer);
+                const bool load_a = w.mt * kTileM + rank * kBM < op.M;
+                const int a_row = w.mt * kTileM + rank * kBM;
+                const int n0 = w.nt * kBN + rank * kHalfN;
                 bool ok = true;
                 for (int kb = 0; kb < nkb; ++kb) {
                     if (!mbar_wait_cluster_bounded(&empty_bar[stage], phase ^ 1u, budget, abort_flag)) {
-                        raise_timeout(P, abort_flag);
+                        raise_timeout(P, abort_flag, kSiteStage, item, kb);
                         ok = false;
                         break;
                     }
                     uint8_t* sa = smem + stage * kStageBytes;
                     const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
                     if (leader) mbar_arrive_expect_tx(&full_bar[stage], bytes_pair);
-                    if (load_a) tma_load_3d_pair(sa, &C.tmA, kb * kBK, a_row, t.b, fb);
+                    if (load_a) tma_load_3d_pair(sa, op.a, kb * kBK, a_row, w.b, fb);
                     if (b_mn) {
                         for (int j = 0; j < nb_self; ++j)
-                            tma_load_3d_pair(sa + kABytes + j * kMnBoxBytes, &C.tmB,
-                                             n0 + j * kBMN, kb * kBK, t.b, fb);
+                            tma_load_3d_pair(sa + kABytes + j * kMnBoxBytes, op.b,
+                                             n0 + j * kBMN, kb * kBK, w.b, fb);
                     } else if (nb_self > 0) {
-                        tma_load_3d_pair(sa + kABytes, &C.tmB, kb * kBK, n0, t.b, fb);
+                        tma_load_3d_pair(sa + kABytes, op.b, kb * kBK, n0, w.b, fb);
                     }
+                    if (!leader) mbar_arrive_cluster(fb);
                     if (++stage == kStages) { stage = 0; phase ^= 1u; }
                 }
                 if (!ok) break;
@@ -247,14 +362,20 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
         // ------------------------------------------- MMA issuer (even CTA)
         if (lane == 0 && leader) {
             uint32_t stage = 0, phase = 0;
-            int it = 0;
-            for (int tile = pair; tile < P.total_tiles; tile += npairs, ++it) {
-                const Tile t = decode_tile(P, tile, sym);
-                const GemmClass& C = P.cls[t.cls];
-                const int nkb = (C.K + kBK - 1) / kBK;
-                const uint32_t acc = it & 1, acc_phase = (it >> 1) & 1;
+            for (int seq = 0;; ++seq) {
+                const int item = kPersistent ? read_item(seq) : static_item(seq);
+                if (item == -2) {
+                    raise_timeout(P, abort_flag, kSiteItem + 16, -2, seq);
+                    break;
+                }
+                if (item < 0) break;
+                const NsWork w = ns_decode(P, item);
+                const bool b_mn = w.kind == kBX;
+                const int K = w.kind == kGram ? P.cls[w.cls].q : P.cls[w.cls].p;
+                const int nkb = (K + kBK - 1) / kBK;
+                const uint32_t acc = seq & 1, acc_phase = (seq >> 1) & 1;
                 if (!mbar_wait_cluster_bounded(&tempty_bar[acc], acc_phase ^ 1u, budget, abort_flag)) {
-                    raise_timeout(P, abort_flag);
+                    raise_timeout(P, abort_flag, kSiteAccFree, item, seq);
                     break;
                 }
                 tc_fence_after();
@@ -262,7 +383,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                 bool ok = true;
                 for (int kb = 0; kb < nkb; ++kb) {
                     if (!mbar_wait_cluster_bounded(&full_bar[stage], phase, budget, abort_flag)) {
-                        raise_timeout(P, abort_flag);
+                        raise_timeout(P, abort_flag, kSiteStageFull, item, kb);
                         ok = false;
                         break;
                     }
@@ -294,7 +415,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
             }
             // Do not release TMEM while MMAs may still be in flight.
             tc_commit_pair_multicast(&drain_bar, 0x1);
-            if (!mbar_wait_cluster_bounded(&drain_bar, 0, budget, nullptr)) raise_timeout(P, abort_flag);
+            if (!mbar_wait_cluster_bounded(&drain_bar, 0, budget, nullptr)) raise_timeout(P, abort_flag, kSiteDrain);
         }
     } else {
         // -------------------------------------------------------- epilogue
@@ -305,33 +426,56 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
         const int colw = (ew >> 2) * kEpiCols;    // first accumulator column of this warp
         const uint32_t tempty_leader0 = mapa_shared(smem_u32(&tempty_bar[0]), 0);
         const uint32_t tempty_leader1 = mapa_shared(smem_u32(&tempty_bar[1]), 0);
-        int it = 0;
-        for (int tile = pair; tile < P.total_tiles; tile += npairs, ++it) {
-            const Tile t = decode_tile(P, tile, sym);
-            const GemmClass& C = P.cls[t.cls];
-            const uint32_t acc = it & 1, acc_phase = (it >> 1) & 1;
+        for (int seq = 0;; ++seq) {
+            int item;
+            if (kPersistent) {
+                int v = 0;
+                if (lane == 0) v = read_item(seq);
+                item = __shfl_sync(0xffffffffu, v, 0);
+            } else {
+                item = static_item(seq);
+            }
+            if (item == -2) {
+                if (lane == 0) raise_timeout(P, abort_flag, kSiteItem + 32, -2, seq);
+                break;
+            }
+            if (item < 0) break;
+            const NsWork w = ns_decode(P, item);
+            const NsClass& C = P.cls[w.cls];
+            const uint32_t acc = seq & 1, acc_phase = (seq >> 1) & 1;
             if (!mbar_wait_cluster_bounded(&tfull_bar[acc], acc_phase, budget, abort_flag)) {
-                raise_timeout(P, abort_flag);
+                raise_timeout(P, abort_flag, kSiteAccFull, item, seq);
                 break;
             }
             tc_fence_after();
-            const int M = C.M, N = C.N;
-            const int row = t.mt * kTileM + rank * kBM + quarter * 32 + lane;
+            const int M = C.p, N = w.kind == kBX ? C.q : C.p;
+            const CUtensorMap* out_map = item_operands(P, w).out;
+            const bool sym = w.kind != kBX;
+            const int row = w.mt * kTileM + rank * kBM + quarter * 32 + lane;
             const bool rok = row < M;
-            const int g = C.mat_of[t.b];
+            const int g = C.mat_of[w.b];
             const MatDesc& md = P.mats[g];
-            const float kx = P.first ? P.scal[g].k : 1.f;
-            const size_t bs = static_cast<size_t>(M) * N;
-            const __nv_bfloat16* ein = C.ein != nullptr ? C.ein + t.b * bs : nullptr;
-            const bool need_ein = (P.phase == kPoly);
-            const bool last_bx = (P.phase == kBX) && P.last;
+            const float kx = w.iter == 0 ? P.scal[g].k : 1.f;
+            const bool need_ein = (w.kind == kPoly);
+            const __nv_bfloat16* ein =
+                need_ein ? C.A + static_cast<size_t>(w.b) * C.p * C.p : nullptr;
+            const bool last_bx = (w.kind == kBX) && (w.iter == P.ns_steps - 1);
+            if (kPersistent && need_ein) {
+                // The polynomial epilogue reads A directly: acquire the Gram
+                // product's completion (already reached: the producer waited
+                // for it before loading this tile's operands).
+                if (!wait_dependency(P, w, abort_flag)) {
+                    raise_timeout(P, abort_flag, kSiteDepEpi, item, seq);
+                    break;
+                }
+            }
             // NS frame row / column scalings of D = L O R (swapped when transposed).
             const float* uvec = md.trans ? md.R : md.L;
             const float* vvec = md.trans ? md.L : md.R;
             const float urow = (last_bx && rok) ? uvec[row] : 0.f;
             float sum_o = 0.f, sum_d = 0.f;
 
-            const int col_base = t.nt * kBN + colw;     // first output column of this warp
+            const int col_base = w.nt * kBN + colw;     // first output column of this warp
             const int nch = max(0, min(kEpiChunks, (N - col_base + 31) / 32));
             const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                                    acc * kBN + colw;
@@ -340,7 +484,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
 #pragma unroll
                 for (int q8 = 0; q8 < 4; ++q8) {
                     if (rok && col0 + q8 * 8 < N)
-                        dst[q8] = __ldg(reinterpret_cast<const uint4*>(
+                        dst[q8] = __ldcg(reinterpret_cast<const uint4*>(
                             ein + static_cast<size_t>(row) * N + col0 + q8 * 8));
                     else
                         dst[q8] = make_uint4(0u, 0u, 0u, 0u);
@@ -348,7 +492,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
             };
             uint4 xin[4];
             uint32_t rv[2][32];
-            const int row0 = t.mt * kTileM + rank * kBM + quarter * 32;   // warp's first row
+            const int row0 = w.mt * kTileM + rank * kBM + quarter * 32;   // warp's first row
             if (nch > 0) {
                 tmem_ld_issue(tbase, rv[0]);
                 tmem_ld_wait(rv[0]);
@@ -364,11 +508,11 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                 float v[32];
 #pragma unroll
                 for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(rv[cur][j]);
-                if (P.phase == kGram) {
+                if (w.kind == kGram) {
                     const float sc = kx * kx;
 #pragma unroll
                     for (int j = 0; j < 32; ++j) v[j] *= sc;
-                } else if (P.phase == kPoly) {
+                } else if (w.kind == kPoly) {
                     float x[32];
 #pragma unroll
                     for (int q8 = 0; q8 < 4; ++q8) unpack8(xin[q8], x + 8 * q8);
@@ -393,12 +537,12 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                     fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0) {
-                        tma_store_3d(&C.tmOut, box, col0, row0, t.b);
+                        tma_store_3d(out_map, box, col0, row0, w.b);
                         bulk_commit_group();
                     }
                     obuf ^= 1;
                 }
-                if (sym && t.nt != t.mt) {
+                if (sym && w.nt != w.mt) {
                     // Mirror an off-diagonal tile of the symmetric product: the
                     // transposed chunk (box row = column j, 32 rows of this warp)
                     // goes to rows [col0, col0+32) x columns [row0, row0+32).
@@ -423,7 +567,7 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                     fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0) {
-                        tma_store_3d(&C.tmOut, box, row0, col0, t.b);
+                        tma_store_3d(out_map, box, row0, col0, w.b);
                         bulk_commit_group();
                     }
                     obuf ^= 1;
@@ -456,11 +600,18 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
                     sum_d += __shfl_xor_sync(0xffffffffu, sum_d, o);
                 }
                 if (lane == 0) {
-                    float* dst = md.nspart + (static_cast<size_t>(t.local) * kNsPartsPerTile +
+                    float* dst = md.nspart + (static_cast<size_t>(w.local) * kNsPartsPerTile +
                                               rank * kEpiWarps + ew) * 2;
                     dst[0] = sum_o;
                     dst[1] = sum_d;
                 }
+            }
+            if (kPersistent && w.s + 1 < 3 * P.ns_steps && lane == 0) {
+                // This warp's part of the tile is in global memory: signal it
+                // (the last product has no reader inside the launch).
+                bulk_wait_group_all();
+                fence_proxy_async_global();
+                red_release_gpu_add(P.done + w.s * P.nmat + g, 1u);
             }
         }
         if (lane == 0) bulk_wait_group_all();     // every output store has landed
@@ -478,7 +629,19 @@ ns_gemm_kernel(const __grid_constant__ GemmParams P) {
 
 size_t ns_gemm_smem_bytes() { return kSmemBytes; }
 
+namespace {
+
+template <bool kPersistent>
+cudaError_t set_smem_attr() {
+    return cudaFuncSetAttribute(ns_gemm_kernel<kPersistent>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(kSmemBytes));
+}
+
+}  // namespace
+
 // Number of CTA pairs that can be resident at once (the persistent grid).
+// Both instantiations have the same block shape and shared memory.
 int ns_gemm_max_pairs() {
     static int cached = -1;
     if (cached > 0) return cached;
@@ -487,9 +650,8 @@ int ns_gemm_max_pairs() {
     cfg.gridDim = dim3(2, 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = kSmemBytes;
-    if (cudaFuncSetAttribute(ns_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(kSmemBytes)) != cudaSuccess ||
-        cudaOccupancyMaxActiveClusters(&n, ns_gemm_kernel, &cfg) != cudaSuccess || n <= 0) {
+    if (set_smem_attr<true>() != cudaSuccess || set_smem_attr<false>() != cudaSuccess ||
+        cudaOccupancyMaxActiveClusters(&n, ns_gemm_kernel<true>, &cfg) != cudaSuccess || n <= 0) {
         cudaGetLastError();
         int dev = 0, sms = 0;
         cudaGetDevice(&dev);
@@ -503,8 +665,8 @@ int ns_gemm_max_pairs() {
 cudaError_t ns_gemm_configure() {
     static bool configured = false;
     if (!configured) {
-        const cudaError_t e = cudaFuncSetAttribute(
-            ns_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kSmemBytes));
+        cudaError_t e = set_smem_attr<true>();
+        if (e == cudaSuccess) e = set_smem_attr<false>();
         if (e != cudaSuccess) return e;
         configured = true;
     }
@@ -512,20 +674,27 @@ cudaError_t ns_gemm_configure() {
     return cudaSuccess;
 }
 
-cudaError_t launch_ns_gemm(const GemmParams& P, int grid_pairs, cudaStream_t s) {
+cudaError_t launch_ns_gemm(const NsParams& P, bool persistent, int grid_pairs, cudaStream_t s) {
     const cudaError_t ce = ns_gemm_configure();
     if (ce != cudaSuccess) return ce;
-    ns_gemm_kernel<<<2 * grid_pairs, kThreads, kSmemBytes, s>>>(P);
+    if (persistent)
+        ns_gemm_kernel<true><<<2 * grid_pairs, kThreads, kSmemBytes, s>>>(P);
+    else
+        ns_gemm_kernel<false><<<2 * grid_pairs, kThreads, kSmemBytes, s>>>(P);
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) {
         cudaFuncAttributes fa{};
-        cudaFuncGetAttributes(&fa, ns_gemm_kernel);
+        if (persistent)
+            cudaFuncGetAttributes(&fa, ns_gemm_kernel<true>);
+        else
+            cudaFuncGetAttributes(&fa, ns_gemm_kernel<false>);
         std::fprintf(stderr,
-                     "malt: ns_gemm_kernel launch (%d CTAs x %d threads, %zu B dynamic smem) "
-                     "refused: %s; kernel uses %d registers, %zu B static smem, allows %d "
-                     "threads and %d B dynamic smem per block\n",
-                     2 * grid_pairs, kThreads, kSmemBytes, cudaGetErrorString(e), fa.numRegs,
-                     fa.sharedSizeBytes, fa.maxThreadsPerBlock, fa.maxDynamicSharedSizeBytes);
+                     "malt: ns_gemm_kernel<%d> launch (%d CTAs x %d threads, %zu B dynamic smem, "
+                     "%zu B parameters) refused: %s; kernel uses %d registers, %zu B static "
+                     "smem, allows %d threads and %d B dynamic smem per block\n",
+                     persistent ? 1 : 0, 2 * grid_pairs, kThreads, kSmemBytes, sizeof(NsParams),
+                     cudaGetErrorString(e), fa.numRegs, fa.sharedSizeBytes,
+                     fa.maxThreadsPerBlock, fa.maxDynamicSharedSizeBytes);
         cudaGetLastError();
     }
     return e;

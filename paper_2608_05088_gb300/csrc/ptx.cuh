@@ -117,6 +117,49 @@ __device__ __forceinline__ bool mbar_wait_cluster_bounded(uint64_t* bar, uint32_
     }
 }
 
+// 32-bit store into shared memory of a CTA of the cluster (shared::cluster address).
+__device__ __forceinline__ void st_cluster_u32(uint32_t cluster_addr, uint32_t v) {
+    asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(cluster_addr), "r"(v) : "memory");
+}
+
+// --------------------------------------------- cross-CTA signals in global memory
+// Orders this thread's generic-proxy accesses of global memory with its
+// async-proxy (TMA) accesses, both ways.
+__device__ __forceinline__ void fence_proxy_async_global() {
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.global.acquire.gpu.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void red_release_gpu_add(uint32_t* p, uint32_t v) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Wait until *ctr >= target (acquire at GPU scope).  Returns false when the
+// budget ran out, when *abort_flag is raised, or when the status word shows
+// any of abort_bits (another block gave up).
+__device__ __forceinline__ bool counter_wait_bounded(const uint32_t* ctr, uint32_t target,
+                                                     uint64_t budget_ns,
+                                                     const int32_t* status, int32_t abort_bits,
+                                                     volatile int* abort_flag) {
+    if (ld_acquire_gpu(ctr) >= target) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t it = 1;; ++it) {
+        __nanosleep(64);
+        if (ld_acquire_gpu(ctr) >= target) return true;
+        if ((it & 15u) == 0u) {
+            if (abort_flag != nullptr && *abort_flag) return false;
+            if (status != nullptr && (*reinterpret_cast<const volatile int32_t*>(status) & abort_bits))
+                return false;
+            if (globaltimer_ns() - t0 > budget_ns) return false;
+        }
+    }
+}
+
 // --------------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");

@@ -31,10 +31,15 @@ EXPORTS = ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
            "malt_set_scalars", "malt_check", "malt_debug_direction", "malt_debug_scalars",
            "malt_debug_wait_timeout", "malt_profile_enable", "malt_profile_read",
            "malt_workspace_bytes", "malt_status_string", "malt_destroy_state",
-           "malt_stats_noalloc", "malt_step_host", "muon_step")
+           "malt_stats_noalloc", "malt_step_host", "muon_step", "malt_set_ns_schedule",
+           "malt_ns_schedule", "malt_debug_timeout_site")
 NOALLOC_SCRATCH_FLOATS = 1048576
 KIND_NAMES = ("bind", "stats", "finalize", "prescale", "norms", "ns_gram", "ns_poly", "ns_bx",
-              "scalars", "apply")
+              "scalars", "apply", "ns_persistent")
+NS_KINDS = ("ns_gram", "ns_poly", "ns_bx", "ns_persistent")
+# Newton-Schulz schedules (malt_set_ns_schedule)
+MALT_NS_PHASED = 0
+MALT_NS_PERSISTENT = 1
 
 
 class malt_param_t(ctypes.Structure):
@@ -102,6 +107,12 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     f32 = ctypes.c_float
     lib.malt_stats_noalloc.argtypes = [vp, i32, vp, vp, vp, vp, vp, i64, i64, f32, f32, f32, vp]
     lib.malt_stats_noalloc.restype = ctypes.c_int
+    lib.malt_debug_timeout_site.argtypes = [vp, P(i32)]
+    lib.malt_debug_timeout_site.restype = ctypes.c_int
+    lib.malt_set_ns_schedule.argtypes = [vp, i32]
+    lib.malt_set_ns_schedule.restype = ctypes.c_int
+    lib.malt_ns_schedule.argtypes = [P(malt_param_t), i32, i32, P(i32), i64, P(i64)]
+    lib.malt_ns_schedule.restype = ctypes.c_int
     for name in ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
                  "malt_set_scalars", "malt_check", "malt_debug_direction",
                  "malt_debug_scalars", "malt_debug_wait_timeout", "malt_profile_enable",
@@ -260,6 +271,37 @@ def malt_destroy_state(st):
     load().malt_destroy_state(st)
 
 
+def malt_debug_timeout_site(st):
+    """(site, item, seq, block, thread) of the last reported device timeout."""
+    out = (ctypes.c_int32 * 5)()
+    _check(load().malt_debug_timeout_site(st, out), "malt_debug_timeout_site")
+    return tuple(int(v) for v in out)
+
+
+def malt_set_ns_schedule(st, schedule: int):
+    _check(load().malt_set_ns_schedule(st, int(schedule)), "malt_set_ns_schedule")
+
+
+def malt_ns_schedule(shapes, ns_steps: int):
+    """The persistent Newton-Schulz work list for these (rows, cols) shapes,
+    computed on the host by the library (no GPU): an int32 array of shape
+    (items, 8) with columns group, s, matrix, tile row, tile column,
+    counter index, counter target, tiles of (s, matrix)."""
+    import numpy as np
+    arr = (malt_param_t * max(len(shapes), 1))()
+    for i, (rows, cols) in enumerate(shapes):
+        arr[i] = malt_param_t(None, MALT_F32, None, MALT_F32, None, None, None, rows, cols)
+    lib = load()
+    count = ctypes.c_int64(0)
+    _check(lib.malt_ns_schedule(arr, len(shapes), ns_steps, None, 0, ctypes.byref(count)),
+           "malt_ns_schedule")
+    out = np.zeros((count.value, 8), dtype=np.int32)
+    _check(lib.malt_ns_schedule(arr, len(shapes), ns_steps,
+                                out.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)),
+                                count.value, ctypes.byref(count)), "malt_ns_schedule")
+    return out
+
+
 # --- convenience wrapper ------------------------------------------------------
 
 class MaltOptimizer:
@@ -302,6 +344,12 @@ class MaltOptimizer:
         out = torch.empty(W.shape, dtype=torch.bfloat16, device=W.device)
         malt_debug_direction(self.state, idx, out, stream)
         return out
+
+    def timeout_site(self):
+        return malt_debug_timeout_site(self.state)
+
+    def set_ns_schedule(self, schedule: int):
+        malt_set_ns_schedule(self.state, schedule)
 
     def profile(self, enable: bool = True):
         malt_profile_enable(self.state, enable)
