@@ -299,27 +299,30 @@ def run_malt(args):
     t_ms = max_over_ranks(e0.elapsed_time(e1), dev)
     value = world * args.steps / (t_ms / 1e3)
 
-    # ---- the same step with the phased Newton-Schulz schedule (one launch
-    # per product) for comparison with the persistent default.
+    # ---- the same step with each Newton-Schulz schedule forced (one launch
+    # per product, or one persistent launch for all products), for
+    # comparison with the default, which picks one per launch group.
     sched = None
     if not args.no_muon:
-        opt.set_ns_schedule(malt.MALT_NS_PHASED)
-        for _ in range(2):
-            opt.step(hp, malter=malter)
-        torch.cuda.synchronize()
-        barrier()
-        p0 = torch.cuda.Event(enable_timing=True)
-        p1 = torch.cuda.Event(enable_timing=True)
-        p0.record(stream)
-        for _ in range(args.steps):
-            opt.step(hp, malter=malter)
-        p1.record(stream)
-        torch.cuda.synchronize()
-        tp = max_over_ranks(p0.elapsed_time(p1), dev) / args.steps
-        opt.set_ns_schedule(malt.MALT_NS_PERSISTENT)
-        if opt.check() != malt.MALT_OK:
-            raise SystemExit("phased-schedule step failed")
-        sched = {"persistent_ms_per_step": t_ms / args.steps, "phased_ms_per_step": tp}
+        sched = {"default": "auto (persistent for shallow products, phased for deep ones)",
+                 "default_ms_per_step": t_ms / args.steps}
+        for name, code in (("phased", malt.MALT_NS_PHASED), ("persistent", malt.MALT_NS_PERSISTENT)):
+            opt.set_ns_schedule(code)
+            for _ in range(2):
+                opt.step(hp, malter=malter)
+            torch.cuda.synchronize()
+            barrier()
+            p0 = torch.cuda.Event(enable_timing=True)
+            p1 = torch.cuda.Event(enable_timing=True)
+            p0.record(stream)
+            for _ in range(args.steps):
+                opt.step(hp, malter=malter)
+            p1.record(stream)
+            torch.cuda.synchronize()
+            sched[f"{name}_ms_per_step"] = max_over_ranks(p0.elapsed_time(p1), dev) / args.steps
+            if opt.check() != malt.MALT_OK:
+                raise SystemExit(f"{name}-schedule step failed")
+        opt.set_ns_schedule(malt.MALT_NS_AUTO)
 
     # ---- the same engine as Muon (identity preconditioners, no statistics):
     # the optimizer-only counterpart of the paper's MALT-vs-Muon overhead table.
@@ -391,8 +394,11 @@ def run_malt(args):
     traffic = ncu_traffic_per_launch()
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "traffic": traffic,
-                "kernel": "ns_gemm_kernel<persistent> (every Gram, Poly and BX product "
-                          "of the k iterations in one launch)",
+                "kernel": ("ns_gemm_kernel, persistent schedule (every Gram, Poly and BX "
+                           "product of the k iterations in one launch)"
+                           if prof["ns_persistent"][1] > 0 else
+                           "ns_gemm_kernel, phased schedule (one launch per Gram, Poly and BX "
+                           "product)"),
                 "peak_source": f"{pk_src}: bf16_tflops_sustained",
                 "flops_per_step": wl.ns_flops_min(),
                 "flops_counted": "3p^2q + p^3 per matrix and NS iteration (symmetric Gram and polynomial)",

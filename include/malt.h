@@ -216,19 +216,23 @@ int malt_profile_read(malt_state_t* st, double* ms_out, int64_t* launches_out, i
 
 /* Newton-Schulz schedule of a state (the Orth step of Algorithm 1: k
  * iterations of A = X X^T, B' = aI + bA + cA^2, X <- B' X per matrix).
- *   MALT_NS_PERSISTENT (default): one persistent launch per group of up to 8
- *     shape classes runs every product of every iteration.  Tiles are claimed
+ *   MALT_NS_PERSISTENT: one persistent launch per group of up to 8 shape
+ *     classes runs every product of every iteration.  Tiles are claimed
  *     dynamically in product order; a tile of matrix j waits on the device
  *     (bounded) only until the previous product of matrix j is stored, so
  *     one matrix's next product overlaps another matrix's current one and
  *     there is no launch gap or wave tail between products.
  *   MALT_NS_PHASED: one launch per product (3 k launches per group), each
  *     product over all matrices finished before the next starts.
- * Both compute every tile with the same arithmetic: results are bitwise
+ *   MALT_NS_AUTO (default): per group, persistent when a Gram product has
+ *     fewer tiles than 16 waves of the resident CTA pairs (shallow products,
+ *     where tails and launch gaps weigh most), phased otherwise.
+ * All compute every tile with the same arithmetic: results are bitwise
  * identical.  Takes effect at the next step.  MALT_ERR_INVALID_ARG for a
  * null state or an unknown schedule. */
 #define MALT_NS_PHASED     0
 #define MALT_NS_PERSISTENT 1
+#define MALT_NS_AUTO       2
 int malt_set_ns_schedule(malt_state_t* st, int32_t schedule);
 
 /* Host only (no GPU, no CUDA call): the persistent schedule's work list for

@@ -126,7 +126,7 @@ struct malt_state {
     std::vector<NsParams> ns_groups;
     uint32_t* d_sched = nullptr;
     int sched_groups_pad = 0;
-    int ns_schedule = MALT_NS_PERSISTENT;
+    int ns_schedule = MALT_NS_AUTO;
     int32_t last_timeout[5] = {};   // site record of the last timeout malt_check reported
     cudaStream_t last_stream = nullptr;
     // Profiling: event pairs recorded around launches, folded in on read.
@@ -236,6 +236,9 @@ struct LaunchScope {
 };
 
 constexpr int kMaxNsSteps = 64;
+// Auto schedule: persistent when a symmetric product has fewer tiles than
+// this many waves of the resident CTA pairs.
+constexpr int kAutoPersistentWaves = 16;
 constexpr int kStatusWords = 8;
 
 // Per-matrix descriptions and shape classes (one per NS frame p x q, in order
@@ -514,24 +517,35 @@ int run_newton_schulz(malt_state* st, const malt_hparams_t* hp, cudaStream_t s) 
         P.b = hp->ns_b;
         P.c = hp->ns_c;
     };
-    if (st->ns_schedule == MALT_NS_PERSISTENT) {
-        LaunchScope ls(st, MALT_KIND_NS_PERSISTENT, s, static_cast<int>(st->ns_groups.size()));
+    // Auto: the persistent schedule where a product is only a few waves of
+    // CTA pairs deep (there the tails and launch gaps between products are a
+    // large share of the time), the phased one where products are deep.
+    auto persistent = [&](const NsParams& G) {
+        if (st->ns_schedule != MALT_NS_AUTO) return st->ns_schedule == MALT_NS_PERSISTENT;
+        return G.sym_items < kAutoPersistentWaves * max_pairs;
+    };
+    bool any_persistent = false;
+    for (const NsParams& G : st->ns_groups) any_persistent |= persistent(G);
+    if (any_persistent) {
+        LaunchScope ls(st, MALT_KIND_NS_PERSISTENT, s, 0);   // launches counted below
         const size_t counters = st->sched_groups_pad + static_cast<size_t>(3 * k) * st->nmat;
         MALT_CUDA(cudaMemsetAsync(st->d_sched, 0, counters * sizeof(uint32_t), s),
                   "cudaMemsetAsync(schedule counters)");
         for (const NsParams& G : st->ns_groups) {
+            if (!persistent(G)) continue;
             prepare(G);
             const int items = k * (2 * G.sym_items + G.full_items);
             P.item_begin = 0;
             P.item_end = items;
             const int pairs = std::max(1, std::min(items, max_pairs));
+            ++st->prof_launches[MALT_KIND_NS_PERSISTENT];
             MALT_CUDA(launch_ns_gemm(P, true, pairs, s), "ns_gemm_kernel (persistent)");
         }
-        return MALT_OK;
     }
     for (int it = 0; it < k; ++it) {
         for (int phase = kGram; phase <= kBX; ++phase) {
             for (const NsParams& G : st->ns_groups) {
+                if (persistent(G)) continue;
                 prepare(G);
                 const int per_iter = 2 * G.sym_items + G.full_items;
                 const int begin = it * per_iter + (phase == kGram ? 0
@@ -905,7 +919,8 @@ int malt_debug_timeout_site(const malt_state_t* st, int32_t* out5) {
 }
 
 int malt_set_ns_schedule(malt_state_t* st, int32_t schedule) {
-    if (st == nullptr || (schedule != MALT_NS_PHASED && schedule != MALT_NS_PERSISTENT))
+    if (st == nullptr ||
+        (schedule != MALT_NS_PHASED && schedule != MALT_NS_PERSISTENT && schedule != MALT_NS_AUTO))
         return MALT_ERR_INVALID_ARG;
     st->ns_schedule = schedule;
     return MALT_OK;

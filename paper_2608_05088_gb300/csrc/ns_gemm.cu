@@ -46,18 +46,20 @@
 // of every product of every NS iteration, product by product.
 //  * Phased: one launch per product (Gram, Poly, BX of one iteration); pair
 //    j takes items j, j + npairs, ...  The stream orders the products.
-//  * Persistent: one launch for all k iterations.  The even CTA's producer
-//    claims the next item with an atomic on a global counter and hands it to
-//    the other roles of both CTAs through an 8-slot ring in shared memory
-//    (mbarrier-guarded; the peer's copy written through shared::cluster).
-//    Each product of a matrix depends only on the previous product of the
-//    same matrix, so a tile waits (bounded, acquire) until every epilogue
+//  * Persistent: one launch for all k iterations.  A scheduler thread per
+//    pair (the odd CTA's otherwise idle MMA-warp thread) claims the next
+//    item with an atomic on a global counter, waits (bounded, acquire) until
+//    the previous product of the item's matrix is complete -- every epilogue
 //    warp of every tile of that product has signalled done[] after its TMA
-//    stores completed.  Tiles of the next product of one matrix start while
-//    the current product of another matrix is still running: no grid-wide
-//    barrier between products, no launch gaps, no wave tails except the
-//    last.  Items are claimed in list order by running CTAs only, so every
-//    item a tile waits for is held by a CTA that is running and whose own
+//    stores completed -- and publishes the item to a 4-slot ring in both
+//    CTAs' shared memory (st.async messages on mbarriers), a few items ahead
+//    of the producers, MMA and epilogues that read it.  Each product of a
+//    matrix depends only on the previous product of the same matrix, so
+//    tiles of the next product of one matrix start while the current
+//    product of another matrix is still running: no grid-wide barrier
+//    between products, no launch gaps, no wave tails except the last.
+//    Items are claimed in list order by running CTAs only, so every item a
+//    tile waits for is held by a CTA that is running and whose own
 //    dependencies come earlier still: the schedule cannot deadlock, whatever
 //    number of CTA pairs is resident.
 //  Both schedules run the same per-tile arithmetic, so their results are
@@ -93,11 +95,12 @@ constexpr uint32_t kStageOutBytes = 2 * kStoreBoxBytes * kEpiWarps;  // double-b
 constexpr size_t kSmemBytes =
     static_cast<size_t>(kStages) * kStageBytes + kStageOutBytes + 1024;
 constexpr uint16_t kPairMask = 0x3;
-// Persistent schedule: slots of the item ring, and the readers of each slot
-// besides the even CTA's producer that fills it (the even CTA's MMA thread,
-// the odd CTA's producer, every epilogue warp of both CTAs).
-constexpr int kItemSlots = 8;
-constexpr uint32_t kItemReaders = 2 + 2 * kEpiWarps;
+// Persistent schedule: slots of the item ring (how far the scheduler may run
+// ahead of the slowest reader, the epilogue), and the readers of each slot:
+// both producers, the even CTA's MMA thread, every epilogue warp of both CTAs.
+constexpr int kItemSlots = 4;
+constexpr int kNoItem = -0x7fffffff;   // never stored in the ring
+constexpr uint32_t kItemReaders = 3 + 2 * kEpiWarps;
 static_assert(2 * kEpiWarps == static_cast<int>(kNsSignalsPerTile),
               "every epilogue warp of the pair signals a finished tile once");
 
@@ -165,14 +168,13 @@ __device__ __forceinline__ uint4 pack8(const float* v) {
 
 // Where a wait gave up (recorded once per status word, for malt_debug_timeout_site).
 enum WaitSite : int32_t {
-    kSiteClaim = 1,      // even producer: a ring slot to become free
-    kSiteDepLoad = 2,    // producer: the previous product of the matrix
+    kSiteClaim = 1,      // scheduler: a ring slot to become free
+    kSiteDepLoad = 2,    // scheduler: the previous product of the item's matrix
     kSiteStage = 3,      // producer: a free operand stage
     kSiteItem = 4,       // ring reader: the next item (+ 16 * role)
     kSiteAccFree = 5,    // MMA: a free accumulator
     kSiteStageFull = 6,  // MMA: operands of a stage
     kSiteAccFull = 7,    // epilogue: a finished accumulator
-    kSiteDepEpi = 8,     // epilogue: the Gram product (polynomial epilogue)
     kSiteDrain = 9,      // MMA: the last MMAs before TMEM is freed
 };
 
@@ -275,8 +277,8 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
     const uint32_t tmem_base = tmem_slot;
 
     // Item number `seq` of this pair.  Phased: static round-robin.  Persistent:
-    // read from the ring (-2 when the wait gave up); only the even CTA's
-    // producer claims items (claim_item).
+    // read from the ring (-2 when the wait gave up), which the scheduler
+    // thread of the odd CTA fills (claim_next, publish_item).
     auto static_item = [&](int seq) -> int {
         const long long it = static_cast<long long>(P.item_begin) + pair +
                              static_cast<long long>(seq) * npairs;
@@ -287,21 +289,35 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
         const uint32_t par = static_cast<uint32_t>(seq / kItemSlots) & 1u;
         if (!mbar_wait_cluster_bounded(&item_full[slot], par, budget, abort_flag)) return -2;
         const int item = *reinterpret_cast<volatile int32_t*>(&item_ring[slot]);
-        mbar_arrive_cluster(mapa_shared(smem_u32(&item_empty[slot]), 0));
+        // Free the slot (its barrier lives in the odd CTA, with the
+        // scheduler).  The arrive carries no data, so it is relaxed; it is
+        // issued only once the slot's value is in hand (the branch depends on
+        // it), so the scheduler cannot overwrite the slot before this read.
+        if (item != kNoItem) mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&item_empty[slot]), 1));
         return item;
     };
-    auto claim_item = [&](int seq) -> int {
+    // Scheduler (odd CTA): claim the next item index (-1 past the end), and
+    // publish an item to the ring slot of sequence number seq in both CTAs
+    // (false when the slot did not come free in time).
+    auto claim_next = [&]() -> int {
+        const uint32_t claimed = atomicAdd(P.queue, 1u);
+        return claimed < static_cast<uint32_t>(P.item_end - P.item_begin)
+                   ? P.item_begin + static_cast<int>(claimed) : -1;
+    };
+    auto publish_item = [&](int seq, int item) -> bool {
         const int slot = seq % kItemSlots;
         const uint32_t par = static_cast<uint32_t>(seq / kItemSlots) & 1u;
-        if (!mbar_wait_cluster_bounded(&item_empty[slot], par ^ 1u, budget, abort_flag)) return -2;
-        const uint32_t claimed = atomicAdd(P.queue, 1u);
-        const int item = claimed < static_cast<uint32_t>(P.item_end - P.item_begin)
-                             ? P.item_begin + static_cast<int>(claimed) : -1;
-        *reinterpret_cast<volatile int32_t*>(&item_ring[slot]) = item;
-        st_cluster_u32(mapa_shared(smem_u32(&item_ring[slot]), 1), static_cast<uint32_t>(item));
-        mbar_arrive_cluster(mapa_shared(smem_u32(&item_full[slot]), 0));
-        mbar_arrive_cluster(mapa_shared(smem_u32(&item_full[slot]), 1));
-        return item;
+        if (!mbar_wait_cluster_bounded(&item_empty[slot], par ^ 1u, budget, abort_flag)) return false;
+        // The item travels as an asynchronous store that completes on the
+        // slot's full barrier in each CTA.  The arrive releases at cluster
+        // scope what this thread acquired from the dependency counter, so a
+        // reader that sees the item also sees the operands the item reads.
+        for (uint32_t r = 0; r < 2; ++r) {
+            const uint32_t bar = mapa_shared(smem_u32(&item_full[slot]), r);
+            mbar_arrive_expect_tx_cluster(bar, 4u);
+            st_async_u32(mapa_shared(smem_u32(&item_ring[slot]), r), static_cast<uint32_t>(item), bar);
+        }
+        return true;
     };
 
     if (warp == 0) {
@@ -309,22 +325,15 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
         if (lane == 0) {
             uint32_t stage = 0, phase = 0;
             for (int seq = 0;; ++seq) {
-                const int item = !kPersistent ? static_item(seq)
-                                 : leader     ? claim_item(seq)
-                                              : read_item(seq);
+                const int item = kPersistent ? read_item(seq) : static_item(seq);
                 if (item == -2) {
-                    raise_timeout(P, abort_flag, leader ? kSiteClaim : kSiteItem, -2, seq);
+                    raise_timeout(P, abort_flag, kSiteItem, -2, seq);
                     break;
                 }
                 if (item < 0) break;
+                // The loads below read what other CTAs stored in this launch.
+                if (kPersistent) fence_proxy_async_global();
                 const NsWork w = ns_decode(P, item);
-                if (kPersistent) {
-                    if (!wait_dependency(P, w, abort_flag)) {
-                        raise_timeout(P, abort_flag, kSiteDepLoad, item, seq);
-                        break;
-                    }
-                    fence_proxy_async_global();   // the loads below read what other CTAs stored
-                }
                 const Ops op = item_operands(P, w);
                 const bool b_mn = w.kind == kBX;
                 const int nkb = (op.K + kBK - 1) / kBK;
@@ -352,13 +361,34 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                     } else if (nb_self > 0) {
                         tma_load_3d_pair(sa + kABytes, op.b, kb * kBK, n0, w.b, fb);
                     }
-                    if (!leader) mbar_arrive_cluster(fb);
+                    if (!leader) mbar_arrive_cluster_relaxed(fb);
                     if (++stage == kStages) { stage = 0; phase ^= 1u; }
                 }
                 if (!ok) break;
             }
         }
     } else if (warp == 1) {
+        if (kPersistent && lane == 0 && !leader) {
+            // ------------------------------------------ scheduler (odd CTA)
+            // Claim items in list order, one ahead; publish each once the
+            // previous product of its matrix is stored, up to kItemSlots
+            // ahead of the slowest reader.  Waiting here keeps the acquire
+            // round trip off the producers' path.
+            int next = claim_next();
+            for (int seq = 0;; ++seq) {
+                const int item = next;
+                if (item >= 0 && !wait_dependency(P, ns_decode(P, item), abort_flag)) {
+                    raise_timeout(P, abort_flag, kSiteDepLoad, item, seq);
+                    break;
+                }
+                if (!publish_item(seq, item)) {
+                    raise_timeout(P, abort_flag, kSiteClaim, item, seq);
+                    break;
+                }
+                if (item < 0) break;
+                next = claim_next();
+            }
+        }
         // ------------------------------------------- MMA issuer (even CTA)
         if (lane == 0 && leader) {
             uint32_t stage = 0, phase = 0;
@@ -460,15 +490,6 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
             const __nv_bfloat16* ein =
                 need_ein ? C.A + static_cast<size_t>(w.b) * C.p * C.p : nullptr;
             const bool last_bx = (w.kind == kBX) && (w.iter == P.ns_steps - 1);
-            if (kPersistent && need_ein) {
-                // The polynomial epilogue reads A directly: acquire the Gram
-                // product's completion (already reached: the producer waited
-                // for it before loading this tile's operands).
-                if (!wait_dependency(P, w, abort_flag)) {
-                    raise_timeout(P, abort_flag, kSiteDepEpi, item, seq);
-                    break;
-                }
-            }
             // NS frame row / column scalings of D = L O R (swapped when transposed).
             const float* uvec = md.trans ? md.R : md.L;
             const float* vvec = md.trans ? md.L : md.R;

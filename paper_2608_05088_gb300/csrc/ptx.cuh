@@ -91,6 +91,13 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
                  ::"r"(cluster_addr) : "memory");
 }
 
+// Arrive without release semantics: only the phase count matters (the data
+// the phase guards arrives through transaction bytes, not through this thread).
+__device__ __forceinline__ void mbar_arrive_cluster_relaxed(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];"
+                 ::"r"(cluster_addr) : "memory");
+}
+
 __device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
@@ -115,6 +122,29 @@ __device__ __forceinline__ bool mbar_wait_cluster_bounded(uint64_t* bar, uint32_
             if (globaltimer_ns() - t0 > budget_ns) return false;
         }
     }
+}
+
+// Asynchronous 32-bit store into shared memory of a CTA of the cluster that
+// completes 4 transaction bytes on an mbarrier of that CTA (both given by
+// shared::cluster addresses): a message whose arrival the barrier reports,
+// with no fence on the sending thread.
+__device__ __forceinline__ void st_async_u32(uint32_t cluster_addr, uint32_t v, uint32_t cluster_bar) {
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.u32 [%0], %1, [%2];"
+                 ::"r"(cluster_addr), "r"(v), "r"(cluster_bar) : "memory");
+}
+
+// Arrive (release, cluster scope) that also expects `bytes` transaction bytes
+// on the phase.
+__device__ __forceinline__ void mbar_arrive_expect_tx_cluster(uint32_t cluster_bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.release.cluster.shared::cluster.b64 _, [%0], %1;"
+                 ::"r"(cluster_bar), "r"(bytes) : "memory");
+}
+
+// Relaxed arrive that also expects `bytes` transaction bytes on the phase.
+__device__ __forceinline__ void mbar_arrive_expect_tx_cluster_relaxed(uint32_t cluster_bar,
+                                                                      uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.relaxed.cluster.shared::cluster.b64 _, [%0], %1;"
+                 ::"r"(cluster_bar), "r"(bytes) : "memory");
 }
 
 // 32-bit store into shared memory of a CTA of the cluster (shared::cluster address).
@@ -155,6 +185,25 @@ __device__ __forceinline__ bool counter_wait_bounded(const uint32_t* ctr, uint32
             if (abort_flag != nullptr && *abort_flag) return false;
             if (status != nullptr && (*reinterpret_cast<const volatile int32_t*>(status) & abort_bits))
                 return false;
+            if (globaltimer_ns() - t0 > budget_ns) return false;
+        }
+    }
+}
+
+// As mbar_wait_cluster_bounded for waits off the critical path: between
+// polls the thread sleeps for about sleep_ns, so it neither competes for
+// issue slots nor for the shared-memory port of the CTA it polls in.
+__device__ __forceinline__ bool mbar_wait_cluster_bounded_sleep(uint64_t* bar, uint32_t parity,
+                                                                uint64_t budget_ns,
+                                                                volatile int* abort_flag,
+                                                                uint32_t sleep_ns) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t it = 1;; ++it) {
+        __nanosleep(sleep_ns);
+        if (mbar_try_wait_cluster(bar, parity)) return true;
+        if ((it & 15u) == 0u) {
+            if (abort_flag != nullptr && *abort_flag) return false;
             if (globaltimer_ns() - t0 > budget_ns) return false;
         }
     }

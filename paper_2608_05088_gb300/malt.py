@@ -40,6 +40,7 @@ NS_KINDS = ("ns_gram", "ns_poly", "ns_bx", "ns_persistent")
 # Newton-Schulz schedules (malt_set_ns_schedule)
 MALT_NS_PHASED = 0
 MALT_NS_PERSISTENT = 1
+MALT_NS_AUTO = 2
 
 
 class malt_param_t(ctypes.Structure):
