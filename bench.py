@@ -267,6 +267,9 @@ def run_malt(args):
     hp = malt.hparams(lr=wl.lr, ns_steps=wl.ns_steps)
     malter = wl.variant == "malter"
     stream = torch.cuda.current_stream()
+    sched_code = {"auto": malt.MALT_NS_AUTO, "phased": malt.MALT_NS_PHASED,
+                  "persistent": malt.MALT_NS_PERSISTENT}[args.ns_schedule]
+    opt.set_ns_schedule(sched_code)
 
     for _ in range(args.warmup):
         opt.step(hp, malter=malter)
@@ -304,8 +307,9 @@ def run_malt(args):
     # comparison with the default, which picks one per launch group.
     sched = None
     if not args.no_muon:
-        sched = {"default": "auto (persistent for shallow products, phased for deep ones)",
-                 "default_ms_per_step": t_ms / args.steps}
+        sched = {"timed": args.ns_schedule + (" (persistent for shallow products, phased for "
+                                              "deep ones)" if args.ns_schedule == "auto" else ""),
+                 "timed_ms_per_step": t_ms / args.steps}
         for name, code in (("phased", malt.MALT_NS_PHASED), ("persistent", malt.MALT_NS_PERSISTENT)):
             opt.set_ns_schedule(code)
             for _ in range(2):
@@ -322,7 +326,7 @@ def run_malt(args):
             sched[f"{name}_ms_per_step"] = max_over_ranks(p0.elapsed_time(p1), dev) / args.steps
             if opt.check() != malt.MALT_OK:
                 raise SystemExit(f"{name}-schedule step failed")
-        opt.set_ns_schedule(malt.MALT_NS_AUTO)
+        opt.set_ns_schedule(sched_code)
 
     # ---- the same engine as Muon (identity preconditioners, no statistics):
     # the optimizer-only counterpart of the paper's MALT-vs-Muon overhead table.
@@ -430,7 +434,8 @@ def run_malt(args):
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_ms / args.steps,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-           "dtype": "bf16", "data": "synthetic", "config": workload_config(wl),
+           "dtype": "bf16", "data": "synthetic",
+           "config": dict(workload_config(wl), ns_schedule=args.ns_schedule),
            "clocks": clk, "e2e": e2e, "gpu_launches": launches, "roofline": roofline,
            "hbm_kernels": mem, "ms_per_step_by_kernel": breakdown,
            "cpu_baseline": cpu, "muon_same_engine": muon, "ns_schedules": sched,
@@ -449,6 +454,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-muon", action="store_true")
+    ap.add_argument("--ns-schedule", choices=("auto", "phased", "persistent"), default="auto",
+                    help="Newton-Schulz schedule of the timed steps (default: the library's auto)")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling only: the first N layers of the workload")
     args = ap.parse_args()

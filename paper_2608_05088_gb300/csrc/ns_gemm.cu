@@ -504,9 +504,15 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                 const int col0 = col_base + ch * 32;
 #pragma unroll
                 for (int q8 = 0; q8 < 4; ++q8) {
-                    if (rok && col0 + q8 * 8 < N)
-                        dst[q8] = __ldcg(reinterpret_cast<const uint4*>(
-                            ein + static_cast<size_t>(row) * N + col0 + q8 * 8));
+                    if (rok && col0 + q8 * 8 < N) {
+                        const uint4* src = reinterpret_cast<const uint4*>(
+                            ein + static_cast<size_t>(row) * N + col0 + q8 * 8);
+                        // Phased: A was written by an earlier launch, so the
+                        // read-only path is safe.  Persistent: A is rewritten
+                        // each iteration inside this launch; a coherent load
+                        // (ordered by the ring's acquire) is required.
+                        dst[q8] = kPersistent ? *src : __ldg(src);
+                    }
                     else
                         dst[q8] = make_uint4(0u, 0u, 0u, 0u);
                 }
