@@ -141,9 +141,10 @@ def peaks():
         return FALLBACK_PEAKS, "fallback"
 
 
-def ncu_traffic_per_launch():
-    """DRAM bytes per NS GEMM launch from the committed ncu summary, or None
-    when the kernel source changed since the capture."""
+def ncu_traffic_per_launch(persistent: bool):
+    """DRAM bytes per NS GEMM launch (of the schedule the timed steps used)
+    from the committed ncu summary, or None when the kernel source changed
+    since the capture."""
     try:
         with open(NCU_SUMMARY) as f:
             s = json.load(f)
@@ -151,7 +152,9 @@ def ncu_traffic_per_launch():
             h = hashlib.sha256(f.read()).hexdigest()
         if s.get("ns_gemm_sha256") != h:
             return None
-        return float(s["dram_bytes_per_launch_full_size"])
+        key = "persistent_dram_bytes_per_launch_full_size" if persistent else \
+              "dram_bytes_per_launch_full_size"
+        return float(s[key])
     except Exception:
         return None
 
@@ -395,7 +398,10 @@ def run_malt(args):
     achieved = flops / (ns_ms / 1e3) / 1e12
     dense_equiv = wl.ns_flops_dense() * args.steps / (ns_ms / 1e3) / 1e12
     peak = float(pk["bf16_tflops_sustained"])
-    traffic = ncu_traffic_per_launch()
+    persistent_timed = prof["ns_persistent"][1] > 0 and prof["ns_bx"][1] == 0
+    # the committed capture is of the 144-matrix GPT-2 Large set only
+    traffic = ncu_traffic_per_launch(persistent_timed) if (
+        wl.name == "gpt2_large" and not args.layers) else None
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "traffic": traffic,
                 "kernel": ("ns_gemm_kernel, persistent schedule (every Gram, Poly and BX "
