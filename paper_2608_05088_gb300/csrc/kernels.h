@@ -11,6 +11,7 @@ struct BindParams {
     UserPtrs p[kBindChunk];
     int32_t count;
     int32_t offset;
+    long long* tcount;   // when set, the launch also adds 1 to the step counter
 };
 
 cudaError_t launch_bind(const BindParams& P, UserPtrs* table, cudaStream_t s);

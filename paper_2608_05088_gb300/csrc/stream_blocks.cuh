@@ -1,0 +1,535 @@
+// stream_blocks.cuh -- the HBM-bound stages of the MALT / MALTER step as
+// block-level device functions of 256 threads (tid 0..255).  The standalone
+// kernels of stream_kernels.cu run one call per CUDA block; the fused step
+// kernel (ns_gemm.cu) runs the same calls on the 8 epilogue warps of a CTA,
+// between Newton-Schulz tiles.  Both run the same arithmetic in the same
+// order, so a step gives bitwise the same result either way.
+//
+//   stats     Algorithm 1, M_t / l_t / r_t lines: one pass over G and M that
+//             updates the momentum and writes per-tile partial sums of G^2 for
+//             every row and every column (eq. dp_preconditioner).
+//   finalize  l, r EMAs from the partials and L = (l+eps)^(-1/8),
+//             R = (r+eps)^(-1/8) (Algorithm 1, L_t / R_t line).
+//   prescale  Mt = L M R (Algorithm 1, Mt line), written as bf16 in the
+//             Newton-Schulz frame (transposed when m > n), with partial sums
+//             of Mt^2 (and of (L G R)^2 for MALTER, Algorithm 2 nu_t line).
+//   norms     ||Mt||_F and ||L G R||_F^2 per matrix from those partials.
+//   scalars   ||O||_F, ||D||_F, MALTER's nu and alpha (Section 3.5) and the
+//             grafted scale lr * alpha * ||O|| / (||D|| + eps) per matrix.
+//   apply     W <- (1 - lr wd) W - scale * L O R (Algorithm 1, W_t line).
+//
+// Template flag kRO: the block may read O through the read-only cache path.
+// True in the standalone kernels (O was written by an earlier launch); false
+// in the fused kernel, which writes O itself.
+#pragma once
+#include <cuda_bf16.h>
+#include <cstdint>
+
+#include "common.cuh"
+
+namespace malt {
+namespace blk {
+
+constexpr int kThreads = 256;
+
+// Block-wide barrier of the threads running a block function.
+struct SyncBlock {
+    __device__ __forceinline__ void operator()() const { __syncthreads(); }
+};
+// The 8 epilogue warps of a CTA of the fused kernel (named barrier 1).
+struct SyncEpilogue {
+    __device__ __forceinline__ void operator()() const {
+        asm volatile("bar.sync 1, 256;" ::: "memory");
+    }
+};
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Sum of v over the first nthreads threads (a multiple of 32) in a fixed
+// order; every thread of the block calls it, the result is valid in tid 0.
+template <class Sync>
+__device__ __forceinline__ float block_sum(float v, float* sh /* >= 32 */, int tid, int nthreads,
+                                           Sync sync) {
+    v = warp_sum(v);
+    const int w = tid >> 5, lane = tid & 31;
+    if (lane == 0 && tid < nthreads) sh[w] = v;
+    sync();
+    float s = 0.f;
+    if (tid == 0) {
+        const int nw = nthreads >> 5;
+        for (int i = 0; i < nw; ++i) s += sh[i];
+    }
+    sync();
+    return s;
+}
+
+template <bool kRO>
+__device__ __forceinline__ uint4 ld_u4(const void* p) {
+    return kRO ? __ldg(reinterpret_cast<const uint4*>(p)) : *reinterpret_cast<const uint4*>(p);
+}
+
+// 8 consecutive elements (bf16 or fp32) at element offset off, as floats.
+template <bool kRO = true>
+__device__ __forceinline__ void load8(const void* base, bool bf16, size_t off, float (&v)[8]) {
+    if (bf16) {
+        const uint4 u = ld_u4<kRO>(static_cast<const __nv_bfloat16*>(base) + off);
+        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float2 f = __bfloat1622float2(h[k]);
+            v[2 * k] = f.x;
+            v[2 * k + 1] = f.y;
+        }
+    } else {
+        const float4* p = reinterpret_cast<const float4*>(static_cast<const float*>(base) + off);
+        float4 a, b;
+        if (kRO) {
+            a = __ldg(p);
+            b = __ldg(p + 1);
+        } else {
+            a = p[0];
+            b = p[1];
+        }
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+        v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    }
+}
+
+__device__ __forceinline__ uint4 pack8_bf16(const float (&v)[8]) {
+    uint4 u;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&u);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) h[k] = __floats2bfloat162_rn(v[2 * k], v[2 * k + 1]);
+    return u;
+}
+
+// ------------------------------------------------------------------ stats
+// Block `local` = kStatRows x kStatCols of W: warp w owns 8 rows, lane owns 8
+// consecutive columns.  Row sums reduce across the warp; column sums
+// accumulate in registers over the warp's rows, then across the 8 warps in
+// shared memory (colsh: 8 x kStatCols floats).  kStats = false (Muon through
+// the same engine): momentum only.  G is never written by the library, so it
+// is read through the read-only path.
+constexpr int kStatRowsPerWarp = kStatRows / 8;
+constexpr int kStatBatch = 4;
+
+template <bool kStats, class Sync>
+__device__ __forceinline__ void stats_block(const MatDesc& d, const UserPtrs& up, int local,
+                                            float mu1, int tid, float* colsh, Sync sync) {
+    const int m = d.m, n = d.n;
+    const int rb = local / d.stat_cb, cb = local - rb * d.stat_cb;
+    const int warp = tid >> 5, lane = tid & 31;
+    const int col = cb * kStatCols + lane * 8;
+    const bool colok = col < n;
+    const int row0 = rb * kStatRows + warp * kStatRowsPerWarp;
+    const bool gbf = d.g_bf16 != 0;
+    float* __restrict__ Mp = up.m;
+    const float om = 1.f - mu1;
+
+    float csum[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) csum[j] = 0.f;
+    float myrow = 0.f;
+
+#pragma unroll
+    for (int rb4 = 0; rb4 < kStatRowsPerWarp; rb4 += kStatBatch) {
+        float gv[kStatBatch][8], mv[kStatBatch][8];
+        bool ok[kStatBatch];
+#pragma unroll
+        for (int u = 0; u < kStatBatch; ++u) {
+            const int row = row0 + rb4 + u;
+            ok[u] = colok && row < m;
+            if (ok[u]) {
+                const size_t off = static_cast<size_t>(row) * n + col;
+                load8<true>(up.g, gbf, off, gv[u]);
+                const float4* mp = reinterpret_cast<const float4*>(Mp + off);
+                const float4 a = mp[0], b = mp[1];
+                mv[u][0] = a.x; mv[u][1] = a.y; mv[u][2] = a.z; mv[u][3] = a.w;
+                mv[u][4] = b.x; mv[u][5] = b.y; mv[u][6] = b.z; mv[u][7] = b.w;
+            } else {
+#pragma unroll
+                for (int j = 0; j < 8; ++j) { gv[u][j] = 0.f; mv[u][j] = 0.f; }
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kStatBatch; ++u) {
+            float rs = 0.f;
+            float nm[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const float gj = gv[u][j];
+                nm[j] = fmaf(mu1, mv[u][j], om * gj);
+                const float sq = gj * gj;
+                rs += sq;
+                csum[j] += sq;
+            }
+            if (ok[u]) {
+                const size_t off = static_cast<size_t>(row0 + rb4 + u) * n + col;
+                float4* mp = reinterpret_cast<float4*>(Mp + off);
+                mp[0] = make_float4(nm[0], nm[1], nm[2], nm[3]);
+                mp[1] = make_float4(nm[4], nm[5], nm[6], nm[7]);
+            }
+            if (kStats) {
+                rs = warp_sum(rs);
+                if (lane == rb4 + u) myrow = rs;
+            }
+        }
+    }
+    if (!kStats) return;
+    if (lane < kStatRowsPerWarp && row0 + lane < m)
+        d.rowpart[static_cast<size_t>(cb) * m + row0 + lane] = myrow;
+
+    float4* cs = reinterpret_cast<float4*>(colsh + warp * kStatCols + lane * 8);
+    cs[0] = make_float4(csum[0], csum[1], csum[2], csum[3]);
+    cs[1] = make_float4(csum[4], csum[5], csum[6], csum[7]);
+    sync();
+    const int c = tid;
+    const int gc = cb * kStatCols + c;
+    if (gc < n) {
+        float s = 0.f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) s += colsh[w * kStatCols + c];
+        d.colpart[static_cast<size_t>(rb) * n + gc] = s;
+    }
+}
+
+// --------------------------------------------------------------- finalize
+// Entry `local` of the matrix's m + n statistics: row i = local (< m) or
+// column j = local - m.  identity (Muon): L = R = 1, statistics untouched.
+__device__ __forceinline__ void finalize_entry(const MatDesc& d, const UserPtrs& up, int local,
+                                               float mu2, float eps, int identity) {
+    if (identity) {
+        if (local < d.m) d.L[local] = 1.f; else d.R[local - d.m] = 1.f;
+        return;
+    }
+    if (local < d.m) {
+        const int i = local;
+        float s = 0.f;
+        for (int cb = 0; cb < d.stat_cb; ++cb) s += d.rowpart[static_cast<size_t>(cb) * d.m + i];
+        const float l = fmaf(mu2, up.l[i], (1.f - mu2) * s);
+        up.l[i] = l;
+        d.L[i] = powf(l + eps, -0.125f);
+    } else {
+        const int j = local - d.m;
+        float s = 0.f;
+        for (int rb = 0; rb < d.stat_rb; ++rb) s += d.colpart[static_cast<size_t>(rb) * d.n + j];
+        const float r = fmaf(mu2, up.r[j], (1.f - mu2) * s);
+        up.r[j] = r;
+        d.R[j] = powf(r + eps, -0.125f);
+    }
+}
+
+// --------------------------------------------------------------- prescale
+// Block `local` = kPreRows x kPreCols of Mt.  A wide matrix is streamed like
+// the statistics pass (warp w owns 8 rows, lane 8 consecutive columns, four
+// rows of loads in flight) and written as bf16 in place of its NS frame; a
+// tall matrix's NS frame is Mt^T, so its block walks four 64 x 64 sub-tiles
+// through shared memory (tile: 64 x 65 floats) and writes each transposed.
+// red: 8 float2.
+template <class Sync>
+__device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs& up, int local,
+                                               int malter, int tid, float (*tile)[65],
+                                               float2* red, Sync sync) {
+    const int m = d.m, n = d.n;
+    const int tr = local / d.pre_tc, tc = local - tr * d.pre_tc;
+    const int r0 = tr * kPreRows, c0 = tc * kPreCols;
+    const int t = tid, warp = t >> 5, lane = t & 31;
+    const float* __restrict__ Lv = d.L;
+    const float* __restrict__ Rv = d.R;
+    const float* __restrict__ Mp = up.m;
+    const bool gbf = d.g_bf16 != 0;
+    float s_mt = 0.f, s_lgr = 0.f;
+
+    if (!d.trans) {
+        const int col = c0 + lane * 8;
+        const bool colok = col < n;
+        float rj[8];
+        if (colok) {
+            const float4 a = *reinterpret_cast<const float4*>(Rv + col);
+            const float4 b = *reinterpret_cast<const float4*>(Rv + col + 4);
+            rj[0] = a.x; rj[1] = a.y; rj[2] = a.z; rj[3] = a.w;
+            rj[4] = b.x; rj[5] = b.y; rj[6] = b.z; rj[7] = b.w;
+        }
+        const int row0 = r0 + warp * 8;
+#pragma unroll
+        for (int rb = 0; rb < 8; rb += 4) {
+            float mv[4][8], li[4];
+            bool ok[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int row = row0 + rb + u;
+                ok[u] = colok && row < m;
+                li[u] = 0.f;
+                if (ok[u]) {
+                    const size_t off = static_cast<size_t>(row) * n + col;
+                    const float4 a = *reinterpret_cast<const float4*>(Mp + off);
+                    const float4 b = *reinterpret_cast<const float4*>(Mp + off + 4);
+                    mv[u][0] = a.x; mv[u][1] = a.y; mv[u][2] = a.z; mv[u][3] = a.w;
+                    mv[u][4] = b.x; mv[u][5] = b.y; mv[u][6] = b.z; mv[u][7] = b.w;
+                    li[u] = Lv[row];
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                if (!ok[u]) continue;
+                const int row = row0 + rb + u;
+                const size_t off = static_cast<size_t>(row) * n + col;
+                float v[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    v[j] = li[u] * mv[u][j] * rj[j];
+                    s_mt = fmaf(v[j], v[j], s_mt);
+                }
+                *reinterpret_cast<uint4*>(d.X0 + off) = pack8_bf16(v);
+                if (malter) {
+                    float gv[8];
+                    load8<true>(up.g, gbf, off, gv);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        const float a = li[u] * gv[j] * rj[j];
+                        s_lgr = fmaf(a, a, s_lgr);
+                    }
+                }
+            }
+        }
+    } else {
+        const int cc = (t & 15) * 4;
+        for (int sub = 0; sub < kPreCols / 64; ++sub) {
+            const int cs = c0 + sub * 64;
+            if (cs >= n) break;                          // uniform across the block
+            const int col = cs + cc;
+            float4 R4 = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (col < n) R4 = *reinterpret_cast<const float4*>(Rv + col);
+#pragma unroll
+            for (int pass = 0; pass < 4; ++pass) {
+                const int rr = pass * 16 + (t >> 4);
+                const int row = r0 + rr;
+                float v0 = 0.f, v1 = 0.f, v2 = 0.f, v3 = 0.f;
+                if (row < m && col < n) {
+                    const size_t off = static_cast<size_t>(row) * n + col;
+                    const float Li = Lv[row];
+                    const float4 mq = *reinterpret_cast<const float4*>(Mp + off);
+                    v0 = Li * mq.x * R4.x; v1 = Li * mq.y * R4.y;
+                    v2 = Li * mq.z * R4.z; v3 = Li * mq.w * R4.w;
+                    s_mt += v0 * v0 + v1 * v1 + v2 * v2 + v3 * v3;
+                    if (malter) {
+                        float gq[4];
+                        if (gbf) {
+                            const uint2 u = *reinterpret_cast<const uint2*>(
+                                static_cast<const __nv_bfloat16*>(up.g) + off);
+                            const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+                            const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+                            gq[0] = a.x; gq[1] = a.y; gq[2] = b.x; gq[3] = b.y;
+                        } else {
+                            const float4 gf = *reinterpret_cast<const float4*>(
+                                static_cast<const float*>(up.g) + off);
+                            gq[0] = gf.x; gq[1] = gf.y; gq[2] = gf.z; gq[3] = gf.w;
+                        }
+                        const float a0 = Li * gq[0] * R4.x, a1 = Li * gq[1] * R4.y;
+                        const float a2 = Li * gq[2] * R4.z, a3 = Li * gq[3] * R4.w;
+                        s_lgr += a0 * a0 + a1 * a1 + a2 * a2 + a3 * a3;
+                    }
+                }
+                tile[rr][cc + 0] = v0; tile[rr][cc + 1] = v1;
+                tile[rr][cc + 2] = v2; tile[rr][cc + 3] = v3;
+            }
+            sync();
+            // Output row = column of Mt, 8 consecutive rows of Mt per thread.
+#pragma unroll
+            for (int pass = 0; pass < 2; ++pass) {
+                const int oc = pass * 32 + (t >> 3);
+                const int seg = (t & 7) * 8;
+                const int gcol = cs + oc, grow = r0 + seg;
+                if (gcol < n && grow < m) {
+                    float v[8];
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) v[j] = tile[seg + j][oc];
+                    *reinterpret_cast<uint4*>(d.X0 + static_cast<size_t>(gcol) * m + grow) =
+                        pack8_bf16(v);
+                }
+            }
+            sync();                                       // tile is reused by the next sub-tile
+        }
+    }
+    // One fixed-order reduction of both partial sums.
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        s_mt += __shfl_xor_sync(0xffffffffu, s_mt, o);
+        s_lgr += __shfl_xor_sync(0xffffffffu, s_lgr, o);
+    }
+    if (lane == 0) red[warp] = make_float2(s_mt, s_lgr);
+    sync();
+    if (t == 0) {
+        float a = 0.f, b = 0.f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) {
+            a += red[w].x;
+            b += red[w].y;
+        }
+        d.prepart[2 * local + 0] = a;
+        d.prepart[2 * local + 1] = b;
+    }
+}
+
+// ------------------------------------------------------------------ norms
+// ||Mt||_F, 1 / (||Mt||_F + ns_eps) and ||L G R||_F^2 of one matrix (256 threads).
+template <class Sync>
+__device__ __forceinline__ void norms_matrix(const MatDesc& d, MatScalars* sc, float ns_eps,
+                                             int malter, int tid, float* red, Sync sync) {
+    const int tiles = d.pre_tr * d.pre_tc;
+    float a = 0.f, b = 0.f;
+    for (int i = tid; i < tiles; i += kThreads) {
+        a += d.prepart[2 * i];
+        b += d.prepart[2 * i + 1];
+    }
+    a = block_sum(a, red, tid, kThreads, sync);
+    b = block_sum(b, red, tid, kThreads, sync);
+    if (tid == 0) {
+        const float nrm = sqrtf(a);
+        sc->norm_mt = nrm;
+        sc->k = 1.f / (nrm + ns_eps);
+        sc->lgr_sq = malter ? b : 0.f;
+    }
+}
+
+// ---------------------------------------------------------------- scalars
+// Graft norms, MALTER's nu and alpha, and the applied scale of one matrix.
+// The sums run over the first kScalarThreads threads (the standalone kernel's
+// block size), so the result does not depend on who runs it.
+constexpr int kScalarThreads = 128;
+
+template <class Sync>
+__device__ __forceinline__ void scalars_matrix(const MatDesc& d, MatScalars* sc,
+                                               const long long* tcount, const StepHyper& hp,
+                                               int tid, float* red, Sync sync) {
+    float a = 0.f, b = 0.f;
+    // One partial per epilogue warp per GEMM tile of the last iteration.
+    if (tid < kScalarThreads) {
+        for (int i = tid; i < kNsPartsPerTile * d.ns_tiles; i += kScalarThreads) {
+            a += d.nspart[2 * i];
+            b += d.nspart[2 * i + 1];
+        }
+    }
+    a = block_sum(a, red, tid, kScalarThreads, sync);
+    b = block_sum(b, red, tid, kScalarThreads, sync);
+    if (tid == 0) {
+        MatScalars s = *sc;
+        const double norm_o = sqrt(static_cast<double>(a));
+        const double norm_d = sqrt(static_cast<double>(b));
+        double alpha = 1.0;
+        if (hp.malter) {
+            // Algorithm 2, nu_t line; alpha_t as displayed in Section 3.5.
+            const double t = static_cast<double>(*tcount);
+            const double nu = static_cast<double>(hp.mu2) * s.nu +
+                              (1.0 - static_cast<double>(hp.mu2)) * s.lgr_sq;
+            const double bc = sqrt(1.0 - pow(static_cast<double>(hp.mu2), t)) /
+                              (1.0 - pow(static_cast<double>(hp.mu1), t) + hp.eps);
+            alpha = bc * s.norm_mt / (sqrt(nu) + hp.eps);
+            s.nu = static_cast<float>(nu);
+        }
+        s.norm_o = static_cast<float>(norm_o);
+        s.norm_d = static_cast<float>(norm_d);
+        s.alpha = static_cast<float>(alpha);
+        s.scale = static_cast<float>(hp.lr * alpha * norm_o / (norm_d + hp.eps));
+        *sc = s;
+    }
+}
+
+// ------------------------------------------------------------------ apply
+__device__ __forceinline__ void apply8(const MatDesc& d, const UserPtrs& up, bool wbf, float s,
+                                       float decay, int i, int j, const float (&o)[8]) {
+    const size_t e = static_cast<size_t>(i) * d.n + j;
+    const float Li = d.L[i];
+    const float4 r0 = *reinterpret_cast<const float4*>(d.R + j);
+    const float4 r1 = *reinterpret_cast<const float4*>(d.R + j + 4);
+    const float rj[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
+    float w[8];
+    if (wbf) {
+        const uint4 u = *reinterpret_cast<const uint4*>(static_cast<__nv_bfloat16*>(up.w) + e);
+        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float2 f = __bfloat1622float2(h[k]);
+            w[2 * k] = f.x;
+            w[2 * k + 1] = f.y;
+        }
+    } else {
+        const float4* wp = reinterpret_cast<const float4*>(static_cast<float*>(up.w) + e);
+        const float4 a = wp[0], b = wp[1];
+        w[0] = a.x; w[1] = a.y; w[2] = a.z; w[3] = a.w;
+        w[4] = b.x; w[5] = b.y; w[6] = b.z; w[7] = b.w;
+    }
+    const float sl = s * Li;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) w[k] = fmaf(-sl * o[k], rj[k], decay * w[k]);
+    if (wbf) {
+        *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(up.w) + e) = pack8_bf16(w);
+    } else {
+        float4* wp = reinterpret_cast<float4*>(static_cast<float*>(up.w) + e);
+        wp[0] = make_float4(w[0], w[1], w[2], w[3]);
+        wp[1] = make_float4(w[4], w[5], w[6], w[7]);
+    }
+}
+
+// Block `local` of the apply pass: kApplyElems contiguous elements of a wide
+// matrix, or rows [64 i, 64 i + 64) x columns [kPreCols j, ...) of a tall one
+// (whose O is stored n x m in the NS frame), read as four 64 x 64 tiles of
+// O^T through shared memory (tile: 64 x 65 floats).  s = the grafted scale.
+template <bool kRO, class Sync>
+__device__ __forceinline__ void apply_block(const MatDesc& d, const UserPtrs& up, int local,
+                                            float s, float decay, int tid, float (*tile)[65],
+                                            Sync sync) {
+    const int m = d.m, n = d.n;
+    const bool wbf = d.w_bf16 != 0;
+    if (d.trans) {
+        const int tiles_c = (n + kPreCols - 1) / kPreCols;
+        const int i0 = (local / tiles_c) * 64, c0 = (local % tiles_c) * kPreCols;
+        const int t = tid;
+        for (int sub = 0; sub < kPreCols / 64; ++sub) {
+            const int j0 = c0 + sub * 64;
+            if (j0 >= n) break;                           // uniform across the block
+#pragma unroll
+            for (int pass = 0; pass < 2; ++pass) {
+                const int jj = pass * 32 + (t >> 3);      // row of O_ns = column of W
+                const int ii = (t & 7) * 8;               // 8 consecutive rows of W
+                float o[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+                if (j0 + jj < n && i0 + ii < m)
+                    load8<kRO>(d.O, true, static_cast<size_t>(j0 + jj) * m + i0 + ii, o);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) tile[ii + k][jj] = o[k];
+            }
+            sync();
+#pragma unroll
+            for (int pass = 0; pass < 2; ++pass) {
+                const int ii = pass * 32 + (t >> 3);      // row of W
+                const int jj = (t & 7) * 8;               // 8 consecutive columns of W
+                if (i0 + ii < m && j0 + jj < n) {
+                    float o[8];
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) o[k] = tile[ii][jj + k];
+                    apply8(d, up, wbf, s, decay, i0 + ii, j0 + jj, o);
+                }
+            }
+            sync();                                       // tile is reused by the next sub-tile
+        }
+        return;
+    }
+    const int32_t total = m * n;
+    const int32_t e0 = local * kApplyElems;
+#pragma unroll 4
+    for (int v = 0; v < kApplyElems / (kThreads * 8); ++v) {
+        const int32_t e = e0 + (v * kThreads + tid) * 8;
+        if (e >= total) break;
+        const int i = e / n, j = e - i * n;
+        float o[8];
+        load8<kRO>(d.O, true, static_cast<size_t>(e), o);
+        apply8(d, up, wbf, s, decay, i, j, o);
+    }
+}
+
+}  // namespace blk
+}  // namespace malt
