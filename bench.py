@@ -271,8 +271,10 @@ def run_malt(args):
     malter = wl.variant == "malter"
     stream = torch.cuda.current_stream()
     sched_code = {"auto": malt.MALT_NS_AUTO, "phased": malt.MALT_NS_PHASED,
-                  "persistent": malt.MALT_NS_PERSISTENT}[args.ns_schedule]
+                  "persistent": malt.MALT_NS_PERSISTENT,
+                  "fused": malt.MALT_NS_FUSED}[args.ns_schedule]
     opt.set_ns_schedule(sched_code)
+    opt.set_overlap_groups(args.overlap_groups)
 
     for _ in range(args.warmup):
         opt.step(hp, malter=malter)
@@ -313,7 +315,8 @@ def run_malt(args):
         sched = {"timed": args.ns_schedule + (" (persistent for shallow products, phased for "
                                               "deep ones)" if args.ns_schedule == "auto" else ""),
                  "timed_ms_per_step": t_ms / args.steps}
-        for name, code in (("phased", malt.MALT_NS_PHASED), ("persistent", malt.MALT_NS_PERSISTENT)):
+        for name, code in (("phased", malt.MALT_NS_PHASED), ("persistent", malt.MALT_NS_PERSISTENT),
+                           ("fused", malt.MALT_NS_FUSED)):
             opt.set_ns_schedule(code)
             for _ in range(2):
                 opt.step(hp, malter=malter)
@@ -389,8 +392,11 @@ def run_malt(args):
 
     # ---- roofline of the dominant kernel (the Newton-Schulz GEMMs)
     pk, pk_src = peaks()
-    ns_ms = sum(prof[k][0] for k in malt.NS_KINDS)
-    ns_launches = sum(prof[k][1] for k in malt.NS_KINDS)
+    fused_timed = prof["step_fused"][1] > 0
+    # the fused schedule runs the whole step in its launches: their time is the kernel's
+    ns_kinds = ("step_fused",) if fused_timed else malt.NS_KINDS
+    ns_ms = sum(prof[k][0] for k in ns_kinds)
+    ns_launches = sum(prof[k][1] for k in ns_kinds)
     # Algorithmic work: the Newton-Schulz flops with the symmetry of the Gram
     # matrix and of the polynomial used (3 p^2 q + p^3 per matrix and iteration),
     # which is what the kernels compute (upper-triangle tiles only).
@@ -401,7 +407,7 @@ def run_malt(args):
     persistent_timed = prof["ns_persistent"][1] > 0 and prof["ns_bx"][1] == 0
     # the committed capture is of the 144-matrix GPT-2 Large set only
     traffic = ncu_traffic_per_launch(persistent_timed) if (
-        wl.name == "gpt2_large" and not args.layers) else None
+        wl.name == "gpt2_large" and not args.layers and not fused_timed) else None
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "traffic": traffic,
                 "kernel": ("ns_gemm_kernel, persistent schedule (every Gram, Poly and BX "
@@ -460,8 +466,11 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-muon", action="store_true")
-    ap.add_argument("--ns-schedule", choices=("auto", "phased", "persistent"), default="auto",
-                    help="Newton-Schulz schedule of the timed steps (default: the library's auto)")
+    ap.add_argument("--ns-schedule", choices=("auto", "phased", "persistent", "fused"),
+                    default="auto",
+                    help="schedule of the timed steps (default: the library's auto)")
+    ap.add_argument("--overlap-groups", type=int, default=0,
+                    help="fused schedule: runs of matrices overlapped (0: automatic)")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling only: the first N layers of the workload")
     args = ap.parse_args()

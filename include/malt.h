@@ -210,45 +210,68 @@ int malt_debug_wait_timeout(int64_t budget_ns, void* stream);
 #define MALT_KIND_SCALARS   8
 #define MALT_KIND_APPLY     9
 #define MALT_KIND_NS_PERSISTENT 10   /* all Newton-Schulz products, persistent schedule */
-#define MALT_NUM_KINDS     11
+#define MALT_KIND_STEP_FUSED 11      /* the whole step in one launch, fused schedule */
+#define MALT_NUM_KINDS     12
 int malt_profile_enable(malt_state_t* st, int32_t enable);
 int malt_profile_read(malt_state_t* st, double* ms_out, int64_t* launches_out, int32_t nkinds);
 
-/* Newton-Schulz schedule of a state (the Orth step of Algorithm 1: k
- * iterations of A = X X^T, B' = aI + bA + cA^2, X <- B' X per matrix).
- *   MALT_NS_PERSISTENT: one persistent launch per group of up to 8 shape
- *     classes runs every product of every iteration.  Tiles are claimed
- *     dynamically in product order; a tile of matrix j waits on the device
- *     (bounded) only until the previous product of matrix j is stored, so
- *     one matrix's next product overlaps another matrix's current one and
+/* Schedule of a state's steps (the Orth step of Algorithm 1 is k iterations
+ * of A = X X^T, B' = aI + bA + cA^2, X <- B' X per matrix).
+ *   MALT_NS_PHASED: one launch per HBM-bound stage (statistics, finalize,
+ *     prescale, norms, scalars, apply) and one per Newton-Schulz product (3 k
+ *     launches per group of up to 8 shape classes), each product over all
+ *     matrices finished before the next starts.
+ *   MALT_NS_PERSISTENT: the same HBM-bound launches; one persistent launch
+ *     per class group runs every product of every iteration.  Tiles are
+ *     claimed dynamically in product order; a tile of matrix j waits on the
+ *     device (bounded) only until the previous product of matrix j is stored,
+ *     so one matrix's next product overlaps another matrix's current one and
  *     there is no launch gap or wave tail between products.
- *   MALT_NS_PHASED: one launch per product (3 k launches per group), each
- *     product over all matrices finished before the next starts.
- *   MALT_NS_AUTO (default): per group, persistent when a Gram product has
- *     fewer tiles than 16 waves of the resident CTA pairs (shallow products,
- *     where tails and launch gaps weigh most), phased otherwise.
- * All compute every tile with the same arithmetic: results are bitwise
- * identical.  Takes effect at the next step.  MALT_ERR_INVALID_ARG for a
- * null state or an unknown schedule. */
+ *   MALT_NS_FUSED: the whole step in one persistent launch per class group.
+ *     The HBM-bound stages run on the GEMM kernel's epilogue warps between
+ *     tiles, chained per matrix by the same device counters; the matrices
+ *     are split into consecutive runs (malt_set_overlap_groups) so that one
+ *     run's statistics / prescale and another run's apply overlap a third
+ *     run's tensor-core products.
+ *   MALT_NS_AUTO (default): per class group, persistent when a Gram product
+ *     has fewer tiles than 16 waves of the resident CTA pairs, phased otherwise.
+ * All compute every tile and element with the same arithmetic: results are
+ * bitwise identical.  Takes effect at the next step.  The persistent and
+ * fused schedules use a work table per ns_steps value, built on the host and
+ * uploaded by the first step that needs it (a synchronising copy: for a
+ * stream capture, take one eager step with the same ns_steps first; the
+ * table for ns_steps = 5 is built at init).  MALT_ERR_INVALID_ARG for a null
+ * state or an unknown schedule. */
 #define MALT_NS_PHASED     0
 #define MALT_NS_PERSISTENT 1
 #define MALT_NS_AUTO       2
+#define MALT_NS_FUSED      3
 int malt_set_ns_schedule(malt_state_t* st, int32_t schedule);
 
-/* Host only (no GPU, no CUDA call): the persistent schedule's work list for
- * these parameter shapes (only rows and cols are read) and ns_steps
- * iterations, in claim order, 8 int32 per item: launch group, product index
- * s = 3 * iteration + (0 Gram, 1 Poly, 2 BX), matrix index, tile row, tile
- * column (256 x 256 tiles of the NS frame; Gram and Poly list the upper
- * triangle only), the index of the counter the tile waits for ((s - 1) *
- * n + matrix, or -1), the count that counter must reach (16 signals per
- * tile of product s - 1), and the number of tiles of product s of this
- * matrix.  Writes min(capacity, total) items to out (capacity * 8 int32,
- * caller-owned) and the total to *count; call with capacity 0 to size out.
- * MALT_ERR_INVALID_ARG for bad arguments or ns_steps outside [1, 64],
- * MALT_ERR_UNSUPPORTED for a shape malt_init_state would reject. */
-int malt_ns_schedule(const malt_param_t* params, int32_t n, int32_t ns_steps, int32_t* out,
-                     int64_t capacity, int64_t* count);
+/* Fused schedule: the number of consecutive runs the matrices are split into
+ * (1..64; 0 = automatic, min(4, matrices / 8)).  More runs hide more of the
+ * HBM-bound stages behind the products but make each run's products
+ * shallower.  Takes effect at the next step (rebuilding the work table).
+ * MALT_ERR_INVALID_ARG for a null state or a count outside 0..64. */
+int malt_set_overlap_groups(malt_state_t* st, int32_t groups);
+
+/* Host only (no GPU, no CUDA call): the work table of the persistent
+ * (fused = 0) or fused (fused = 1) schedule for these parameter shapes (only
+ * rows and cols are read), ns_steps iterations and overlap_groups runs (0 =
+ * automatic), in claim order, 8 int32 per item: launch group, stage, stage
+ * kind (0 Gram, 1 Poly, 2 B*X, 3 statistics, 4 finalize, 5 prescale,
+ * 6 norms, 7 scalars, 8 apply), matrix index, local index (the tile of the
+ * product, 256 x 256 tiles of the NS frame with Gram and Poly listing the
+ * upper triangle only; the block pair or 0 for a memory stage), the index of
+ * the counter the item waits for ((stage - 1) * n + matrix, or -1), the count
+ * that counter must reach (16 signals per item of the previous stage), and
+ * the number of items of (stage, matrix).  Writes min(capacity, total) items
+ * to out (capacity * 8 int32, caller-owned) and the total to *count; call
+ * with capacity 0 to size out.  MALT_ERR_INVALID_ARG for bad arguments or
+ * ns_steps outside [1, 64], MALT_ERR_UNSUPPORTED for a shape
+ * malt_init_state would reject. */
+int malt_ns_schedule(const malt_param_t* params, int32_t n, int32_t ns_steps, int32_t fused,
+                     int32_t overlap_groups, int32_t* out, int64_t capacity, int64_t* count);
 
 /* Statistics stage of ONE matrix without any device allocation.
  * The paper has no counterpart: this exists for callers that cannot allocate

@@ -87,8 +87,37 @@ struct StepHyper {
 // ------------------------------------------------------ Newton-Schulz engine
 enum GemmPhase : int32_t { kGram = 0, kPoly = 1, kBX = 2 };
 
-// Epilogue warps of a CTA pair; each one signals a finished tile once.
+// Launch modes of the Newton-Schulz kernel: one product with a static tile
+// split; a persistent work table of products; a persistent work table of
+// the whole step (products and the HBM-bound stages around them).
+enum NsMode : int32_t { kNsPhased = 0, kNsPersistent = 1, kNsFused = 2 };
+
+// Epilogue warps of a CTA pair; each one signals a finished item once.
 constexpr uint32_t kNsSignalsPerTile = 2 * kEpiWarpsPerCta;
+
+// Stage kinds of a persistent work table.  The products of Newton-Schulz
+// iteration i are stages front + 3 i + {kGram, kPoly, kBX}; a fused step puts
+// the HBM-bound stages around them (kFrontStages before, kBackStages after).
+enum StageKind : int32_t {
+    kKindStats = 3, kKindFinalize = 4, kKindPrescale = 5, kKindNorms = 6,
+    kKindScalars = 7, kKindApply = 8
+};
+constexpr int kFrontStages = 4;   // stats, finalize, prescale, norms
+constexpr int kBackStages = 2;    // scalars, apply
+
+// One item of a persistent work table.
+struct __align__(16) NsEntry {
+    int32_t code;     // stage (bits 0-11) | class slot (bits 12-15) | batch slot (bits 16-31)
+    int32_t g;        // matrix; -1 marks the end of the table
+    int32_t local;    // tile of the product, block pair of a memory stage, 0 otherwise
+    uint32_t target;  // signals the previous stage of matrix g must reach (0: none)
+};
+
+__host__ __device__ __forceinline__ int32_t entry_stage(const NsEntry& e) { return e.code & 0xfff; }
+__host__ __device__ __forceinline__ int32_t entry_cls(const NsEntry& e) { return (e.code >> 12) & 0xf; }
+__host__ __device__ __forceinline__ int32_t entry_b(const NsEntry& e) {
+    return static_cast<int32_t>(static_cast<uint32_t>(e.code) >> 16);
+}
 
 // One shape class (every matrix whose NS frame is p x q, stored batched) with
 // all the tensor maps of the three products of an NS iteration.
@@ -121,11 +150,22 @@ struct NsParams {
     int32_t item_begin, item_end;
     float a, b, c;
     const MatDesc* mats;
-    const MatScalars* scal;
+    MatScalars* scal;
     int32_t* status;
     uint32_t* queue;              // next unclaimed item (persistent schedule)
-    uint32_t* done;               // [3 ns_steps][nmat] finished-tile signals (persistent)
+    uint32_t* done;               // [stages][nmat] finished-item signals (persistent)
     uint64_t budget_ns;
+    // Persistent launches: the work table (item_end entries) and its stages.
+    const NsEntry* table;
+    int32_t front;                // memory stages before the products (0 or kFrontStages)
+    int32_t nstages;              // front + 3 ns_steps (+ kBackStages when fused)
+    // Fused step: what the memory stages need.
+    const UserPtrs* ptrs;
+    const long long* tcount;
+    StepHyper hp;
+    float decay;                  // 1 - lr * weight_decay
+    int32_t with_stats;           // 0 for Muon through the same engine (momentum only)
+    int32_t identity;             // 1 for Muon: L = R = 1
 };
 
 // One decoded work item: a 256 x 256 output tile of one product.
@@ -141,6 +181,32 @@ struct NsWork {
 // upper triangle (nt >= mt) for the symmetric Gram and polynomial products.
 __host__ __device__ __forceinline__ int32_t ns_phase_tiles(const NsClass& C, int32_t kind) {
     return kind == kBX ? C.tiles_p * C.tiles_q : C.tiles_p * (C.tiles_p + 1) / 2;
+}
+
+// Tile row / column of the rem-th tile of one matrix's product of this kind
+// (row-major over all tiles for B*X, the upper triangle row by row otherwise).
+__host__ __device__ __forceinline__ void ns_tile_coords(const NsClass& C, int32_t kind, int32_t rem,
+                                                        int32_t* mt, int32_t* nt) {
+    if (kind == kBX) {
+        *mt = rem / C.tiles_q;
+        *nt = rem - *mt * C.tiles_q;
+        return;
+    }
+    int32_t r = 0, u = rem;
+    while (u >= C.tiles_p - r) {
+        u -= C.tiles_p - r;
+        ++r;
+    }
+    *mt = r;
+    *nt = r + u;
+}
+
+// Blocks of the apply pass of one matrix: kApplyElems contiguous elements of
+// a wide matrix, 64 x kPreCols of a tall one.
+__host__ __device__ __forceinline__ int32_t mat_apply_blocks(const MatDesc& d) {
+    return d.trans ? ((d.m + 63) / 64) * ((d.n + kPreCols - 1) / kPreCols)
+                   : static_cast<int32_t>((static_cast<int64_t>(d.m) * d.n + kApplyElems - 1) /
+                                          kApplyElems);
 }
 
 __host__ __device__ __forceinline__ NsWork ns_decode(const NsParams& P, int32_t item) {
@@ -168,30 +234,8 @@ __host__ __device__ __forceinline__ NsWork ns_decode(const NsParams& P, int32_t 
     w.b = local / per;
     const int32_t rem = local - w.b * per;
     w.local = rem;
-    if (!sym) {
-        w.mt = rem / C.tiles_q;
-        w.nt = rem - w.mt * C.tiles_q;
-    } else {
-        int32_t mt = 0, u = rem;
-        while (u >= C.tiles_p - mt) {
-            u -= C.tiles_p - mt;
-            ++mt;
-        }
-        w.mt = mt;
-        w.nt = mt + u;
-    }
+    ns_tile_coords(C, w.kind, rem, &w.mt, &w.nt);
     return w;
-}
-
-// The counter a work item of matrix g waits for under the persistent
-// schedule -- its matrix's previous product, s - 1 -- and the number of
-// signals that means "every tile stored".  -1 for the first product.
-__host__ __device__ __forceinline__ int32_t ns_dependency(const NsParams& P, const NsWork& w,
-                                                          int32_t g, uint32_t* target) {
-    if (w.s == 0) return -1;
-    const int32_t prev_kind = (w.kind + 2) % 3;
-    *target = kNsSignalsPerTile * static_cast<uint32_t>(ns_phase_tiles(P.cls[w.cls], prev_kind));
-    return (w.s - 1) * P.nmat + g;
 }
 
 }  // namespace malt

@@ -34,12 +34,13 @@ cudaError_t launch_wait_probe(int32_t* status, uint64_t budget_ns, cudaStream_t 
 cudaError_t launch_transpose_bf16(const __nv_bfloat16* src, __nv_bfloat16* dst, int rows, int cols,
                                   cudaStream_t s);
 
-// Newton-Schulz products over up to kMaxClasses shape classes: the items
-// [P.item_begin, P.item_end) of the work list, on grid_pairs CTA pairs
-// (clusters of two).  persistent: items claimed dynamically, each waiting for
-// its matrix's previous product (P.queue and P.done zeroed before the launch);
-// otherwise static round-robin over one product.
-cudaError_t launch_ns_gemm(const NsParams& P, bool persistent, int grid_pairs, cudaStream_t s);
+// Newton-Schulz products over up to kMaxClasses shape classes on grid_pairs
+// CTA pairs (clusters of two).  mode kNsPhased: the items
+// [P.item_begin, P.item_end) of one product, static round-robin.
+// kNsPersistent / kNsFused: the work table P.table, claimed dynamically, each
+// item waiting for its matrix's previous stage (P.queue and P.done zeroed
+// before the launch); kNsFused tables also hold the HBM-bound stages.
+cudaError_t launch_ns_gemm(const NsParams& P, int mode, int grid_pairs, cudaStream_t s);
 size_t ns_gemm_smem_bytes();
 int ns_gemm_max_pairs();
 // Opt the GEMM kernel into its shared memory and cache the resident pair count.

@@ -72,6 +72,7 @@
 #include "common.cuh"
 #include "kernels.h"
 #include "ptx.cuh"
+#include "stream_blocks.cuh"
 
 namespace malt {
 
@@ -190,23 +191,100 @@ __device__ __forceinline__ void raise_timeout(const NsParams& P, volatile int* a
     *abort_flag = 1;
 }
 
-// Persistent schedule: wait until the product this item reads from is
-// complete for its matrix.
-__device__ __forceinline__ bool wait_dependency(const NsParams& P, const NsWork& w,
-                                                volatile int* abort_flag) {
-    uint32_t target = 0;
-    const int g = P.cls[w.cls].mat_of[w.b];
-    const int idx = ns_dependency(P, w, g, &target);
-    if (idx < 0) return true;
-    return counter_wait_bounded(P.done + idx, target, P.budget_ns, P.status, kStatusTimeout,
-                                abort_flag);
+// One unit of work as a role of the pair sees it.
+enum JobState : int32_t { kJobWork = 0, kJobEnd = -1, kJobTimeout = -2 };
+struct Job {
+    int32_t state;
+    int32_t stage;    // stage of the work table (persistent) or product index (phased)
+    int32_t mem;      // memory stage kind (kKindStats..kKindApply), 0 for a product tile
+    int32_t g;        // matrix (-1 when not known yet: phased)
+    int32_t local;
+    NsWork w;         // product tiles only
+};
+
+__device__ __forceinline__ Job job_of_entry(const NsParams& P, const NsEntry& e) {
+    Job j;
+    if (e.g < 0) {
+        j.state = kJobEnd;
+        return j;
+    }
+    j.state = kJobWork;
+    j.stage = entry_stage(e);
+    j.g = e.g;
+    j.local = e.local;
+    const int s_ns = j.stage - P.front;
+    if (s_ns < 0) {
+        j.mem = kKindStats + j.stage;
+    } else if (s_ns >= 3 * P.ns_steps) {
+        j.mem = kKindScalars + (s_ns - 3 * P.ns_steps);
+    } else {
+        j.mem = 0;
+        j.w.s = s_ns;
+        j.w.iter = s_ns / 3;
+        j.w.kind = s_ns - 3 * j.w.iter;
+        j.w.cls = entry_cls(e);
+        j.w.b = entry_b(e);
+        j.w.local = e.local;
+        ns_tile_coords(P.cls[j.w.cls], j.w.kind, e.local, &j.w.mt, &j.w.nt);
+    }
+    return j;
+}
+
+// One HBM-bound stage item of a fused step on the 8 epilogue warps of a CTA
+// (tid 0..255): CTA `rank` of the pair takes block 2 local + rank of a stats,
+// prescale or apply item; finalize splits rows (even CTA) and columns (odd
+// CTA); norms and scalars run on the even CTA.  Kept out of line so that its
+// registers do not weigh on the tile epilogue.
+__device__ __noinline__ void run_memory_stage(const NsParams& P, int mem, int g, int local,
+                                              int rank, int tid, float* scratch) {
+    blk::SyncEpilogue sync;
+    const MatDesc& d = P.mats[g];
+    const UserPtrs up = P.ptrs[g];
+    const int bi = 2 * local + rank;
+    switch (mem) {
+        case kKindStats:
+            if (bi < d.stat_rb * d.stat_cb) {
+                if (P.with_stats)
+                    blk::stats_block<true>(d, up, bi, P.hp.mu1, tid, scratch, sync);
+                else
+                    blk::stats_block<false>(d, up, bi, P.hp.mu1, tid, scratch, sync);
+            }
+            break;
+        case kKindFinalize: {
+            const int lo = rank ? d.m : 0, hi = rank ? d.m + d.n : d.m;
+            for (int x = lo + tid; x < hi; x += blk::kThreads)
+                blk::finalize_entry<true>(d, up, x, P.hp.mu2, P.hp.eps, P.identity);
+            break;
+        }
+        case kKindPrescale:
+            if (bi < d.pre_tr * d.pre_tc)
+                blk::prescale_block<true>(d, up, bi, P.hp.malter, tid,
+                                          reinterpret_cast<float(*)[65]>(scratch),
+                                          reinterpret_cast<float2*>(scratch + 64 * 66), sync);
+            break;
+        case kKindNorms:
+            if (rank == 0)
+                blk::norms_matrix<true>(d, P.scal + g, P.hp.ns_eps, P.hp.malter, tid, scratch, sync);
+            break;
+        case kKindScalars:
+            if (rank == 0)
+                blk::scalars_matrix<true>(d, P.scal + g, P.tcount, P.hp, tid, scratch, sync);
+            break;
+        default:                                             // kKindApply
+            if (bi < mat_apply_blocks(d))
+                blk::apply_block<true>(d, up, bi, __ldcg(&P.scal[g].scale), P.decay, tid,
+                                       reinterpret_cast<float(*)[65]>(scratch), sync);
+            break;
+    }
 }
 
 }  // namespace
 
-template <bool kPersistent>
+template <int kMode>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 ns_gemm_kernel(const __grid_constant__ NsParams P) {
+    constexpr bool kPersistent = kMode != kNsPhased;   // table-driven, claimed dynamically
+    constexpr bool kFused = kMode == kNsFused;         // the table also holds memory stages
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[kStages];
     __shared__ __align__(8) uint64_t empty_bar[kStages];
@@ -215,7 +293,7 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
     __shared__ __align__(8) uint64_t drain_bar;
     __shared__ __align__(8) uint64_t item_full[kItemSlots];
     __shared__ __align__(8) uint64_t item_empty[kItemSlots];
-    __shared__ int32_t item_ring[kItemSlots];
+    __shared__ NsEntry item_ring[kItemSlots];
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_sh;
     volatile int* abort_flag = &abort_sh;
@@ -276,46 +354,87 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
     tc_fence_after();
     const uint32_t tmem_base = tmem_slot;
 
-    // Item number `seq` of this pair.  Phased: static round-robin.  Persistent:
-    // read from the ring (-2 when the wait gave up), which the scheduler
-    // thread of the odd CTA fills (claim_next, publish_item).
-    auto static_item = [&](int seq) -> int {
+    // Work number `seq` of this pair.  Phased: static round-robin over the
+    // product's item range.  Persistent: the next entry of the ring, which
+    // the scheduler thread of the odd CTA fills from the work table.
+    auto static_job = [&](int seq) -> Job {
+        Job j;
         const long long it = static_cast<long long>(P.item_begin) + pair +
                              static_cast<long long>(seq) * npairs;
-        return it < P.item_end ? static_cast<int>(it) : -1;
+        if (it >= P.item_end) {
+            j.state = kJobEnd;
+            return j;
+        }
+        j.state = kJobWork;
+        j.w = ns_decode(P, static_cast<int>(it));
+        j.stage = j.w.s;
+        j.mem = 0;
+        j.g = -1;
+        j.local = j.w.local;
+        return j;
     };
-    auto read_item = [&](int seq) -> int {
+    // The ring entry of sequence number seq (false when the wait gave up).
+    auto ring_entry = [&](int seq, NsEntry& e) -> bool {
         const int slot = seq % kItemSlots;
         const uint32_t par = static_cast<uint32_t>(seq / kItemSlots) & 1u;
-        if (!mbar_wait_cluster_bounded(&item_full[slot], par, budget, abort_flag)) return -2;
-        const int item = *reinterpret_cast<volatile int32_t*>(&item_ring[slot]);
+        if (!mbar_wait_cluster_bounded(&item_full[slot], par, budget, abort_flag)) return false;
+        const volatile int32_t* v = reinterpret_cast<const volatile int32_t*>(&item_ring[slot]);
+        e.code = v[0];
+        e.g = v[1];
+        e.local = v[2];
+        e.target = static_cast<uint32_t>(v[3]);
         // Free the slot (its barrier lives in the odd CTA, with the
         // scheduler).  The arrive carries no data, so it is relaxed; it is
         // issued only once the slot's value is in hand (the branch depends on
         // it), so the scheduler cannot overwrite the slot before this read.
-        if (item != kNoItem) mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&item_empty[slot]), 1));
-        return item;
+        if (e.code != kNoItem)
+            mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&item_empty[slot]), 1));
+        return true;
     };
-    // Scheduler (odd CTA): claim the next item index (-1 past the end), and
-    // publish an item to the ring slot of sequence number seq in both CTAs
-    // (false when the slot did not come free in time).
-    auto claim_next = [&]() -> int {
+    auto ring_job = [&](int seq) -> Job {
+        NsEntry e;
+        if (!ring_entry(seq, e)) {
+            Job j;
+            j.state = kJobTimeout;
+            return j;
+        }
+        return job_of_entry(P, e);
+    };
+    auto next_job = [&](int seq) -> Job { return kPersistent ? ring_job(seq) : static_job(seq); };
+    // Scheduler (odd CTA): the table entry of the next claimed item (an end
+    // marker past the end), and its publication to the ring slot of sequence
+    // number seq in both CTAs (false when the slot did not come free in time).
+    auto claim_next = [&]() -> NsEntry {
         const uint32_t claimed = atomicAdd(P.queue, 1u);
-        return claimed < static_cast<uint32_t>(P.item_end - P.item_begin)
-                   ? P.item_begin + static_cast<int>(claimed) : -1;
+        if (claimed >= static_cast<uint32_t>(P.item_end - P.item_begin)) {
+            NsEntry e;
+            e.code = 0;
+            e.g = -1;
+            e.local = 0;
+            e.target = 0;
+            return e;
+        }
+        const int4 v = __ldg(reinterpret_cast<const int4*>(P.table + P.item_begin + claimed));
+        NsEntry e;
+        e.code = v.x;
+        e.g = v.y;
+        e.local = v.z;
+        e.target = static_cast<uint32_t>(v.w);
+        return e;
     };
-    auto publish_item = [&](int seq, int item) -> bool {
+    auto publish_item = [&](int seq, const NsEntry& e) -> bool {
         const int slot = seq % kItemSlots;
         const uint32_t par = static_cast<uint32_t>(seq / kItemSlots) & 1u;
         if (!mbar_wait_cluster_bounded(&item_empty[slot], par ^ 1u, budget, abort_flag)) return false;
-        // The item travels as an asynchronous store that completes on the
+        // The entry travels as an asynchronous store that completes on the
         // slot's full barrier in each CTA.  The arrive releases at cluster
         // scope what this thread acquired from the dependency counter, so a
-        // reader that sees the item also sees the operands the item reads.
+        // reader that sees the item also sees the data the item reads.
         for (uint32_t r = 0; r < 2; ++r) {
             const uint32_t bar = mapa_shared(smem_u32(&item_full[slot]), r);
-            mbar_arrive_expect_tx_cluster(bar, 4u);
-            st_async_u32(mapa_shared(smem_u32(&item_ring[slot]), r), static_cast<uint32_t>(item), bar);
+            mbar_arrive_expect_tx_cluster(bar, 16u);
+            st_async_v4(mapa_shared(smem_u32(&item_ring[slot]), r), e.code, e.g, e.local,
+                        static_cast<int32_t>(e.target), bar);
         }
         return true;
     };
@@ -325,15 +444,17 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
         if (lane == 0) {
             uint32_t stage = 0, phase = 0;
             for (int seq = 0;; ++seq) {
-                const int item = kPersistent ? read_item(seq) : static_item(seq);
-                if (item == -2) {
+                const Job job = next_job(seq);
+                if (job.state == kJobTimeout) {
                     raise_timeout(P, abort_flag, kSiteItem, -2, seq);
                     break;
                 }
-                if (item < 0) break;
+                if (job.state == kJobEnd) break;
+                if (kFused && job.mem) continue;         // memory stages load no operands
+                const int item = job.local;
                 // The loads below read what other CTAs stored in this launch.
                 if (kPersistent) fence_proxy_async_global();
-                const NsWork w = ns_decode(P, item);
+                const NsWork& w = job.w;
                 const Ops op = item_operands(P, w);
                 const bool b_mn = w.kind == kBX;
                 const int nkb = (op.K + kBK - 1) / kBK;
@@ -370,40 +491,46 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
     } else if (warp == 1) {
         if (kPersistent && lane == 0 && !leader) {
             // ------------------------------------------ scheduler (odd CTA)
-            // Claim items in list order, one ahead; publish each once the
-            // previous product of its matrix is stored, up to kItemSlots
+            // Claim items in table order, one ahead; publish each once the
+            // previous stage of its matrix is complete, up to kItemSlots
             // ahead of the slowest reader.  Waiting here keeps the acquire
             // round trip off the producers' path.
-            int next = claim_next();
+            NsEntry next = claim_next();
             for (int seq = 0;; ++seq) {
-                const int item = next;
-                if (item >= 0 && !wait_dependency(P, ns_decode(P, item), abort_flag)) {
-                    raise_timeout(P, abort_flag, kSiteDepLoad, item, seq);
+                const NsEntry e = next;
+                if (e.g >= 0 && e.target > 0 &&
+                    !counter_wait_bounded(P.done + (entry_stage(e) - 1) * P.nmat + e.g, e.target,
+                                          P.budget_ns, P.status, kStatusTimeout, abort_flag)) {
+                    raise_timeout(P, abort_flag, kSiteDepLoad, e.local, seq);
                     break;
                 }
-                if (!publish_item(seq, item)) {
-                    raise_timeout(P, abort_flag, kSiteClaim, item, seq);
+                if (!publish_item(seq, e)) {
+                    raise_timeout(P, abort_flag, kSiteClaim, e.local, seq);
                     break;
                 }
-                if (item < 0) break;
+                if (e.g < 0) break;
                 next = claim_next();
             }
         }
         // ------------------------------------------- MMA issuer (even CTA)
         if (lane == 0 && leader) {
             uint32_t stage = 0, phase = 0;
+            int gi = 0;                                  // product tiles so far (accumulator)
             for (int seq = 0;; ++seq) {
-                const int item = kPersistent ? read_item(seq) : static_item(seq);
-                if (item == -2) {
+                const Job job = next_job(seq);
+                if (job.state == kJobTimeout) {
                     raise_timeout(P, abort_flag, kSiteItem + 16, -2, seq);
                     break;
                 }
-                if (item < 0) break;
-                const NsWork w = ns_decode(P, item);
+                if (job.state == kJobEnd) break;
+                if (kFused && job.mem) continue;
+                const int item = job.local;
+                const NsWork& w = job.w;
                 const bool b_mn = w.kind == kBX;
                 const int K = w.kind == kGram ? P.cls[w.cls].q : P.cls[w.cls].p;
                 const int nkb = (K + kBK - 1) / kBK;
-                const uint32_t acc = seq & 1, acc_phase = (seq >> 1) & 1;
+                const uint32_t acc = gi & 1, acc_phase = (gi >> 1) & 1;
+                ++gi;
                 if (!mbar_wait_cluster_bounded(&tempty_bar[acc], acc_phase ^ 1u, budget, abort_flag)) {
                     raise_timeout(P, abort_flag, kSiteAccFree, item, seq);
                     break;
@@ -456,23 +583,57 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
         const int colw = (ew >> 2) * kEpiCols;    // first accumulator column of this warp
         const uint32_t tempty_leader0 = mapa_shared(smem_u32(&tempty_bar[0]), 0);
         const uint32_t tempty_leader1 = mapa_shared(smem_u32(&tempty_bar[1]), 0);
+        const int tid = ew * 32 + lane;           // thread of the 256 running memory stages
+        float* scratch = reinterpret_cast<float*>(stage_out);
+        int gi = 0;                               // product tiles so far (accumulator)
         for (int seq = 0;; ++seq) {
-            int item;
+            Job job;
             if (kPersistent) {
-                int v = 0;
-                if (lane == 0) v = read_item(seq);
-                item = __shfl_sync(0xffffffffu, v, 0);
+                // One lane waits on the ring; the warp shares the entry.
+                NsEntry e;
+                e.code = 0;
+                e.g = -1;
+                e.local = 0;
+                e.target = 0;
+                int ok = 1;
+                if (lane == 0) ok = ring_entry(seq, e) ? 1 : 0;
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                e.code = __shfl_sync(0xffffffffu, e.code, 0);
+                e.g = __shfl_sync(0xffffffffu, e.g, 0);
+                e.local = __shfl_sync(0xffffffffu, e.local, 0);
+                if (!ok) {
+                    job.state = kJobTimeout;
+                } else {
+                    job = job_of_entry(P, e);
+                }
             } else {
-                item = static_item(seq);
+                job = static_job(seq);
             }
-            if (item == -2) {
+            if (job.state == kJobTimeout) {
                 if (lane == 0) raise_timeout(P, abort_flag, kSiteItem + 32, -2, seq);
                 break;
             }
-            if (item < 0) break;
-            const NsWork w = ns_decode(P, item);
+            if (job.state == kJobEnd) break;
+            const int item = job.local;
+            if (kFused && job.mem) {
+                // ---- an HBM-bound stage of the fused step, on the 8 epilogue
+                // warps of each CTA; the staging area is its shared scratch.
+                if (lane == 0) bulk_wait_group_read<0>();   // no tile store still reads it
+                blk::SyncEpilogue sync;
+                sync();
+                run_memory_stage(P, job.mem, job.g, job.local, rank, tid, scratch);
+                sync();                                      // scratch free for tile stores again
+                __syncwarp();
+                if (lane == 0 && job.stage + 1 < P.nstages) {
+                    __threadfence();
+                    red_release_gpu_add(P.done + job.stage * P.nmat + job.g, 1u);
+                }
+                continue;
+            }
+            const NsWork& w = job.w;
             const NsClass& C = P.cls[w.cls];
-            const uint32_t acc = seq & 1, acc_phase = (seq >> 1) & 1;
+            const uint32_t acc = gi & 1, acc_phase = (gi >> 1) & 1;
+            ++gi;
             if (!mbar_wait_cluster_bounded(&tfull_bar[acc], acc_phase, budget, abort_flag)) {
                 raise_timeout(P, abort_flag, kSiteAccFull, item, seq);
                 break;
@@ -483,9 +644,11 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
             const bool sym = w.kind != kBX;
             const int row = w.mt * kTileM + rank * kBM + quarter * 32 + lane;
             const bool rok = row < M;
-            const int g = C.mat_of[w.b];
+            const int g = job.g >= 0 ? job.g : C.mat_of[w.b];
             const MatDesc& md = P.mats[g];
-            const float kx = w.iter == 0 ? P.scal[g].k : 1.f;
+            // Persistent launches read what the launch itself wrote (1/||Mt||,
+            // L, R, A) through L2 only.
+            const float kx = w.iter == 0 ? (kPersistent ? __ldcg(&P.scal[g].k) : P.scal[g].k) : 1.f;
             const bool need_ein = (w.kind == kPoly);
             const __nv_bfloat16* ein =
                 need_ein ? C.A + static_cast<size_t>(w.b) * C.p * C.p : nullptr;
@@ -493,7 +656,7 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
             // NS frame row / column scalings of D = L O R (swapped when transposed).
             const float* uvec = md.trans ? md.R : md.L;
             const float* vvec = md.trans ? md.L : md.R;
-            const float urow = (last_bx && rok) ? uvec[row] : 0.f;
+            const float urow = (last_bx && rok) ? (kPersistent ? __ldcg(uvec + row) : uvec[row]) : 0.f;
             float sum_o = 0.f, sum_d = 0.f;
 
             const int col_base = w.nt * kBN + colw;     // first output column of this warp
@@ -509,9 +672,9 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                             ein + static_cast<size_t>(row) * N + col0 + q8 * 8);
                         // Phased: A was written by an earlier launch, so the
                         // read-only path is safe.  Persistent: A is rewritten
-                        // each iteration inside this launch; a coherent load
-                        // (ordered by the ring's acquire) is required.
-                        dst[q8] = kPersistent ? *src : __ldg(src);
+                        // each iteration inside this launch; read through L2
+                        // (ordered by the ring's acquire).
+                        dst[q8] = kPersistent ? __ldcg(src) : __ldg(src);
                     }
                     else
                         dst[q8] = make_uint4(0u, 0u, 0u, 0u);
@@ -603,7 +766,9 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                     // Partial sums of O^2 and (O v)^2 over the stored (bf16) O of this
                     // row; D^2 = u_row^2 (O v)^2 is formed once per tile.  Lane j holds
                     // v[col0 + j] and broadcasts it (columns past N contribute 0).
-                    const float vl = (col0 + lane < N) ? vvec[col0 + lane] : 0.f;
+                    const float vl = (col0 + lane < N)
+                                         ? (kPersistent ? __ldcg(vvec + col0 + lane) : vvec[col0 + lane])
+                                         : 0.f;
 #pragma unroll
                     for (int j = 0; j < 32; ++j) {
                         const float vj = __shfl_sync(0xffffffffu, vl, j);
@@ -633,12 +798,12 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                     dst[1] = sum_d;
                 }
             }
-            if (kPersistent && w.s + 1 < 3 * P.ns_steps && lane == 0) {
+            if (kPersistent && job.stage + 1 < P.nstages && lane == 0) {
                 // This warp's part of the tile is in global memory: signal it
-                // (the last product has no reader inside the launch).
+                // (the last stage has no reader inside the launch).
                 bulk_wait_group_all();
                 fence_proxy_async_global();
-                red_release_gpu_add(P.done + w.s * P.nmat + g, 1u);
+                red_release_gpu_add(P.done + job.stage * P.nmat + g, 1u);
             }
         }
         if (lane == 0) bulk_wait_group_all();     // every output store has landed
@@ -658,17 +823,23 @@ size_t ns_gemm_smem_bytes() { return kSmemBytes; }
 
 namespace {
 
-template <bool kPersistent>
+template <int kMode>
 cudaError_t set_smem_attr() {
-    return cudaFuncSetAttribute(ns_gemm_kernel<kPersistent>,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+    return cudaFuncSetAttribute(ns_gemm_kernel<kMode>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 static_cast<int>(kSmemBytes));
+}
+
+cudaError_t set_all_smem_attrs() {
+    cudaError_t e = set_smem_attr<kNsPhased>();
+    if (e == cudaSuccess) e = set_smem_attr<kNsPersistent>();
+    if (e == cudaSuccess) e = set_smem_attr<kNsFused>();
+    return e;
 }
 
 }  // namespace
 
 // Number of CTA pairs that can be resident at once (the persistent grid).
-// Both instantiations have the same block shape and shared memory.
+// All instantiations have the same block shape and shared memory.
 int ns_gemm_max_pairs() {
     static int cached = -1;
     if (cached > 0) return cached;
@@ -677,8 +848,8 @@ int ns_gemm_max_pairs() {
     cfg.gridDim = dim3(2, 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = kSmemBytes;
-    if (set_smem_attr<true>() != cudaSuccess || set_smem_attr<false>() != cudaSuccess ||
-        cudaOccupancyMaxActiveClusters(&n, ns_gemm_kernel<true>, &cfg) != cudaSuccess || n <= 0) {
+    if (set_all_smem_attrs() != cudaSuccess ||
+        cudaOccupancyMaxActiveClusters(&n, ns_gemm_kernel<kNsFused>, &cfg) != cudaSuccess || n <= 0) {
         cudaGetLastError();
         int dev = 0, sms = 0;
         cudaGetDevice(&dev);
@@ -692,8 +863,7 @@ int ns_gemm_max_pairs() {
 cudaError_t ns_gemm_configure() {
     static bool configured = false;
     if (!configured) {
-        cudaError_t e = set_smem_attr<true>();
-        if (e == cudaSuccess) e = set_smem_attr<false>();
+        const cudaError_t e = set_all_smem_attrs();
         if (e != cudaSuccess) return e;
         configured = true;
     }
@@ -701,25 +871,29 @@ cudaError_t ns_gemm_configure() {
     return cudaSuccess;
 }
 
-cudaError_t launch_ns_gemm(const NsParams& P, bool persistent, int grid_pairs, cudaStream_t s) {
+cudaError_t launch_ns_gemm(const NsParams& P, int mode, int grid_pairs, cudaStream_t s) {
     const cudaError_t ce = ns_gemm_configure();
     if (ce != cudaSuccess) return ce;
-    if (persistent)
-        ns_gemm_kernel<true><<<2 * grid_pairs, kThreads, kSmemBytes, s>>>(P);
+    if (mode == kNsFused)
+        ns_gemm_kernel<kNsFused><<<2 * grid_pairs, kThreads, kSmemBytes, s>>>(P);
+    else if (mode == kNsPersistent)
+        ns_gemm_kernel<kNsPersistent><<<2 * grid_pairs, kThreads, kSmemBytes, s>>>(P);
     else
-        ns_gemm_kernel<false><<<2 * grid_pairs, kThreads, kSmemBytes, s>>>(P);
+        ns_gemm_kernel<kNsPhased><<<2 * grid_pairs, kThreads, kSmemBytes, s>>>(P);
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) {
         cudaFuncAttributes fa{};
-        if (persistent)
-            cudaFuncGetAttributes(&fa, ns_gemm_kernel<true>);
+        if (mode == kNsFused)
+            cudaFuncGetAttributes(&fa, ns_gemm_kernel<kNsFused>);
+        else if (mode == kNsPersistent)
+            cudaFuncGetAttributes(&fa, ns_gemm_kernel<kNsPersistent>);
         else
-            cudaFuncGetAttributes(&fa, ns_gemm_kernel<false>);
+            cudaFuncGetAttributes(&fa, ns_gemm_kernel<kNsPhased>);
         std::fprintf(stderr,
                      "malt: ns_gemm_kernel<%d> launch (%d CTAs x %d threads, %zu B dynamic smem, "
                      "%zu B parameters) refused: %s; kernel uses %d registers, %zu B static "
                      "smem, allows %d threads and %d B dynamic smem per block\n",
-                     persistent ? 1 : 0, 2 * grid_pairs, kThreads, kSmemBytes, sizeof(NsParams),
+                     mode, 2 * grid_pairs, kThreads, kSmemBytes, sizeof(NsParams),
                      cudaGetErrorString(e), fa.numRegs, fa.sharedSizeBytes,
                      fa.maxThreadsPerBlock, fa.maxDynamicSharedSizeBytes);
         cudaGetLastError();

@@ -140,6 +140,15 @@ __device__ __forceinline__ void mbar_arrive_expect_tx_cluster(uint32_t cluster_b
                  ::"r"(cluster_bar), "r"(bytes) : "memory");
 }
 
+// Asynchronous 16-byte store (four 32-bit words, 16-byte aligned address) into
+// shared memory of a CTA of the cluster, completing 16 transaction bytes on
+// an mbarrier of that CTA.
+__device__ __forceinline__ void st_async_v4(uint32_t cluster_addr, int32_t a, int32_t b, int32_t c,
+                                            int32_t d, uint32_t cluster_bar) {
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, [%5];"
+                 ::"r"(cluster_addr), "r"(a), "r"(b), "r"(c), "r"(d), "r"(cluster_bar) : "memory");
+}
+
 // Relaxed arrive that also expects `bytes` transaction bytes on the phase.
 __device__ __forceinline__ void mbar_arrive_expect_tx_cluster_relaxed(uint32_t cluster_bar,
                                                                       uint32_t bytes) {

@@ -18,9 +18,10 @@
 //             grafted scale lr * alpha * ||O|| / (||D|| + eps) per matrix.
 //   apply     W <- (1 - lr wd) W - scale * L O R (Algorithm 1, W_t line).
 //
-// Template flag kRO: the block may read O through the read-only cache path.
-// True in the standalone kernels (O was written by an earlier launch); false
-// in the fused kernel, which writes O itself.
+// Template flag kL2: data that an earlier stage of the same launch may have
+// written (M, L, R, the partial sums, the per-matrix scalars, O) is read
+// through L2 only (ld.global.cg), so a stale L1 line is never used.  False in
+// the standalone kernels, where every input comes from an earlier launch.
 #pragma once
 #include <cuda_bf16.h>
 #include <cstdint>
@@ -67,16 +68,37 @@ __device__ __forceinline__ float block_sum(float v, float* sh /* >= 32 */, int t
     return s;
 }
 
-template <bool kRO>
+// Load paths: read-only cache, plain (L1 and L2), L2 only.
+enum LoadPath { kLdRO = 0, kLdPlain = 1, kLdL2 = 2 };
+
+template <int kPath>
 __device__ __forceinline__ uint4 ld_u4(const void* p) {
-    return kRO ? __ldg(reinterpret_cast<const uint4*>(p)) : *reinterpret_cast<const uint4*>(p);
+    const uint4* q = reinterpret_cast<const uint4*>(p);
+    return kPath == kLdRO ? __ldg(q) : kPath == kLdL2 ? __ldcg(q) : *q;
 }
 
+template <int kPath>
+__device__ __forceinline__ float4 ld_f4(const float* p) {
+    const float4* q = reinterpret_cast<const float4*>(p);
+    return kPath == kLdRO ? __ldg(q) : kPath == kLdL2 ? __ldcg(q) : *q;
+}
+
+template <int kPath>
+__device__ __forceinline__ float ld_f(const float* p) {
+    return kPath == kLdRO ? __ldg(p) : kPath == kLdL2 ? __ldcg(p) : *p;
+}
+
+// Path of data an earlier stage of the same launch may have written.
+template <bool kL2>
+struct Mut {
+    static constexpr int kPath = kL2 ? kLdL2 : kLdPlain;
+};
+
 // 8 consecutive elements (bf16 or fp32) at element offset off, as floats.
-template <bool kRO = true>
+template <int kPath = kLdRO>
 __device__ __forceinline__ void load8(const void* base, bool bf16, size_t off, float (&v)[8]) {
     if (bf16) {
-        const uint4 u = ld_u4<kRO>(static_cast<const __nv_bfloat16*>(base) + off);
+        const uint4 u = ld_u4<kPath>(static_cast<const __nv_bfloat16*>(base) + off);
         const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
@@ -85,15 +107,8 @@ __device__ __forceinline__ void load8(const void* base, bool bf16, size_t off, f
             v[2 * k + 1] = f.y;
         }
     } else {
-        const float4* p = reinterpret_cast<const float4*>(static_cast<const float*>(base) + off);
-        float4 a, b;
-        if (kRO) {
-            a = __ldg(p);
-            b = __ldg(p + 1);
-        } else {
-            a = p[0];
-            b = p[1];
-        }
+        const float* p = static_cast<const float*>(base) + off;
+        const float4 a = ld_f4<kPath>(p), b = ld_f4<kPath>(p + 4);
         v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
         v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
     }
@@ -145,7 +160,7 @@ __device__ __forceinline__ void stats_block(const MatDesc& d, const UserPtrs& up
             ok[u] = colok && row < m;
             if (ok[u]) {
                 const size_t off = static_cast<size_t>(row) * n + col;
-                load8<true>(up.g, gbf, off, gv[u]);
+                load8<kLdRO>(up.g, gbf, off, gv[u]);
                 const float4* mp = reinterpret_cast<const float4*>(Mp + off);
                 const float4 a = mp[0], b = mp[1];
                 mv[u][0] = a.x; mv[u][1] = a.y; mv[u][2] = a.z; mv[u][3] = a.w;
@@ -200,8 +215,10 @@ __device__ __forceinline__ void stats_block(const MatDesc& d, const UserPtrs& up
 // --------------------------------------------------------------- finalize
 // Entry `local` of the matrix's m + n statistics: row i = local (< m) or
 // column j = local - m.  identity (Muon): L = R = 1, statistics untouched.
+template <bool kL2 = false>
 __device__ __forceinline__ void finalize_entry(const MatDesc& d, const UserPtrs& up, int local,
                                                float mu2, float eps, int identity) {
+    constexpr int P = Mut<kL2>::kPath;
     if (identity) {
         if (local < d.m) d.L[local] = 1.f; else d.R[local - d.m] = 1.f;
         return;
@@ -209,14 +226,14 @@ __device__ __forceinline__ void finalize_entry(const MatDesc& d, const UserPtrs&
     if (local < d.m) {
         const int i = local;
         float s = 0.f;
-        for (int cb = 0; cb < d.stat_cb; ++cb) s += d.rowpart[static_cast<size_t>(cb) * d.m + i];
+        for (int cb = 0; cb < d.stat_cb; ++cb) s += ld_f<P>(d.rowpart + static_cast<size_t>(cb) * d.m + i);
         const float l = fmaf(mu2, up.l[i], (1.f - mu2) * s);
         up.l[i] = l;
         d.L[i] = powf(l + eps, -0.125f);
     } else {
         const int j = local - d.m;
         float s = 0.f;
-        for (int rb = 0; rb < d.stat_rb; ++rb) s += d.colpart[static_cast<size_t>(rb) * d.n + j];
+        for (int rb = 0; rb < d.stat_rb; ++rb) s += ld_f<P>(d.colpart + static_cast<size_t>(rb) * d.n + j);
         const float r = fmaf(mu2, up.r[j], (1.f - mu2) * s);
         up.r[j] = r;
         d.R[j] = powf(r + eps, -0.125f);
@@ -230,10 +247,11 @@ __device__ __forceinline__ void finalize_entry(const MatDesc& d, const UserPtrs&
 // tall matrix's NS frame is Mt^T, so its block walks four 64 x 64 sub-tiles
 // through shared memory (tile: 64 x 65 floats) and writes each transposed.
 // red: 8 float2.
-template <class Sync>
+template <bool kL2, class Sync>
 __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs& up, int local,
                                                int malter, int tid, float (*tile)[65],
                                                float2* red, Sync sync) {
+    constexpr int P = Mut<kL2>::kPath;
     const int m = d.m, n = d.n;
     const int tr = local / d.pre_tc, tc = local - tr * d.pre_tc;
     const int r0 = tr * kPreRows, c0 = tc * kPreCols;
@@ -249,8 +267,8 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
         const bool colok = col < n;
         float rj[8];
         if (colok) {
-            const float4 a = *reinterpret_cast<const float4*>(Rv + col);
-            const float4 b = *reinterpret_cast<const float4*>(Rv + col + 4);
+            const float4 a = ld_f4<P>(Rv + col);
+            const float4 b = ld_f4<P>(Rv + col + 4);
             rj[0] = a.x; rj[1] = a.y; rj[2] = a.z; rj[3] = a.w;
             rj[4] = b.x; rj[5] = b.y; rj[6] = b.z; rj[7] = b.w;
         }
@@ -266,11 +284,11 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
                 li[u] = 0.f;
                 if (ok[u]) {
                     const size_t off = static_cast<size_t>(row) * n + col;
-                    const float4 a = *reinterpret_cast<const float4*>(Mp + off);
-                    const float4 b = *reinterpret_cast<const float4*>(Mp + off + 4);
+                    const float4 a = ld_f4<P>(Mp + off);
+                    const float4 b = ld_f4<P>(Mp + off + 4);
                     mv[u][0] = a.x; mv[u][1] = a.y; mv[u][2] = a.z; mv[u][3] = a.w;
                     mv[u][4] = b.x; mv[u][5] = b.y; mv[u][6] = b.z; mv[u][7] = b.w;
-                    li[u] = Lv[row];
+                    li[u] = ld_f<P>(Lv + row);
                 }
             }
 #pragma unroll
@@ -287,7 +305,7 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
                 *reinterpret_cast<uint4*>(d.X0 + off) = pack8_bf16(v);
                 if (malter) {
                     float gv[8];
-                    load8<true>(up.g, gbf, off, gv);
+                    load8<kLdRO>(up.g, gbf, off, gv);
 #pragma unroll
                     for (int j = 0; j < 8; ++j) {
                         const float a = li[u] * gv[j] * rj[j];
@@ -303,7 +321,7 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
             if (cs >= n) break;                          // uniform across the block
             const int col = cs + cc;
             float4 R4 = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (col < n) R4 = *reinterpret_cast<const float4*>(Rv + col);
+            if (col < n) R4 = ld_f4<P>(Rv + col);
 #pragma unroll
             for (int pass = 0; pass < 4; ++pass) {
                 const int rr = pass * 16 + (t >> 4);
@@ -311,8 +329,8 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
                 float v0 = 0.f, v1 = 0.f, v2 = 0.f, v3 = 0.f;
                 if (row < m && col < n) {
                     const size_t off = static_cast<size_t>(row) * n + col;
-                    const float Li = Lv[row];
-                    const float4 mq = *reinterpret_cast<const float4*>(Mp + off);
+                    const float Li = ld_f<P>(Lv + row);
+                    const float4 mq = ld_f4<P>(Mp + off);
                     v0 = Li * mq.x * R4.x; v1 = Li * mq.y * R4.y;
                     v2 = Li * mq.z * R4.z; v3 = Li * mq.w * R4.w;
                     s_mt += v0 * v0 + v1 * v1 + v2 * v2 + v3 * v3;
@@ -377,14 +395,15 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
 
 // ------------------------------------------------------------------ norms
 // ||Mt||_F, 1 / (||Mt||_F + ns_eps) and ||L G R||_F^2 of one matrix (256 threads).
-template <class Sync>
+template <bool kL2, class Sync>
 __device__ __forceinline__ void norms_matrix(const MatDesc& d, MatScalars* sc, float ns_eps,
                                              int malter, int tid, float* red, Sync sync) {
+    constexpr int P = Mut<kL2>::kPath;
     const int tiles = d.pre_tr * d.pre_tc;
     float a = 0.f, b = 0.f;
     for (int i = tid; i < tiles; i += kThreads) {
-        a += d.prepart[2 * i];
-        b += d.prepart[2 * i + 1];
+        a += ld_f<P>(d.prepart + 2 * i);
+        b += ld_f<P>(d.prepart + 2 * i + 1);
     }
     a = block_sum(a, red, tid, kThreads, sync);
     b = block_sum(b, red, tid, kThreads, sync);
@@ -402,22 +421,29 @@ __device__ __forceinline__ void norms_matrix(const MatDesc& d, MatScalars* sc, f
 // block size), so the result does not depend on who runs it.
 constexpr int kScalarThreads = 128;
 
-template <class Sync>
+template <bool kL2, class Sync>
 __device__ __forceinline__ void scalars_matrix(const MatDesc& d, MatScalars* sc,
                                                const long long* tcount, const StepHyper& hp,
                                                int tid, float* red, Sync sync) {
+    constexpr int P = Mut<kL2>::kPath;
     float a = 0.f, b = 0.f;
     // One partial per epilogue warp per GEMM tile of the last iteration.
     if (tid < kScalarThreads) {
         for (int i = tid; i < kNsPartsPerTile * d.ns_tiles; i += kScalarThreads) {
-            a += d.nspart[2 * i];
-            b += d.nspart[2 * i + 1];
+            a += ld_f<P>(d.nspart + 2 * i);
+            b += ld_f<P>(d.nspart + 2 * i + 1);
         }
     }
     a = block_sum(a, red, tid, kScalarThreads, sync);
     b = block_sum(b, red, tid, kScalarThreads, sync);
     if (tid == 0) {
-        MatScalars s = *sc;
+        MatScalars s;
+        {
+            const float4 lo = ld_f4<P>(reinterpret_cast<const float*>(sc));
+            const float4 hi = ld_f4<P>(reinterpret_cast<const float*>(sc) + 4);
+            s.k = lo.x; s.norm_mt = lo.y; s.lgr_sq = lo.z; s.scale = lo.w;
+            s.norm_o = hi.x; s.norm_d = hi.y; s.alpha = hi.z; s.nu = hi.w;
+        }
         const double norm_o = sqrt(static_cast<double>(a));
         const double norm_d = sqrt(static_cast<double>(b));
         double alpha = 1.0;
@@ -440,12 +466,13 @@ __device__ __forceinline__ void scalars_matrix(const MatDesc& d, MatScalars* sc,
 }
 
 // ------------------------------------------------------------------ apply
+template <int P>
 __device__ __forceinline__ void apply8(const MatDesc& d, const UserPtrs& up, bool wbf, float s,
                                        float decay, int i, int j, const float (&o)[8]) {
     const size_t e = static_cast<size_t>(i) * d.n + j;
-    const float Li = d.L[i];
-    const float4 r0 = *reinterpret_cast<const float4*>(d.R + j);
-    const float4 r1 = *reinterpret_cast<const float4*>(d.R + j + 4);
+    const float Li = ld_f<P>(d.L + i);
+    const float4 r0 = ld_f4<P>(d.R + j);
+    const float4 r1 = ld_f4<P>(d.R + j + 4);
     const float rj[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
     float w[8];
     if (wbf) {
@@ -479,10 +506,12 @@ __device__ __forceinline__ void apply8(const MatDesc& d, const UserPtrs& up, boo
 // matrix, or rows [64 i, 64 i + 64) x columns [kPreCols j, ...) of a tall one
 // (whose O is stored n x m in the NS frame), read as four 64 x 64 tiles of
 // O^T through shared memory (tile: 64 x 65 floats).  s = the grafted scale.
-template <bool kRO, class Sync>
+template <bool kL2, class Sync>
 __device__ __forceinline__ void apply_block(const MatDesc& d, const UserPtrs& up, int local,
                                             float s, float decay, int tid, float (*tile)[65],
                                             Sync sync) {
+    constexpr int P = Mut<kL2>::kPath;
+    constexpr int PO = kL2 ? kLdL2 : kLdRO;       // O: read-only path unless written in-launch
     const int m = d.m, n = d.n;
     const bool wbf = d.w_bf16 != 0;
     if (d.trans) {
@@ -498,7 +527,7 @@ __device__ __forceinline__ void apply_block(const MatDesc& d, const UserPtrs& up
                 const int ii = (t & 7) * 8;               // 8 consecutive rows of W
                 float o[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
                 if (j0 + jj < n && i0 + ii < m)
-                    load8<kRO>(d.O, true, static_cast<size_t>(j0 + jj) * m + i0 + ii, o);
+                    load8<PO>(d.O, true, static_cast<size_t>(j0 + jj) * m + i0 + ii, o);
 #pragma unroll
                 for (int k = 0; k < 8; ++k) tile[ii + k][jj] = o[k];
             }
@@ -511,7 +540,7 @@ __device__ __forceinline__ void apply_block(const MatDesc& d, const UserPtrs& up
                     float o[8];
 #pragma unroll
                     for (int k = 0; k < 8; ++k) o[k] = tile[ii][jj + k];
-                    apply8(d, up, wbf, s, decay, i0 + ii, j0 + jj, o);
+                    apply8<P>(d, up, wbf, s, decay, i0 + ii, j0 + jj, o);
                 }
             }
             sync();                                       // tile is reused by the next sub-tile
@@ -526,8 +555,8 @@ __device__ __forceinline__ void apply_block(const MatDesc& d, const UserPtrs& up
         if (e >= total) break;
         const int i = e / n, j = e - i * n;
         float o[8];
-        load8<kRO>(d.O, true, static_cast<size_t>(e), o);
-        apply8(d, up, wbf, s, decay, i, j, o);
+        load8<PO>(d.O, true, static_cast<size_t>(e), o);
+        apply8<P>(d, up, wbf, s, decay, i, j, o);
     }
 }
 

@@ -56,7 +56,7 @@ finalize_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ p
     if (x == 0) *tcount += 1;                 // 1-based step count
     if (x >= total) return;
     const int g = find_mat(pref, nmat, x);
-    blk::finalize_entry(mats[g], ptrs[g], x - __ldg(pref + g), mu2, eps, identity);
+    blk::finalize_entry<false>(mats[g], ptrs[g], x - __ldg(pref + g), mu2, eps, identity);
 }
 
 // --------------------------------------------------------------- prescale
@@ -66,7 +66,7 @@ prescale_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ p
     __shared__ float tile[64][65];
     __shared__ float2 red[8];
     const int g = find_mat(pref, nmat, blockIdx.x);
-    blk::prescale_block(mats[g], ptrs[g], blockIdx.x - __ldg(pref + g), malter, threadIdx.x,
+    blk::prescale_block<false>(mats[g], ptrs[g], blockIdx.x - __ldg(pref + g), malter, threadIdx.x,
                         tile, red, blk::SyncBlock{});
 }
 
@@ -76,7 +76,7 @@ norms_kernel(const MatDesc* __restrict__ mats, MatScalars* __restrict__ scal, fl
              int malter) {
     __shared__ float red[32];
     const int g = blockIdx.x;
-    blk::norms_matrix(mats[g], scal + g, ns_eps, malter, threadIdx.x, red, blk::SyncBlock{});
+    blk::norms_matrix<false>(mats[g], scal + g, ns_eps, malter, threadIdx.x, red, blk::SyncBlock{});
 }
 
 // ---------------------------------------------------------------- scalars
@@ -85,7 +85,7 @@ scalars_kernel(const MatDesc* __restrict__ mats, MatScalars* __restrict__ scal,
                const long long* __restrict__ tcount, StepHyper hp) {
     __shared__ float red[32];
     const int g = blockIdx.x;
-    blk::scalars_matrix(mats[g], scal + g, tcount, hp, threadIdx.x, red, blk::SyncBlock{});
+    blk::scalars_matrix<false>(mats[g], scal + g, tcount, hp, threadIdx.x, red, blk::SyncBlock{});
 }
 
 // ------------------------------------------------------------------ apply
@@ -95,7 +95,7 @@ apply_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs
              float decay) {
     __shared__ float tile[64][65];
     const int g = find_mat(pref, nmat, blockIdx.x);
-    blk::apply_block<true>(mats[g], ptrs[g], blockIdx.x - __ldg(pref + g), scal[g].scale, decay,
+    blk::apply_block<false>(mats[g], ptrs[g], blockIdx.x - __ldg(pref + g), scal[g].scale, decay,
                            threadIdx.x, tile, blk::SyncBlock{});
 }
 
@@ -112,7 +112,7 @@ transpose_bf16_kernel(const __nv_bfloat16* __restrict__ src, __nv_bfloat16* __re
         const int rr = pass * 32 + (t >> 3), cc = (t & 7) * 8;
         float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         if (r0 + rr < rows && c0 + cc < cols)
-            blk::load8<true>(src, true, static_cast<size_t>(r0 + rr) * cols + c0 + cc, v);
+            blk::load8<blk::kLdRO>(src, true, static_cast<size_t>(r0 + rr) * cols + c0 + cc, v);
 #pragma unroll
         for (int k = 0; k < 8; ++k) tile[rr][cc + k] = v[k];
     }

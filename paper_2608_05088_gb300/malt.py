@@ -32,15 +32,19 @@ EXPORTS = ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
            "malt_debug_wait_timeout", "malt_profile_enable", "malt_profile_read",
            "malt_workspace_bytes", "malt_status_string", "malt_destroy_state",
            "malt_stats_noalloc", "malt_step_host", "muon_step", "malt_set_ns_schedule",
-           "malt_ns_schedule", "malt_debug_timeout_site")
+           "malt_ns_schedule", "malt_debug_timeout_site", "malt_set_overlap_groups")
 NOALLOC_SCRATCH_FLOATS = 1048576
 KIND_NAMES = ("bind", "stats", "finalize", "prescale", "norms", "ns_gram", "ns_poly", "ns_bx",
-              "scalars", "apply", "ns_persistent")
+              "scalars", "apply", "ns_persistent", "step_fused")
 NS_KINDS = ("ns_gram", "ns_poly", "ns_bx", "ns_persistent")
 # Newton-Schulz schedules (malt_set_ns_schedule)
 MALT_NS_PHASED = 0
 MALT_NS_PERSISTENT = 1
 MALT_NS_AUTO = 2
+MALT_NS_FUSED = 3
+# stage kinds of malt_ns_schedule
+STAGE_KIND_NAMES = ("gram", "poly", "bx", "stats", "finalize", "prescale", "norms", "scalars",
+                    "apply")
 
 
 class malt_param_t(ctypes.Structure):
@@ -112,7 +116,9 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.malt_debug_timeout_site.restype = ctypes.c_int
     lib.malt_set_ns_schedule.argtypes = [vp, i32]
     lib.malt_set_ns_schedule.restype = ctypes.c_int
-    lib.malt_ns_schedule.argtypes = [P(malt_param_t), i32, i32, P(i32), i64, P(i64)]
+    lib.malt_ns_schedule.argtypes = [P(malt_param_t), i32, i32, i32, i32, P(i32), i64, P(i64)]
+    lib.malt_set_overlap_groups.argtypes = [vp, i32]
+    lib.malt_set_overlap_groups.restype = ctypes.c_int
     lib.malt_ns_schedule.restype = ctypes.c_int
     for name in ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
                  "malt_set_scalars", "malt_check", "malt_debug_direction",
@@ -283,24 +289,29 @@ def malt_set_ns_schedule(st, schedule: int):
     _check(load().malt_set_ns_schedule(st, int(schedule)), "malt_set_ns_schedule")
 
 
-def malt_ns_schedule(shapes, ns_steps: int):
-    """The persistent Newton-Schulz work list for these (rows, cols) shapes,
-    computed on the host by the library (no GPU): an int32 array of shape
-    (items, 8) with columns group, s, matrix, tile row, tile column,
-    counter index, counter target, tiles of (s, matrix)."""
+def malt_ns_schedule(shapes, ns_steps: int, fused: bool = False, overlap_groups: int = 0):
+    """The work table of the persistent (or, with fused=True, the fused-step)
+    schedule for these (rows, cols) shapes, computed on the host by the
+    library (no GPU): an int32 array of shape (items, 8) with columns launch
+    group, stage, stage kind (STAGE_KIND_NAMES), matrix, local index,
+    counter index, counter target, items of (stage, matrix)."""
     import numpy as np
     arr = (malt_param_t * max(len(shapes), 1))()
     for i, (rows, cols) in enumerate(shapes):
         arr[i] = malt_param_t(None, MALT_F32, None, MALT_F32, None, None, None, rows, cols)
     lib = load()
     count = ctypes.c_int64(0)
-    _check(lib.malt_ns_schedule(arr, len(shapes), ns_steps, None, 0, ctypes.byref(count)),
-           "malt_ns_schedule")
+    _check(lib.malt_ns_schedule(arr, len(shapes), ns_steps, int(fused), overlap_groups, None, 0,
+                                ctypes.byref(count)), "malt_ns_schedule")
     out = np.zeros((count.value, 8), dtype=np.int32)
-    _check(lib.malt_ns_schedule(arr, len(shapes), ns_steps,
+    _check(lib.malt_ns_schedule(arr, len(shapes), ns_steps, int(fused), overlap_groups,
                                 out.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)),
                                 count.value, ctypes.byref(count)), "malt_ns_schedule")
     return out
+
+
+def malt_set_overlap_groups(st, groups: int):
+    _check(load().malt_set_overlap_groups(st, int(groups)), "malt_set_overlap_groups")
 
 
 # --- convenience wrapper ------------------------------------------------------
@@ -351,6 +362,9 @@ class MaltOptimizer:
 
     def set_ns_schedule(self, schedule: int):
         malt_set_ns_schedule(self.state, schedule)
+
+    def set_overlap_groups(self, groups: int):
+        malt_set_overlap_groups(self.state, groups)
 
     def profile(self, enable: bool = True):
         malt_profile_enable(self.state, enable)

@@ -18,24 +18,34 @@ RAGGED = ((200, 328), (392, 136), (8, 8), (136, 1000), (520, 520), (64, 2056), (
 TEN_CLASSES = tuple((64 * (i + 1), 512) for i in range(8)) + ((520, 8), (16, 16))
 
 
-def run_both(wl, steps, w_dtypes=None, ns_coeffs=None):
+# (schedule, overlap groups): the fused step with automatic, one and three runs
+SCHEDULES = [(malt.MALT_NS_PHASED, 0), (malt.MALT_NS_PERSISTENT, 0), (malt.MALT_NS_FUSED, 0),
+             (malt.MALT_NS_FUSED, 1), (malt.MALT_NS_FUSED, 3)]
+
+
+def run_both(wl, steps, w_dtypes=None, ns_coeffs=None, schedules=SCHEDULES):
+    """The same steps under every schedule: all results bitwise equal."""
     import torch
     kw = {} if ns_coeffs is None else {"ns_coeffs": ns_coeffs}
     out = []
-    for sched in (malt.MALT_NS_PHASED, malt.MALT_NS_PERSISTENT):
+    for sched, groups in schedules:
         run = Run(wl, check=[], w_dtypes=w_dtypes, **kw)
         run.opt.set_ns_schedule(sched)
+        run.opt.set_overlap_groups(groups)
         for _ in range(steps):
             run.step(oracle=False)
-        assert run.status() == malt.MALT_OK
+        assert run.status() == malt.MALT_OK, (sched, groups, run.opt.timeout_site())
         torch.cuda.synchronize()
         res = [run.host(t) for t in run.W + run.M + run.l + run.r]
         res += [run.host(run.opt.direction(i)) for i in range(len(wl.shapes))]
         res.append(np.asarray(run.opt.debug_scalars()))
+        nu, t = run.opt.scalars()
+        res += [np.asarray(nu), np.asarray([t])]
         out.append(res)
         run.close()
-    for a, b in zip(*out):
-        assert np.array_equal(a, b)
+    for (sched, groups), res in zip(schedules[1:], out[1:]):
+        for i, (a, b) in enumerate(zip(out[0], res)):
+            assert np.array_equal(a, b), (sched, groups, i)
 
 
 @pytest.mark.parametrize("variant", ["malt", "malter"])
@@ -57,6 +67,30 @@ def test_two_launch_groups_bitwise():
 
 def test_gpt2_large_layers_bitwise():
     wl = inputs.first_layers(inputs.WORKLOADS["gpt2_large"], 2)
+    run_both(wl, 2)
+
+
+@pytest.mark.parametrize("variant", ["malt", "malter", "muon"])
+def test_fused_against_oracle(variant):
+    """The whole step in one launch (statistics to apply on the GEMM
+    kernel's epilogue warps), against the oracle, 3 steps (the inputs of the
+    phased parity tests of tests/test_gpu_parity.py)."""
+    shapes = RAGGED[:6] if variant == "muon" else RAGGED
+    seed = 36 if variant == "muon" else 31
+    wl = inputs.Workload("fusedo", seed, shapes, "f32", 1.5, 0.02, variant, 3)
+    run = Run(wl, w_dtypes=["f32", "bf16"] * (len(shapes) // 2))
+    run.opt.set_ns_schedule(malt.MALT_NS_FUSED)
+    run.opt.set_overlap_groups(2)
+    for s in range(wl.steps):
+        run.step()
+        assert run.status() == malt.MALT_OK, run.opt.timeout_site()
+        for i in range(len(wl.shapes)):
+            run.assert_close(i, f"{variant} step {s}")
+    run.close()
+
+
+def test_fused_muon_bitwise():
+    wl = inputs.Workload("fusedmu", 56, RAGGED[:6], "f32", 1.5, 0.02, "muon", 2)
     run_both(wl, 2)
 
 

@@ -1,21 +1,26 @@
-"""The persistent Newton-Schulz schedule's work list, checked on the host.
+"""The persistent work tables, checked on the host.
 
-The library computes the list with the same decode the kernel runs
-(malt_ns_schedule needs no GPU).  The Orth step of Algorithm 1 iterates
-A = X X^T, B' = aI + bA + cA^2, X <- B' X on each matrix's own data, so:
-  * every 256 x 256 tile of every product of every iteration of every matrix
-    appears exactly once (the upper triangle for the symmetric A and B');
-  * a tile waits exactly for the previous product of its own matrix, complete;
-  * the list is topologically ordered: when a tile is claimed, every tile it
-    waits for was claimed before it.  Claims happen only in running CTAs, so
-    this order is what makes the schedule deadlock-free.
+The library builds the tables the persistent launches claim from with the
+same code the GPU path uses (malt_ns_schedule needs no GPU).  The Orth step
+of Algorithm 1 iterates A = X X^T, B' = aI + bA + cA^2, X <- B' X on each
+matrix's own data, and the fused step chains the HBM-bound stages of each
+matrix around them (statistics, finalize, prescale, norms; scalars, apply),
+so for each table:
+  * every item of every stage of every matrix appears exactly once (all
+    256 x 256 tiles of a product, the upper triangle for the symmetric A and
+    B'; every block pair of a memory stage);
+  * an item waits exactly for the previous stage of its own matrix, complete;
+  * the table is topologically ordered: when an item is claimed, every item
+    it waits for was claimed before it.  Claims happen only in running CTAs,
+    so this order is what makes the schedule deadlock-free.
 """
 import numpy as np
 import pytest
 
 from paper_2608_05088_gb300 import build, inputs
 
-SIGNALS_PER_TILE = 16   # epilogue warps of a CTA pair
+SIGNALS_PER_ITEM = 16   # epilogue warps of a CTA pair
+STATS, FINALIZE, PRESCALE, NORMS, SCALARS, APPLY = 3, 4, 5, 6, 7, 8
 
 
 @pytest.fixture(scope="module")
@@ -25,47 +30,61 @@ def malt():
     return m
 
 
-def tiles(n):
-    return (n + 255) // 256
+def cdiv(a, b):
+    return (a + b - 1) // b
 
 
-def expected_tiles(rows, cols, s):
+def expected_items(rows, cols, kind):
     p, q = min(rows, cols), max(rows, cols)
-    kind = s % 3
+    tp, tq = cdiv(p, 256), cdiv(q, 256)
     if kind == 2:
-        return {(i, j) for i in range(tiles(p)) for j in range(tiles(q))}
-    return {(i, j) for i in range(tiles(p)) for j in range(i, tiles(p))}
+        return tp * tq
+    if kind in (0, 1):
+        return tp * (tp + 1) // 2
+    if kind == STATS:
+        return cdiv(cdiv(rows, 64) * cdiv(cols, 256), 2)
+    if kind == PRESCALE:
+        return cdiv(cdiv(rows, 64) * cdiv(cols, 256), 2)
+    if kind == APPLY:
+        blocks = cdiv(rows, 64) * cdiv(cols, 256) if rows > cols else cdiv(rows * cols, 16384)
+        return cdiv(blocks, 2)
+    return 1
 
 
-def check_schedule(sched, shapes, k):
+def stage_kinds(k, fused):
+    kinds = [0, 1, 2] * k
+    return [STATS, FINALIZE, PRESCALE, NORMS] + kinds + [SCALARS, APPLY] if fused else kinds
+
+
+def check_table(tab, shapes, k, fused):
     n = len(shapes)
+    kinds = stage_kinds(k, fused)
     seen = {}
-    for g, s, mat, mt, nt, dep, target, ntiles in sched:
-        key = (int(s), int(mat))
-        seen.setdefault(key, []).append((int(mt), int(nt)))
+    for grp, st, kind, mat, local, dep, target, nitems in tab:
+        assert kind == kinds[st]
         rows, cols = shapes[mat]
-        assert ntiles == len(expected_tiles(rows, cols, s))
-        if s == 0:
-            assert dep == -1
+        assert nitems == expected_items(rows, cols, kind), (st, kind, mat)
+        seen.setdefault((int(st), int(mat)), []).append(int(local))
+        if st == 0:
+            assert dep == -1 and target == 0
         else:
-            assert dep == (s - 1) * n + mat
-            assert target == SIGNALS_PER_TILE * len(expected_tiles(rows, cols, s - 1))
-    assert set(seen) == {(s, i) for s in range(3 * k) for i in range(n)}
-    for (s, mat), tl in seen.items():
-        assert len(tl) == len(set(tl)), (s, mat)
-        assert set(tl) == expected_tiles(*shapes[mat], s), (s, mat)
-    # topological order per launch group: replay the claims with every tile
-    # finishing at once; each tile's counter must be complete when claimed
-    for grp in np.unique(sched[:, 0]):
-        ctr = np.zeros(3 * k * n, dtype=np.int64)
+            assert dep == (st - 1) * n + mat
+            assert target == SIGNALS_PER_ITEM * expected_items(rows, cols, kinds[st - 1])
+    assert set(seen) == {(s, i) for s in range(len(kinds)) for i in range(n)}
+    for (st, mat), locs in seen.items():
+        assert sorted(locs) == list(range(expected_items(*shapes[mat], kinds[st]))), (st, mat)
+    # topological order per launch group: replay the claims with every item
+    # finishing at once; each item's counter must be complete when claimed
+    for grp in np.unique(tab[:, 0]):
+        ctr = np.zeros(len(kinds) * n, dtype=np.int64)
         mats_here = set()
-        for _, s, mat, mt, nt, dep, target, ntiles in sched[sched[:, 0] == grp]:
+        for _, st, kind, mat, local, dep, target, nitems in tab[tab[:, 0] == grp]:
             mats_here.add(int(mat))
             if dep >= 0:
-                assert ctr[dep] == target, (s, mat, mt, nt)
-            ctr[s * n + mat] += SIGNALS_PER_TILE
-        # a matrix's whole solve runs in one launch
-        assert not mats_here & set(sched[sched[:, 0] != grp][:, 2].tolist())
+                assert ctr[dep] == target, (st, mat, local)
+            ctr[st * n + mat] += SIGNALS_PER_ITEM
+        # a matrix's whole step runs in one launch
+        assert not mats_here & set(tab[tab[:, 0] != grp][:, 3].tolist())
 
 
 RAGGED = [(200, 328), (392, 136), (8, 8), (136, 1000), (520, 520), (64, 2056), (1032, 264),
@@ -73,30 +92,48 @@ RAGGED = [(200, 328), (392, 136), (8, 8), (136, 1000), (520, 520), (64, 2056), (
 
 
 @pytest.mark.parametrize("k", [1, 2, 5])
-def test_ragged_shapes(malt, k):
-    sched = malt.malt_ns_schedule(RAGGED, k)
-    check_schedule(sched, RAGGED, k)
+def test_products_ragged(malt, k):
+    check_table(malt.malt_ns_schedule(RAGGED, k), RAGGED, k, False)
+
+
+@pytest.mark.parametrize("groups", [0, 1, 2, 3, 8])
+def test_fused_ragged(malt, groups):
+    tab = malt.malt_ns_schedule(RAGGED, 3, fused=True, overlap_groups=groups)
+    check_table(tab, RAGGED, 3, True)
 
 
 def test_gpt2_large(malt):
     shapes = list(inputs.WORKLOADS["gpt2_large"].shapes)
-    sched = malt.malt_ns_schedule(shapes, 5)
-    check_schedule(sched, shapes, 5)
+    tab = malt.malt_ns_schedule(shapes, 5)
+    check_table(tab, shapes, 5, False)
     # 36 of each of 1280x3840, 1280^2, 1280x5120, 5120x1280 (frames 1280 x
     # {3840, 1280, 5120, 5120}): 15 upper tiles per Gram / Poly, 5 x q/256 per BX
     per_iter = 144 * 15 * 2 + 36 * (5 * 15 + 5 * 5 + 2 * 5 * 20)
-    assert len(sched) == 5 * per_iter
+    assert len(tab) == 5 * per_iter
     # heaviest Gram reductions (q = 5120) are claimed first
-    first = sched[: 72 * 15]
-    assert all(max(shapes[m]) == 5120 for m in first[:, 2])
+    first = tab[: 72 * 15]
+    assert all(max(shapes[m]) == 5120 for m in first[:, 3])
+
+
+def test_gpt2_large_fused(malt):
+    shapes = list(inputs.WORKLOADS["gpt2_large"].shapes)
+    tab = malt.malt_ns_schedule(shapes, 5, fused=True)
+    check_table(tab, shapes, 5, True)
+    # the memory stages of later runs are interleaved with earlier products
+    kinds = tab[:, 2]
+    first_product = int(np.argmax(kinds <= 2))
+    last_product = len(kinds) - 1 - int(np.argmax(kinds[::-1] <= 2))
+    inside = kinds[first_product:last_product]
+    assert np.sum(inside > 2) > 0.5 * np.sum(kinds > 2)
 
 
 def test_more_classes_than_one_launch(malt):
     # ten distinct NS frames: two launch groups (at most eight classes each)
     shapes = [(64 * (i + 1), 512) for i in range(8)] + [(520, 8), (16, 16)]
-    sched = malt.malt_ns_schedule(shapes, 3)
-    assert set(np.unique(sched[:, 0]).tolist()) == {0, 1}
-    check_schedule(sched, shapes, 3)
+    for fused in (False, True):
+        tab = malt.malt_ns_schedule(shapes, 3, fused=fused)
+        assert set(np.unique(tab[:, 0]).tolist()) == {0, 1}
+        check_table(tab, shapes, 3, fused)
 
 
 def test_bad_arguments(malt):
@@ -106,3 +143,5 @@ def test_bad_arguments(malt):
         malt.malt_ns_schedule([(256, 512)], 65)
     with pytest.raises(malt.MaltError):
         malt.malt_ns_schedule([(250, 512)], 5)
+    with pytest.raises(malt.MaltError):
+        malt.malt_ns_schedule([(256, 512)], 5, fused=True, overlap_groups=65)
