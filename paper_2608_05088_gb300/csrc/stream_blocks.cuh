@@ -491,12 +491,9 @@ __device__ __forceinline__ void scalars_matrix(const MatDesc& d, MatScalars* sc,
 }
 
 // ------------------------------------------------------------------ apply
-// W <- decay W - s L_i O R_j for 8 consecutive elements of row i, from the
-// raw W bits wq (one uint4 of bf16, or two uint4 holding 8 floats).
 template <int P>
-__device__ __forceinline__ void apply8_w(const MatDesc& d, const UserPtrs& up, bool wbf, float s,
-                                         float decay, int i, int j, const float (&o)[8],
-                                         const uint4 (&wq)[2]) {
+__device__ __forceinline__ void apply8(const MatDesc& d, const UserPtrs& up, bool wbf, float s,
+                                       float decay, int i, int j, const float (&o)[8]) {
     const size_t e = static_cast<size_t>(i) * d.n + j;
     const float Li = ld_f<P>(d.L + i);
     const float4 r0 = ld_f4<P>(d.R + j);
@@ -504,7 +501,8 @@ __device__ __forceinline__ void apply8_w(const MatDesc& d, const UserPtrs& up, b
     const float rj[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
     float w[8];
     if (wbf) {
-        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&wq[0]);
+        const uint4 u = *reinterpret_cast<const uint4*>(static_cast<__nv_bfloat16*>(up.w) + e);
+        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
             const float2 f = __bfloat1622float2(h[k]);
@@ -512,8 +510,8 @@ __device__ __forceinline__ void apply8_w(const MatDesc& d, const UserPtrs& up, b
             w[2 * k + 1] = f.y;
         }
     } else {
-        const float4 a = *reinterpret_cast<const float4*>(&wq[0]);
-        const float4 b = *reinterpret_cast<const float4*>(&wq[1]);
+        const float4* wp = reinterpret_cast<const float4*>(static_cast<float*>(up.w) + e);
+        const float4 a = wp[0], b = wp[1];
         w[0] = a.x; w[1] = a.y; w[2] = a.z; w[3] = a.w;
         w[4] = b.x; w[5] = b.y; w[6] = b.z; w[7] = b.w;
     }
@@ -527,22 +525,6 @@ __device__ __forceinline__ void apply8_w(const MatDesc& d, const UserPtrs& up, b
         wp[0] = make_float4(w[0], w[1], w[2], w[3]);
         wp[1] = make_float4(w[4], w[5], w[6], w[7]);
     }
-}
-
-template <int P>
-__device__ __forceinline__ void apply8(const MatDesc& d, const UserPtrs& up, bool wbf, float s,
-                                       float decay, int i, int j, const float (&o)[8]) {
-    const size_t e = static_cast<size_t>(i) * d.n + j;
-    uint4 wq[2];
-    if (wbf) {
-        wq[0] = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(up.w) + e);
-        wq[1] = make_uint4(0u, 0u, 0u, 0u);
-    } else {
-        const uint4* wp = reinterpret_cast<const uint4*>(static_cast<const float*>(up.w) + e);
-        wq[0] = wp[0];
-        wq[1] = wp[1];
-    }
-    apply8_w<P>(d, up, wbf, s, decay, i, j, o, wq);
 }
 
 // Block `local` of the apply pass: kApplyElems contiguous elements of a wide
@@ -561,59 +543,19 @@ __device__ __forceinline__ void apply_block(const MatDesc& d, const UserPtrs& up
         const int tiles_c = (n + kPreCols - 1) / kPreCols;
         const int i0 = (local / tiles_c) * 64, c0 = (local % tiles_c) * kPreCols;
         const int t = tid;
-        constexpr int kSubs = kPreCols / 64;
-        // O of each 64 x 64 sub-tile (two rows of the NS-frame O = columns of
-        // W, 8 consecutive bf16 per thread) is loaded two sub-tiles ahead, and
-        // a sub-tile's W is loaded before its O goes through shared memory.
-        auto load_o = [&](int sub, uint4 (&dst)[2]) {
+        for (int sub = 0; sub < kPreCols / 64; ++sub) {
             const int j0 = c0 + sub * 64;
+            if (j0 >= n) break;                           // uniform across the block
 #pragma unroll
             for (int pass = 0; pass < 2; ++pass) {
                 const int jj = pass * 32 + (t >> 3);      // row of O_ns = column of W
                 const int ii = (t & 7) * 8;               // 8 consecutive rows of W
-                dst[pass] = (j0 + jj < n && i0 + ii < m)
-                                ? ld_u4<PO>(d.O + static_cast<size_t>(j0 + jj) * m + i0 + ii)
-                                : make_uint4(0u, 0u, 0u, 0u);
+                float o[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+                if (j0 + jj < n && i0 + ii < m)
+                    load8<PO>(d.O, true, static_cast<size_t>(j0 + jj) * m + i0 + ii, o);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) tile[ii + k][jj] = o[k];
             }
-        };
-        uint4 oq[2][2];
-        load_o(0, oq[0]);
-        load_o(1, oq[1]);
-#pragma unroll
-        for (int sub = 0; sub < kSubs; ++sub) {
-            const int j0 = c0 + sub * 64;
-            if (j0 >= n) break;                           // uniform across the block
-            // this thread's W elements of the sub-tile: rows ii of both passes
-            uint4 wq[2][2];
-#pragma unroll
-            for (int pass = 0; pass < 2; ++pass) {
-                const int ii = pass * 32 + (t >> 3);
-                const int jj = (t & 7) * 8;
-                wq[pass][0] = wq[pass][1] = make_uint4(0u, 0u, 0u, 0u);
-                if (i0 + ii < m && j0 + jj < n) {
-                    const size_t e = static_cast<size_t>(i0 + ii) * n + j0 + jj;
-                    if (wbf) {
-                        wq[pass][0] = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(up.w) + e);
-                    } else {
-                        const uint4* wp = reinterpret_cast<const uint4*>(static_cast<const float*>(up.w) + e);
-                        wq[pass][0] = wp[0];
-                        wq[pass][1] = wp[1];
-                    }
-                }
-            }
-#pragma unroll
-            for (int pass = 0; pass < 2; ++pass) {
-                const int jj = pass * 32 + (t >> 3);
-                const int ii = (t & 7) * 8;
-                const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&oq[sub & 1][pass]);
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    const float2 f = __bfloat1622float2(h[k]);
-                    tile[ii + 2 * k][jj] = f.x;
-                    tile[ii + 2 * k + 1][jj] = f.y;
-                }
-            }
-            if (sub + 2 < kSubs) load_o(sub + 2, oq[sub & 1]);
             sync();
 #pragma unroll
             for (int pass = 0; pass < 2; ++pass) {
@@ -623,7 +565,7 @@ __device__ __forceinline__ void apply_block(const MatDesc& d, const UserPtrs& up
                     float o[8];
 #pragma unroll
                     for (int k = 0; k < 8; ++k) o[k] = tile[ii][jj + k];
-                    apply8_w<P>(d, up, wbf, s, decay, i0 + ii, j0 + jj, o, wq[pass]);
+                    apply8<P>(d, up, wbf, s, decay, i0 + ii, j0 + jj, o);
                 }
             }
             sync();                                       // tile is reused by the next sub-tile

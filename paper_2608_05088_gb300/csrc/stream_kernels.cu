@@ -89,8 +89,7 @@ scalars_kernel(const MatDesc* __restrict__ mats, MatScalars* __restrict__ scal,
 }
 
 // ------------------------------------------------------------------ apply
-// Five blocks per SM: the wide-matrix stream needs the occupancy.
-__global__ void __launch_bounds__(256, 5)
+__global__ void __launch_bounds__(256)
 apply_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
              const MatScalars* __restrict__ scal, const int32_t* __restrict__ pref, int nmat,
              float decay) {
