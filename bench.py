@@ -240,6 +240,56 @@ def workload_config(wl):
                 wl.elements * 26 / 1e9)}
 
 
+# ------------------------------------------------------- cuBLAS comparison
+def run_compare_cublas(args):
+    """The GEMM shape of GPT-2 Large's B*X product for its 36 1280x5120
+    matrices, timed through cuBLAS and through the library (context for the
+    Newton-Schulz kernel's tensor-pipe efficiency; not a bench line)."""
+    import torch
+    import paper_2608_05088_gb300.malt as malt
+    from paper_2608_05088_gb300 import build, inputs
+    build.build()
+    dev = torch.device("cuda:0")
+    flops = 2.0 * 36 * 1280 * 1280 * 5120
+    a = torch.randn(36, 1280, 1280, device=dev, dtype=torch.bfloat16)
+    b = torch.randn(36, 1280, 5120, device=dev, dtype=torch.bfloat16)
+    for _ in range(args.warmup):
+        torch.matmul(a, b)
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        torch.matmul(a, b)
+    e1.record()
+    torch.cuda.synchronize()
+    cub_ms = e0.elapsed_time(e1) / args.steps
+    del a, b
+    wl = inputs.Workload("bx36", 81, ((1280, 5120),) * 36, "bf16", 1.5, 0.0007, "malt", 1)
+    W = [torch.from_numpy(w).to(dev).to(torch.bfloat16) for w in inputs.initial_weights(wl)]
+    G = [torch.from_numpy(g).to(dev) for g in inputs.gradients_for_step(wl, 0)]
+    M = [torch.empty(s_, dtype=torch.float32, device=dev) for s_ in wl.shapes]
+    l = [torch.empty(s_[0], dtype=torch.float32, device=dev) for s_ in wl.shapes]
+    r = [torch.empty(s_[1], dtype=torch.float32, device=dev) for s_ in wl.shapes]
+    opt = malt.MaltOptimizer(list(zip(W, G, M, l, r)))
+    opt.set_ns_schedule(malt.MALT_NS_PHASED)
+    hp = malt.hparams(lr=wl.lr)
+    for _ in range(args.warmup):
+        opt.step(hp)
+    torch.cuda.synchronize()
+    opt.profile(True)
+    opt.profile_read()
+    for _ in range(max(1, args.steps // 5)):
+        opt.step(hp)
+    prof = opt.profile_read()
+    opt.profile(False)
+    ours_ms = prof["ns_bx"][0] / prof["ns_bx"][1]
+    opt.close()
+    print(json.dumps({"compare": "B*X product, 36 x (1280x1280 @ 1280x5120) bf16",
+                      "cublas_ms": cub_ms, "cublas_tflops": flops / cub_ms / 1e9,
+                      "library_ms": ours_ms, "library_tflops": flops / ours_ms / 1e9}), flush=True)
+
+
 # --------------------------------------------------------------------- MALT
 def run_malt(args):
     import numpy as np
@@ -473,10 +523,15 @@ def main():
                     help="fused schedule: runs of matrices overlapped (0: automatic)")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling only: the first N layers of the workload")
+    ap.add_argument("--compare-cublas", action="store_true",
+                    help="one B*X-shaped product (36 x 1280^2 @ 1280x5120, bf16) through "
+                         "cuBLAS (torch.matmul) and through this library's phased B*X launch")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.impl == "reference":
+    if args.compare_cublas:
+        run_compare_cublas(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_malt(args)
