@@ -167,6 +167,7 @@ struct NsParams {
     int32_t with_stats;           // 0 for Muon through the same engine (momentum only)
     int32_t identity;             // 1 for Muon: L = R = 1
 };
+static_assert(sizeof(NsParams) <= 32764, "NsParams is passed by value as the kernel parameter");
 
 // One decoded work item: a 256 x 256 output tile of one product.
 struct NsWork {

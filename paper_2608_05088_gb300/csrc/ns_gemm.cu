@@ -23,11 +23,14 @@
 // Work split.  A cluster of two CTAs (a CTA pair on two SMs) computes one
 // 256 x 256 output tile per turn: CTA r owns rows [128 r, 128 r + 128) of the
 // tile in its own TMEM.  Per 64-wide reduction slice each CTA loads its 128
-// rows of A and its half (128 N-rows or N-columns) of B, 32 KB, into a
-// kStages-deep ring; the MMA, issued by one thread of the even CTA, reads both
-// CTAs' shared memory.  Each SM therefore pulls 32 KB from L2 per
-// 128 x 256 x 64 of MMA work instead of 48 KB, and the 6-stage ring covers
-// half as much again of load latency.
+// rows of A and its half (128 N-rows or N-columns) of B, 32 KB, into one of
+// kStages slice slots; the MMA, issued by one thread of the even CTA, reads
+// both CTAs' shared memory.  Each SM therefore pulls 32 KB from L2 per
+// 128 x 256 x 64 of MMA work instead of 48 KB.  The slots are filled,
+// awaited and released in groups of kGroup slices (a 3-stage ring of 128-wide
+// reductions): every barrier wait and commit on the MMA thread's path stalls
+// the tensor pipe a little, and one per 8 MMAs measured 4 % faster on B*X
+// than one per 4.
 //
 // Roles per CTA: warp 0 issues TMA loads (the peer's loads complete on the
 // even CTA's full barrier, and both producers arrive on it), warp 1 owns
@@ -85,7 +88,13 @@ constexpr int kEpiChunks = kEpiCols / 32;
 constexpr int kHalfN = kBN / 2;                        // B rows (or columns) per CTA
 constexpr uint32_t kABytes = kBM * kBK * 2;            // 16 KB
 constexpr uint32_t kBBytes = kHalfN * kBK * 2;         // 16 KB
-constexpr uint32_t kStageBytes = kABytes + kBBytes;
+constexpr uint32_t kStageBytes = kABytes + kBBytes;     // one 64-wide reduction slice
+// Ring granularity: the producer fills, and the MMA thread waits for and
+// releases, kGroup slices at a time.  A barrier wait and a commit sit on the
+// MMA issue path once per kGroup slices (8 MMAs) instead of once per 4 MMAs.
+constexpr int kGroup = 2;
+constexpr int kRing = kStages / kGroup;
+static_assert(kStages % kGroup == 0, "the slice slots form whole ring stages");
 constexpr uint32_t kTmemCols = 2 * kBN;
 constexpr uint32_t kIdesc = idesc_bf16_f32(kTileM, kBN);
 constexpr uint32_t kIdescBmn = idesc_bf16_f32(kTileM, kBN, true);
@@ -286,8 +295,8 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
     constexpr bool kPersistent = kMode != kNsPhased;   // table-driven, claimed dynamically
     constexpr bool kFused = kMode == kNsFused;         // the table also holds memory stages
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t full_bar[kStages];
-    __shared__ __align__(8) uint64_t empty_bar[kStages];
+    __shared__ __align__(8) uint64_t full_bar[kRing];
+    __shared__ __align__(8) uint64_t empty_bar[kRing];
     __shared__ __align__(8) uint64_t tfull_bar[2];
     __shared__ __align__(8) uint64_t tempty_bar[2];
     __shared__ __align__(8) uint64_t drain_bar;
@@ -309,9 +318,9 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
     const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kStages; ++s) {
+        for (int s = 0; s < kRing; ++s) {
             // Both producers arrive on the even CTA's full barrier for every
-            // slice (the even one with the pair's transaction bytes), so the
+            // ring stage (the even one with the pair's transaction bytes), so the
             // MMA never consumes a slice the odd producer has not reached --
             // even when the odd CTA loads nothing (M or N within its partner's
             // half) -- and the odd producer can never fall a whole parity
@@ -465,25 +474,29 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                 const int a_row = w.mt * kTileM + rank * kBM;
                 const int n0 = w.nt * kBN + rank * kHalfN;
                 bool ok = true;
-                for (int kb = 0; kb < nkb; ++kb) {
+                for (int k0 = 0; k0 < nkb; k0 += kGroup) {
                     if (!mbar_wait_cluster_bounded(&empty_bar[stage], phase ^ 1u, budget, abort_flag)) {
-                        raise_timeout(P, abort_flag, kSiteStage, item, kb);
+                        raise_timeout(P, abort_flag, kSiteStage, item, k0);
                         ok = false;
                         break;
                     }
-                    uint8_t* sa = smem + stage * kStageBytes;
+                    const int nsub = min(kGroup, nkb - k0);
                     const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
-                    if (leader) mbar_arrive_expect_tx(&full_bar[stage], bytes_pair);
-                    if (load_a) tma_load_3d_pair(sa, op.a, kb * kBK, a_row, w.b, fb);
-                    if (b_mn) {
-                        for (int j = 0; j < nb_self; ++j)
-                            tma_load_3d_pair(sa + kABytes + j * kMnBoxBytes, op.b,
-                                             n0 + j * kBMN, kb * kBK, w.b, fb);
-                    } else if (nb_self > 0) {
-                        tma_load_3d_pair(sa + kABytes, op.b, kb * kBK, n0, w.b, fb);
+                    if (leader) mbar_arrive_expect_tx(&full_bar[stage], nsub * bytes_pair);
+                    for (int j = 0; j < nsub; ++j) {
+                        const int kb = k0 + j;
+                        uint8_t* sa = smem + (stage * kGroup + j) * kStageBytes;
+                        if (load_a) tma_load_3d_pair(sa, op.a, kb * kBK, a_row, w.b, fb);
+                        if (b_mn) {
+                            for (int jb = 0; jb < nb_self; ++jb)
+                                tma_load_3d_pair(sa + kABytes + jb * kMnBoxBytes, op.b,
+                                                 n0 + jb * kBMN, kb * kBK, w.b, fb);
+                        } else if (nb_self > 0) {
+                            tma_load_3d_pair(sa + kABytes, op.b, kb * kBK, n0, w.b, fb);
+                        }
                     }
                     if (!leader) mbar_arrive_cluster_relaxed(fb);
-                    if (++stage == kStages) { stage = 0; phase ^= 1u; }
+                    if (++stage == kRing) { stage = 0; phase ^= 1u; }
                 }
                 if (!ok) break;
             }
@@ -538,34 +551,38 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + acc * kBN;
                 bool ok = true;
-                for (int kb = 0; kb < nkb; ++kb) {
+                for (int k0 = 0; k0 < nkb; k0 += kGroup) {
                     if (!mbar_wait_cluster_bounded(&full_bar[stage], phase, budget, abort_flag)) {
-                        raise_timeout(P, abort_flag, kSiteStageFull, item, kb);
+                        raise_timeout(P, abort_flag, kSiteStageFull, item, k0);
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t sa = smem_u32(smem + stage * kStageBytes);
-                    const uint64_t da = smem_desc_k_sw128(sa);
-                    if (b_mn) {
-                        const uint64_t db = smem_desc_mn_sw128(sa + kABytes, kMnLbo);
+                    const int nsub = min(kGroup, nkb - k0);
+                    for (int j = 0; j < nsub; ++j) {
+                        const int kb = k0 + j;
+                        const uint32_t sa = smem_u32(smem + (stage * kGroup + j) * kStageBytes);
+                        const uint64_t da = smem_desc_k_sw128(sa);
+                        if (b_mn) {
+                            const uint64_t db = smem_desc_mn_sw128(sa + kABytes, kMnLbo);
 #pragma unroll
-                        for (int kk = 0; kk < kBK / 16; ++kk) {
-                            // A: +32 bytes along K; B: +16 K-rows = two 1024-byte atoms.
-                            tc_mma_bf16_pair(d_tmem, da + 2 * kk, db + (2048u >> 4) * kk,
-                                             kIdescBmn, (kb | kk) != 0 ? 1u : 0u);
-                        }
-                    } else {
-                        const uint64_t db = smem_desc_k_sw128(sa + kABytes);
+                            for (int kk = 0; kk < kBK / 16; ++kk) {
+                                // A: +32 bytes along K; B: +16 K-rows = two 1024-byte atoms.
+                                tc_mma_bf16_pair(d_tmem, da + 2 * kk, db + (2048u >> 4) * kk,
+                                                 kIdescBmn, (kb | kk) != 0 ? 1u : 0u);
+                            }
+                        } else {
+                            const uint64_t db = smem_desc_k_sw128(sa + kABytes);
 #pragma unroll
-                        for (int kk = 0; kk < kBK / 16; ++kk) {
-                            // +32 bytes along K per 16-element MMA slice (encoded >> 4).
-                            tc_mma_bf16_pair(d_tmem, da + 2 * kk, db + 2 * kk, kIdesc,
-                                             (kb | kk) != 0 ? 1u : 0u);
+                            for (int kk = 0; kk < kBK / 16; ++kk) {
+                                // +32 bytes along K per 16-element MMA slice (encoded >> 4).
+                                tc_mma_bf16_pair(d_tmem, da + 2 * kk, db + 2 * kk, kIdesc,
+                                                 (kb | kk) != 0 ? 1u : 0u);
+                            }
                         }
                     }
                     tc_commit_pair_multicast(&empty_bar[stage], kPairMask);
-                    if (++stage == kStages) { stage = 0; phase ^= 1u; }
+                    if (++stage == kRing) { stage = 0; phase ^= 1u; }
                 }
                 if (!ok) break;
                 tc_commit_pair_multicast(&tfull_bar[acc], kPairMask);
@@ -634,11 +651,6 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
             const NsClass& C = P.cls[w.cls];
             const uint32_t acc = gi & 1, acc_phase = (gi >> 1) & 1;
             ++gi;
-            if (!mbar_wait_cluster_bounded(&tfull_bar[acc], acc_phase, budget, abort_flag)) {
-                raise_timeout(P, abort_flag, kSiteAccFull, item, seq);
-                break;
-            }
-            tc_fence_after();
             const int M = C.p, N = w.kind == kBX ? C.q : C.p;
             const CUtensorMap* out_map = item_operands(P, w).out;
             const bool sym = w.kind != kBX;
@@ -683,6 +695,14 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
             uint4 xin[4];
             uint32_t rv[2][32];
             const int row0 = w.mt * kTileM + rank * kBM + quarter * 32;   // warp's first row
+            // The first chunk's A values (and the scalars above) are in flight
+            // while the accumulator is still being computed.
+            if (need_ein && nch > 0) load_ein(0, xin);
+            if (!mbar_wait_cluster_bounded(&tfull_bar[acc], acc_phase, budget, abort_flag)) {
+                raise_timeout(P, abort_flag, kSiteAccFull, item, seq);
+                break;
+            }
+            tc_fence_after();
             if (nch > 0) {
                 tmem_ld_issue(tbase, rv[0]);
                 tmem_ld_wait(rv[0]);
@@ -691,7 +711,10 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
             for (int ch = 0; ch < kEpiChunks; ++ch) {
                 if (ch >= nch) break;
                 const int cur = ch & 1;
-                if (need_ein) load_ein(ch, xin);
+                uint4 xcur[4];
+#pragma unroll
+                for (int q8 = 0; q8 < 4; ++q8) xcur[q8] = xin[q8];
+                if (need_ein && ch + 1 < nch) load_ein(ch + 1, xin);   // next chunk's A, one ahead
                 // Keep the next chunk's TMEM load in flight.
                 if (ch + 1 < nch) tmem_ld_issue(tbase + (ch + 1) * 32, rv[cur ^ 1]);
                 const int col0 = col_base + ch * 32;
@@ -705,7 +728,7 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                 } else if (w.kind == kPoly) {
                     float x[32];
 #pragma unroll
-                    for (int q8 = 0; q8 < 4; ++q8) unpack8(xin[q8], x + 8 * q8);
+                    for (int q8 = 0; q8 < 4; ++q8) unpack8(xcur[q8], x + 8 * q8);
 #pragma unroll
                     for (int j = 0; j < 32; ++j)
                         v[j] = fmaf(P.b, x[j], P.c * v[j]) + (col0 + j == row ? P.a : 0.f);
