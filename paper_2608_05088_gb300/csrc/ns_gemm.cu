@@ -693,7 +693,7 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                 }
             };
             uint4 xin[4];
-            uint32_t rv[2][32];
+            uint32_t rv[32];
             const int row0 = w.mt * kTileM + rank * kBM + quarter * 32;   // warp's first row
             // The first chunk's A values (and the scalars above) are in flight
             // while the accumulator is still being computed.
@@ -704,23 +704,23 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
             }
             tc_fence_after();
             if (nch > 0) {
-                tmem_ld_issue(tbase, rv[0]);
-                tmem_ld_wait(rv[0]);
+                tmem_ld_issue(tbase, rv);
+                tmem_ld_wait(rv);
             }
 #pragma unroll
             for (int ch = 0; ch < kEpiChunks; ++ch) {
                 if (ch >= nch) break;
-                const int cur = ch & 1;
                 uint4 xcur[4];
 #pragma unroll
                 for (int q8 = 0; q8 < 4; ++q8) xcur[q8] = xin[q8];
                 if (need_ein && ch + 1 < nch) load_ein(ch + 1, xin);   // next chunk's A, one ahead
-                // Keep the next chunk's TMEM load in flight.
-                if (ch + 1 < nch) tmem_ld_issue(tbase + (ch + 1) * 32, rv[cur ^ 1]);
+
                 const int col0 = col_base + ch * 32;
                 float v[32];
 #pragma unroll
-                for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(rv[cur][j]);
+                for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(rv[j]);
+                // The next chunk's TMEM load is in flight during this chunk's work.
+                if (ch + 1 < nch) tmem_ld_issue(tbase + (ch + 1) * 32, rv);
                 if (w.kind == kGram) {
                     const float sc = kx * kx;
 #pragma unroll
@@ -801,7 +801,7 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                         sum_d = fmaf(ov, ov, sum_d);
                     }
                 }
-                if (ch + 1 < nch) tmem_ld_wait(rv[cur ^ 1]);
+                if (ch + 1 < nch) tmem_ld_wait(rv);
             }
             tc_fence_before();
             __syncwarp();
