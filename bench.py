@@ -290,6 +290,74 @@ def run_compare_cublas(args):
                       "library_ms": ours_ms, "library_tflops": flops / ours_ms / 1e9}), flush=True)
 
 
+STRESS_SHAPES = ((4096, 4096), (4096, 16384), (16384, 4096))
+
+
+def run_stress_sweep(args):
+    """The shape / anisotropy stress set: one large bf16 matrix with fp32
+    state per case (4096^2, 4096x16384, 16384x4096; row / column scale sigma
+    in {0, 1, 3}; 5 or 8 Newton-Schulz iterations).  Per case, one JSON line:
+    steps/s, the Newton-Schulz products' rate against the measured sustained
+    bf16 peak, and the statistics / prescale / apply kernels' HBM rate
+    against the measured copy bandwidth (device-resident inputs, CUDA events
+    of the library's per-kernel profiling).  Not a bench line."""
+    import torch
+    import paper_2608_05088_gb300.malt as malt
+    from paper_2608_05088_gb300 import build, inputs
+    build.build()
+    dev = torch.device("cuda:0")
+    pk, pk_src = peaks()
+    sigmas = (0.0, 1.0, 3.0) if args.stress_sigma is None else (args.stress_sigma,)
+    ks = (5, 8) if args.stress_k is None else (args.stress_k,)
+    for rows, cols in STRESS_SHAPES:
+        for sigma in sigmas:
+            for k in ks:
+                wl = inputs.stress_workload(rows, cols, sigma, k)
+                W = [torch.from_numpy(w).to(dev).to(torch.bfloat16) for w in inputs.initial_weights(wl)]
+                G = [torch.from_numpy(g).to(dev) for g in inputs.gradients_for_step(wl, 0)]
+                M = [torch.empty(s_, dtype=torch.float32, device=dev) for s_ in wl.shapes]
+                l = [torch.empty(s_[0], dtype=torch.float32, device=dev) for s_ in wl.shapes]
+                r = [torch.empty(s_[1], dtype=torch.float32, device=dev) for s_ in wl.shapes]
+                opt = malt.MaltOptimizer(list(zip(W, G, M, l, r)))
+                hp = malt.hparams(lr=wl.lr, ns_steps=k)
+                for _ in range(args.warmup):
+                    opt.step(hp)
+                torch.cuda.synchronize()
+                opt.profile(True)
+                opt.profile_read()
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record()
+                for _ in range(args.steps):
+                    opt.step(hp)
+                e1.record()
+                torch.cuda.synchronize()
+                prof = opt.profile_read()
+                opt.profile(False)
+                if opt.check() != malt.MALT_OK:
+                    raise SystemExit(f"stress step failed: {wl.name}")
+                t_ms = e0.elapsed_time(e1) / args.steps
+                ns_ms = sum(prof[x][0] for x in malt.NS_KINDS) / args.steps
+                ns_tf = wl.ns_flops_min() / (ns_ms / 1e3) / 1e12
+                elems = wl.elements
+                mem = {}
+                for kind, bpe in (("stats", 12.0), ("prescale", 6.0), ("apply", 6.0)):
+                    ms = prof[kind][0] / args.steps
+                    gbs = bpe * elems / (ms / 1e3) / 1e9
+                    mem[kind] = {"ms": round(ms, 4), "GB/s": round(gbs, 1),
+                                 "frac_of_hbm": round(gbs / float(pk["hbm_gbs"]), 3)}
+                print(json.dumps({
+                    "case": wl.name, "shape": f"{rows}x{cols}", "sigma": sigma, "ns_steps": k,
+                    "steps_per_s": round(1e3 / t_ms, 2), "ms_per_step": round(t_ms, 4),
+                    "ns": {"ms": round(ns_ms, 4), "tflops_symmetric": round(ns_tf, 1),
+                           "frac_of_sustained_bf16": round(ns_tf / float(pk["bf16_tflops_sustained"]), 3),
+                           "schedule": "persistent" if prof["ns_persistent"][1] > 0 else "phased"},
+                    "hbm": mem, "peaks": pk_src}), flush=True)
+                opt.close()
+                del W, G, M, l, r
+                torch.cuda.empty_cache()
+
+
 # --------------------------------------------------------------------- MALT
 def run_malt(args):
     import numpy as np
@@ -526,11 +594,19 @@ def main():
     ap.add_argument("--compare-cublas", action="store_true",
                     help="one B*X-shaped product (36 x 1280^2 @ 1280x5120, bf16) through "
                          "cuBLAS (torch.matmul) and through this library's phased B*X launch")
+    ap.add_argument("--stress-sweep", action="store_true",
+                    help="the shape / anisotropy stress set, one JSON line per case (not a bench line)")
+    ap.add_argument("--stress-sigma", type=float, default=None,
+                    help="stress sweep: only this row / column scale sigma")
+    ap.add_argument("--stress-k", type=int, default=None,
+                    help="stress sweep: only this Newton-Schulz iteration count")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
     if args.compare_cublas:
         run_compare_cublas(args)
+    elif args.stress_sweep:
+        run_stress_sweep(args)
     elif args.impl == "reference":
         run_reference(args)
     else:
