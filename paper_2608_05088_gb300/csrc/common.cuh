@@ -66,7 +66,7 @@ struct MatDesc {
     float* prepart;          // [pre_tiles][2]  sum Mt^2, sum (L G R)^2
     float* nspart;           // [ns_tiles][kNsPartsPerTile][2]: sum O^2, sum D^2
     __nv_bfloat16* X0;       // NS-frame Mt (p x q, bf16): Mt, or Mt^T when trans
-    __nv_bfloat16* O;        // [p][q] orthogonalised direction in the NS frame
+    __nv_bfloat16* O;        // orthogonalised direction in W's layout (m x n)
 };
 
 // Per-matrix scalars kept on the device (index = matrix).
@@ -126,6 +126,7 @@ struct NsClass {  // 64-byte aligned through its CUtensorMap members
     CUtensorMap tmXmn[2];         // the same buffers as an MN-major [K][N] operand (box kBMN x kBK)
     CUtensorMap tmA, tmB;         // A = X X^T and B' = aI + bA + cA^2, K-major rows
     CUtensorMap stX[2], stA, stB, stO;   // epilogue stores: box 32 x 32, 64-byte swizzle
+    CUtensorMap stOt;             // the O buffer as [q][p]: a tall W's O, stored in W's layout
     int32_t p, q, batch;
     int32_t tiles_p, tiles_q;     // 256-wide tiles along p and along q
     int32_t sym_begin;            // first item of this class within a Gram or Poly phase
@@ -202,12 +203,10 @@ __host__ __device__ __forceinline__ void ns_tile_coords(const NsClass& C, int32_
     *nt = r + u;
 }
 
-// Blocks of the apply pass of one matrix: kApplyElems contiguous elements of
-// a wide matrix, 64 x kPreCols of a tall one.
+// Blocks of the apply pass of one matrix: kApplyElems contiguous elements
+// (O is stored in W's layout for every matrix).
 __host__ __device__ __forceinline__ int32_t mat_apply_blocks(const MatDesc& d) {
-    return d.trans ? ((d.m + 63) / 64) * ((d.n + kPreCols - 1) / kPreCols)
-                   : static_cast<int32_t>((static_cast<int64_t>(d.m) * d.n + kApplyElems - 1) /
-                                          kApplyElems);
+    return static_cast<int32_t>((static_cast<int64_t>(d.m) * d.n + kApplyElems - 1) / kApplyElems);
 }
 
 __host__ __device__ __forceinline__ NsWork ns_decode(const NsParams& P, int32_t item) {

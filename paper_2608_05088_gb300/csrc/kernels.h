@@ -30,9 +30,6 @@ cudaError_t launch_apply(const MatDesc* mats, const UserPtrs* ptrs, const MatSca
                          const int32_t* pref, int nmat, int32_t blocks, float decay,
                          cudaStream_t s);
 cudaError_t launch_wait_probe(int32_t* status, uint64_t budget_ns, cudaStream_t s);
-// dst (cols x rows) = src (rows x cols)^T, bf16, rows and cols multiples of 8.
-cudaError_t launch_transpose_bf16(const __nv_bfloat16* src, __nv_bfloat16* dst, int rows, int cols,
-                                  cudaStream_t s);
 
 // Newton-Schulz products over up to kMaxClasses shape classes on grid_pairs
 // CTA pairs (clusters of two).  mode kNsPhased: the items

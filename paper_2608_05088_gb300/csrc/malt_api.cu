@@ -74,9 +74,10 @@ struct ShapeClass {
     __nv_bfloat16* X[2] = {nullptr, nullptr};   // ping-pong NS iterates [batch][p][q]
     __nv_bfloat16* A = nullptr;                  // X X^T        [batch][p][p]
     __nv_bfloat16* B = nullptr;                  // aI + bA + cA^2 [batch][p][p]
-    __nv_bfloat16* O = nullptr;                  // last iterate   [batch][p][q]
+    __nv_bfloat16* O = nullptr;                  // last iterate, per matrix in W's layout:
+                                                 // [p][q] (wide) or [q][p] (tall)
     CUtensorMap tmX[2], tmXmn[2], tmA, tmB;    // 128-row K-major boxes; 64x64 MN boxes
-    CUtensorMap stX[2], stA, stB, stO;         // epilogue store maps
+    CUtensorMap stX[2], stA, stB, stO, stOt;   // epilogue store maps (stOt: O as [q][p])
 };
 
 struct Carver {
@@ -331,6 +332,7 @@ void plan_ns_groups(const std::vector<ShapeClass>& classes, int nmat, std::vecto
             C.stA = S.stA;
             C.stB = S.stB;
             C.stO = S.stO;
+            C.stOt = S.stOt;
             C.p = S.p;
             C.q = S.q;
             C.batch = S.batch;
@@ -591,16 +593,11 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
     for (int j = 0; j < 4; ++j) pref[j].assign(n + 1, 0);
     for (int i = 0; i < n; ++i) {
         const MatDesc& d = st->hmats[i];
-        const int64_t elems = static_cast<int64_t>(d.m) * d.n;
         pref[0][i + 1] = pref[0][i] + d.stat_rb * d.stat_cb;
         pref[1][i + 1] = pref[1][i] + d.m + d.n;
         pref[2][i + 1] = pref[2][i] + d.pre_tr * d.pre_tc;
-        // apply: contiguous runs of kApplyElems, or 64 x kPreCols blocks for a
-        // tall matrix whose O is read transposed from the NS frame
-        const int32_t apply_blocks =
-            d.trans ? ((d.m + 63) / 64) * ((d.n + kPreCols - 1) / kPreCols)
-                    : static_cast<int32_t>((elems + kApplyElems - 1) / kApplyElems);
-        pref[3][i + 1] = pref[3][i] + apply_blocks;
+        // apply: contiguous runs of kApplyElems (O is in W's layout)
+        pref[3][i + 1] = pref[3][i] + mat_apply_blocks(d);
     }
     st->blocks_stats = pref[0][n];
     st->total_fin = pref[1][n];
@@ -622,6 +619,7 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         ok &= encode_store(&C.stA, C.A, C.p, C.p, C.batch);
         ok &= encode_store(&C.stB, C.B, C.p, C.p, C.batch);
         ok &= encode_store(&C.stO, C.O, C.q, C.p, C.batch);
+        ok &= encode_store(&C.stOt, C.O, C.p, C.q, C.batch);
         if (!ok) {
             std::fprintf(stderr, "malt: cuTensorMapEncodeTiled failed for class %d x %d\n", C.p, C.q);
             return MALT_ERR_CUDA;
@@ -1067,14 +1065,10 @@ int malt_debug_direction(malt_state_t* st, int32_t idx, void* out, void* stream)
     if (st == nullptr || idx < 0 || idx >= st->nmat || out == nullptr) return MALT_ERR_INVALID_ARG;
     const MatDesc& d = st->hmats[idx];
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if (d.trans) {
-        // O is kept in the NS frame (n x m) for a tall matrix: transpose on the way out.
-        MALT_CUDA(launch_transpose_bf16(d.O, static_cast<__nv_bfloat16*>(out), d.n, d.m, s),
-                  "transpose_bf16_kernel");
-    } else {
-        MALT_CUDA(cudaMemcpyAsync(out, d.O, static_cast<size_t>(d.m) * d.n * 2,
-                                  cudaMemcpyDeviceToDevice, s), "cudaMemcpyAsync(O)");
-    }
+    // O is stored in W's layout for every matrix (the last B*X epilogue
+    // writes a tall matrix's tiles transposed).
+    MALT_CUDA(cudaMemcpyAsync(out, d.O, static_cast<size_t>(d.m) * d.n * 2,
+                              cudaMemcpyDeviceToDevice, s), "cudaMemcpyAsync(O)");
     return MALT_OK;
 }
 

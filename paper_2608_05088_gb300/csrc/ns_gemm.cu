@@ -17,8 +17,9 @@
 // 1/(||Mt||_F + ns_eps) normalisation is folded into the first iteration's
 // epilogues (A scaled by k^2, X' by k).  The last iteration's epilogue writes O
 // in W's orientation and per-warp partial sums of O^2 and of D^2 with
-// D = L O R (Algorithm 1, D_t line) for the graft; O stays in the NS frame
-// (the apply pass reads a tall matrix's O transposed).
+// D = L O R (Algorithm 1, D_t line) for the graft.  O is stored in W's layout:
+// a tall matrix's tiles go out transposed (the staging used for the mirror
+// of a symmetric tile), so the apply pass streams every matrix the same way.
 //
 // Work split.  A cluster of two CTAs (a CTA pair on two SMs) computes one
 // 256 x 256 output tile per turn: CTA r owns rows [128 r, 128 r + 128) of the
@@ -281,8 +282,7 @@ __device__ __noinline__ void run_memory_stage(const NsParams& P, int mem, int g,
             break;
         default:                                             // kKindApply
             if (bi < mat_apply_blocks(d))
-                blk::apply_block<true>(d, up, bi, __ldcg(&P.scal[g].scale), P.decay, tid,
-                                       reinterpret_cast<float(*)[65]>(scratch), sync);
+                blk::apply_block<true>(d, up, bi, __ldcg(&P.scal[g].scale), P.decay, tid, sync);
             break;
     }
 }
@@ -652,7 +652,7 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
             const uint32_t acc = gi & 1, acc_phase = (gi >> 1) & 1;
             ++gi;
             const int M = C.p, N = w.kind == kBX ? C.q : C.p;
-            const CUtensorMap* out_map = item_operands(P, w).out;
+            const CUtensorMap* out_map0 = item_operands(P, w).out;
             const bool sym = w.kind != kBX;
             const int row = w.mt * kTileM + rank * kBM + quarter * 32 + lane;
             const bool rok = row < M;
@@ -665,6 +665,9 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
             const __nv_bfloat16* ein =
                 need_ein ? C.A + static_cast<size_t>(w.b) * C.p * C.p : nullptr;
             const bool last_bx = (w.kind == kBX) && (w.iter == P.ns_steps - 1);
+            // O of a tall W (NS frame = W^T) goes out transposed, in W's layout.
+            const bool store_t = last_bx && md.trans;
+            const CUtensorMap* out_map = store_t ? &C.stOt : out_map0;
             // NS frame row / column scalings of D = L O R (swapped when transposed).
             const float* uvec = md.trans ? md.R : md.L;
             const float* vvec = md.trans ? md.L : md.R;
@@ -736,7 +739,7 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
 #pragma unroll
                     for (int j = 0; j < 32; ++j) v[j] *= kx;
                 }
-                {
+                if (!store_t) {
                     // Stage the 32 x 32 chunk (row = lane, 64 bytes) with the 64-byte
                     // swizzle the store map expects, then one TMA store writes it
                     // (A, B', the next X, or O in the NS frame on the last iteration).
@@ -755,10 +758,11 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                     }
                     obuf ^= 1;
                 }
-                if (sym && w.nt != w.mt) {
-                    // Mirror an off-diagonal tile of the symmetric product: the
-                    // transposed chunk (box row = column j, 32 rows of this warp)
-                    // goes to rows [col0, col0+32) x columns [row0, row0+32).
+                if (store_t || (sym && w.nt != w.mt)) {
+                    // Mirror an off-diagonal tile of the symmetric product, or
+                    // store a tall matrix's O in W's layout: the transposed chunk
+                    // (box row = column j, 32 rows of this warp) goes to rows
+                    // [col0, col0+32) x columns [row0, row0+32) of the map.
                     // Lane pairs swap one value per column pair so each lane
                     // writes a 32-bit (two-row) word.
                     uint8_t* box = stage_out + (ew * 2 + obuf) * kStoreBoxBytes;

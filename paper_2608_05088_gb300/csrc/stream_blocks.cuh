@@ -527,51 +527,16 @@ __device__ __forceinline__ void apply8(const MatDesc& d, const UserPtrs& up, boo
     }
 }
 
-// Block `local` of the apply pass: kApplyElems contiguous elements of a wide
-// matrix, or rows [64 i, 64 i + 64) x columns [kPreCols j, ...) of a tall one
-// (whose O is stored n x m in the NS frame), read as four 64 x 64 tiles of
-// O^T through shared memory (tile: 64 x 65 floats).  s = the grafted scale.
+// Block `local` of the apply pass: kApplyElems contiguous elements (O is in
+// W's layout).  s = the grafted scale.
 template <bool kL2, class Sync>
 __device__ __forceinline__ void apply_block(const MatDesc& d, const UserPtrs& up, int local,
-                                            float s, float decay, int tid, float (*tile)[65],
-                                            Sync sync) {
+                                            float s, float decay, int tid, Sync sync) {
     constexpr int P = Mut<kL2>::kPath;
     constexpr int PO = kL2 ? kLdL2 : kLdRO;       // O: read-only path unless written in-launch
     const int m = d.m, n = d.n;
     const bool wbf = d.w_bf16 != 0;
-    if (d.trans) {
-        const int tiles_c = (n + kPreCols - 1) / kPreCols;
-        const int i0 = (local / tiles_c) * 64, c0 = (local % tiles_c) * kPreCols;
-        const int t = tid;
-        for (int sub = 0; sub < kPreCols / 64; ++sub) {
-            const int j0 = c0 + sub * 64;
-            if (j0 >= n) break;                           // uniform across the block
-#pragma unroll
-            for (int pass = 0; pass < 2; ++pass) {
-                const int jj = pass * 32 + (t >> 3);      // row of O_ns = column of W
-                const int ii = (t & 7) * 8;               // 8 consecutive rows of W
-                float o[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-                if (j0 + jj < n && i0 + ii < m)
-                    load8<PO>(d.O, true, static_cast<size_t>(j0 + jj) * m + i0 + ii, o);
-#pragma unroll
-                for (int k = 0; k < 8; ++k) tile[ii + k][jj] = o[k];
-            }
-            sync();
-#pragma unroll
-            for (int pass = 0; pass < 2; ++pass) {
-                const int ii = pass * 32 + (t >> 3);      // row of W
-                const int jj = (t & 7) * 8;               // 8 consecutive columns of W
-                if (i0 + ii < m && j0 + jj < n) {
-                    float o[8];
-#pragma unroll
-                    for (int k = 0; k < 8; ++k) o[k] = tile[ii][jj + k];
-                    apply8<P>(d, up, wbf, s, decay, i0 + ii, j0 + jj, o);
-                }
-            }
-            sync();                                       // tile is reused by the next sub-tile
-        }
-        return;
-    }
+    (void)sync;
     const int32_t total = m * n;
     const int32_t e0 = local * kApplyElems;
 #pragma unroll 4

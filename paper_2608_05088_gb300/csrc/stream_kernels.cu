@@ -1,7 +1,7 @@
 // stream_kernels.cu -- standalone launches of the HBM-bound stages of the
 // MALT / MALTER step (stats, finalize, prescale, norms, scalars, apply; the
 // block bodies and their paper references are in stream_blocks.cuh), plus
-// pointer binding, a debug transpose and the bounded-wait probe.
+// pointer binding and the bounded-wait probe.
 //
 // All reductions run in a fixed order (no atomics), so a step is bitwise
 // reproducible.
@@ -93,41 +93,9 @@ __global__ void __launch_bounds__(256)
 apply_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
              const MatScalars* __restrict__ scal, const int32_t* __restrict__ pref, int nmat,
              float decay) {
-    __shared__ float tile[64][65];
     const int g = find_mat(pref, nmat, blockIdx.x);
     blk::apply_block<false>(mats[g], ptrs[g], blockIdx.x - __ldg(pref + g), scal[g].scale, decay,
-                           threadIdx.x, tile, blk::SyncBlock{});
-}
-
-// dst (cols x rows) = src^T through 64 x 64 shared-memory tiles (debug copy of O).
-__global__ void __launch_bounds__(256)
-transpose_bf16_kernel(const __nv_bfloat16* __restrict__ src, __nv_bfloat16* __restrict__ dst,
-                      int rows, int cols) {
-    __shared__ float tile[64][65];
-    const int tiles_c = (cols + 63) / 64;
-    const int r0 = (blockIdx.x / tiles_c) * 64, c0 = (blockIdx.x % tiles_c) * 64;
-    const int t = threadIdx.x;
-#pragma unroll
-    for (int pass = 0; pass < 2; ++pass) {
-        const int rr = pass * 32 + (t >> 3), cc = (t & 7) * 8;
-        float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        if (r0 + rr < rows && c0 + cc < cols)
-            blk::load8<blk::kLdRO>(src, true, static_cast<size_t>(r0 + rr) * cols + c0 + cc, v);
-#pragma unroll
-        for (int k = 0; k < 8; ++k) tile[rr][cc + k] = v[k];
-    }
-    __syncthreads();
-#pragma unroll
-    for (int pass = 0; pass < 2; ++pass) {
-        const int cc = pass * 32 + (t >> 3), rr = (t & 7) * 8;
-        if (c0 + cc < cols && r0 + rr < rows) {
-            float v[8];
-#pragma unroll
-            for (int k = 0; k < 8; ++k) v[k] = tile[rr + k][cc];
-            *reinterpret_cast<uint4*>(dst + static_cast<size_t>(c0 + cc) * rows + r0 + rr) =
-                blk::pack8_bf16(v);
-        }
-    }
+                           threadIdx.x, blk::SyncBlock{});
 }
 
 // ------------------------------------------------------------- wait probe
@@ -195,12 +163,6 @@ cudaError_t launch_apply(const MatDesc* mats, const UserPtrs* ptrs, const MatSca
     return cudaGetLastError();
 }
 
-cudaError_t launch_transpose_bf16(const __nv_bfloat16* src, __nv_bfloat16* dst, int rows, int cols,
-                                  cudaStream_t s) {
-    const int blocks = ((rows + 63) / 64) * ((cols + 63) / 64);
-    transpose_bf16_kernel<<<blocks, 256, 0, s>>>(src, dst, rows, cols);
-    return cudaGetLastError();
-}
 
 cudaError_t launch_wait_probe(int32_t* status, uint64_t budget_ns, cudaStream_t s) {
     wait_probe_kernel<<<1, 32, 0, s>>>(status, budget_ns);

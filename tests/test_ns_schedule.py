@@ -45,9 +45,8 @@ def expected_items(rows, cols, kind):
         return cdiv(cdiv(rows, 64) * cdiv(cols, 256), 2)
     if kind == PRESCALE:
         return cdiv(cdiv(rows, 64) * cdiv(cols, 256), 2)
-    if kind == APPLY:
-        blocks = cdiv(rows, 64) * cdiv(cols, 256) if rows > cols else cdiv(rows * cols, 16384)
-        return cdiv(blocks, 2)
+    if kind == APPLY:                   # 16384-element runs (O is in W's layout)
+        return cdiv(cdiv(rows * cols, 16384), 2)
     return 1
 
 
