@@ -701,7 +701,10 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
             // The first chunk's A values (and the scalars above) are in flight
             // while the accumulator is still being computed.
             if (need_ein && nch > 0) load_ein(0, xin);
-            if (!mbar_wait_cluster_bounded(&tfull_bar[acc], acc_phase, budget, abort_flag)) {
+            // The epilogue warps poll with a short sleep: sixteen warps spinning
+            // on this barrier cost issue slots and power the MMA and load
+            // warps need (measured 0.5-1 % on every product).
+            if (!mbar_wait_cluster_bounded_sleep(&tfull_bar[acc], acc_phase, budget, abort_flag, 128)) {
                 raise_timeout(P, abort_flag, kSiteAccFull, item, seq);
                 break;
             }
