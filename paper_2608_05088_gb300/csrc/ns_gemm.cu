@@ -745,7 +745,7 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                 if (!store_t) {
                     // Stage the 32 x 32 chunk (row = lane, 64 bytes) with the 64-byte
                     // swizzle the store map expects, then one TMA store writes it
-                    // (A, B', the next X, or O in the NS frame on the last iteration).
+                    // (A, B', the next X, or a wide matrix's O on the last iteration).
                     uint8_t* box = stage_out + (ew * 2 + obuf) * kStoreBoxBytes;
                     if (lane == 0) bulk_wait_group_read<1>();   // this buffer's last store read it
                     __syncwarp();

@@ -16,7 +16,8 @@
 //   norms     ||Mt||_F and ||L G R||_F^2 per matrix from those partials.
 //   scalars   ||O||_F, ||D||_F, MALTER's nu and alpha (Section 3.5) and the
 //             grafted scale lr * alpha * ||O|| / (||D|| + eps) per matrix.
-//   apply     W <- (1 - lr wd) W - scale * L O R (Algorithm 1, W_t line).
+//   apply     W <- (1 - lr wd) W - scale * L O R (Algorithm 1, W_t line), with
+//             O in W's layout, streamed contiguously.
 //
 // Template flag kL2: data that an earlier stage of the same launch may have
 // written (M, L, R, the partial sums, the per-matrix scalars, O) is read
