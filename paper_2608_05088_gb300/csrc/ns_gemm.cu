@@ -466,10 +466,18 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                 const NsWork& w = job.w;
                 const Ops op = item_operands(P, w);
                 const bool b_mn = w.kind == kBX;
+                // A diagonal tile of a symmetric product: each CTA's half of B is
+                // its own rows of A, so B is not loaded and the MMA reads A twice.
+                const bool same_ab = !b_mn && w.mt == w.nt;
                 const int nkb = (op.K + kBK - 1) / kBK;
                 int nb_self = 0, nb_peer = 0;
-                const uint32_t bytes_self = slice_bytes(op, w, rank, b_mn, &nb_self);
-                const uint32_t bytes_pair = bytes_self + slice_bytes(op, w, rank ^ 1, b_mn, &nb_peer);
+                uint32_t bytes_pair = slice_bytes(op, w, rank, b_mn, &nb_self) +
+                                      slice_bytes(op, w, rank ^ 1, b_mn, &nb_peer);
+                if (same_ab) {
+                    nb_self = 0;
+                    bytes_pair = (w.mt * kTileM < op.M ? kABytes : 0u) +
+                                 (w.mt * kTileM + kBM < op.M ? kABytes : 0u);
+                }
                 const bool load_a = w.mt * kTileM + rank * kBM < op.M;
                 const int a_row = w.mt * kTileM + rank * kBM;
                 const int n0 = w.nt * kBN + rank * kHalfN;
@@ -572,7 +580,8 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                                                  kIdescBmn, (kb | kk) != 0 ? 1u : 0u);
                             }
                         } else {
-                            const uint64_t db = smem_desc_k_sw128(sa + kABytes);
+                            // (a diagonal tile of a symmetric product reads B from A's rows)
+                            const uint64_t db = smem_desc_k_sw128(w.mt == w.nt ? sa : sa + kABytes);
 #pragma unroll
                             for (int kk = 0; kk < kBK / 16; ++kk) {
                                 // +32 bytes along K per 16-element MMA slice (encoded >> 4).
