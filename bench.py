@@ -537,6 +537,9 @@ def run_malt(args):
                 "flops_per_step": wl.ns_flops_min(),
                 "flops_counted": "3p^2q + p^3 per matrix and NS iteration (symmetric Gram and polynomial)",
                 "dense_equivalent_tflops": dense_equiv,
+                # what the tensor cores execute: symmetric products as whole
+                # 256 x 256 tiles on and above the diagonal
+                "issued_tflops": wl.ns_flops_issued() * args.steps / (ns_ms / 1e3) / 1e12,
                 "launch_avg_ms": ns_ms / max(ns_launches, 1)}
     elems = wl.elements
     wbytes = 2 if wl.weight_dtype == "bf16" else 4

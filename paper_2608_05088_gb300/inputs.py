@@ -53,6 +53,19 @@ class Workload:
             tot += 3.0 * p * p * q + p ** 3
         return tot * self.ns_steps
 
+    def ns_flops_issued(self, tile: int = 256) -> float:
+        """Tensor-core flops the Newton-Schulz products issue in one step with
+        tile x tile output tiles over the padded NS frame: every tile on or
+        above the diagonal of the symmetric Gram and polynomial products (a
+        diagonal tile is computed whole), every tile of B X."""
+        tot = 0.0
+        for m, n in self.shapes:
+            p, q = min(m, n), max(m, n)
+            tp, tq = -(-p // tile), -(-q // tile)
+            sym = tp * (tp + 1) // 2
+            tot += 2.0 * tile * tile * (sym * tq * tile + sym * tp * tile + tp * tq * tp * tile)
+        return tot * self.ns_steps
+
     def ns_flops_dense(self) -> float:
         """Dense Newton-Schulz flops of one step: per matrix and iteration
         4 p^2 q + 2 p^3 with p = min(m, n), q = max(m, n)."""

@@ -57,3 +57,18 @@ def test_reference_arm_nonzero_rank_is_silent():
                           "--workload", "single_256x512", "--steps", "1"],
                          capture_output=True, text=True, timeout=600, cwd=ROOT, env=env)
     assert out.returncode == 0 and out.stdout.strip() == ""
+
+
+def test_issued_flops_accounting():
+    """Tensor-core flops issued per step: whole 256x256 tiles on and above
+    the diagonal of the symmetric products, every tile of B X.  For a 256 x
+    512 frame: Gram 1 tile x K 512, Poly 1 tile x K 256, B X 2 tiles x K 256."""
+    from paper_2608_05088_gb300 import inputs
+    one = inputs.Workload("t", 1, ((256, 512),), "f32", 1.0, 0.02, "malt", 1, ns_steps=1)
+    t = 2.0 * 256 * 256
+    assert one.ns_flops_issued() == t * (512 + 256 + 2 * 256)
+    # with p a multiple of 256 the B X product is exact, the symmetric ones
+    # carry the upper halves of the diagonal tiles on top of the minimum
+    large = inputs.WORKLOADS["gpt2_large"]
+    assert abs(large.ns_flops_issued() - 16.307453952e12) < 1e3
+    assert large.ns_flops_min() < large.ns_flops_issued() < large.ns_flops_dense()
