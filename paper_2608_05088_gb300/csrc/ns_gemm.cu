@@ -27,7 +27,8 @@
 // rows of A and its half (128 N-rows or N-columns) of B, 32 KB, into one of
 // kStages slice slots; the MMA, issued by one thread of the even CTA, reads
 // both CTAs' shared memory.  Each SM therefore pulls 32 KB from L2 per
-// 128 x 256 x 64 of MMA work instead of 48 KB.  The slots are filled,
+// 128 x 256 x 64 of MMA work instead of 48 KB (16 KB on a diagonal tile of
+// a symmetric product, whose B half is the CTA's own A rows).  The slots are filled,
 // awaited and released in groups of kGroup slices (a 3-stage ring of 128-wide
 // reductions): every barrier wait and commit on the MMA thread's path stalls
 // the tensor pipe a little, and one per 8 MMAs measured 4 % faster on B*X
