@@ -452,6 +452,37 @@ def run_malt(args):
                 raise SystemExit(f"{name}-schedule step failed")
         opt.set_ns_schedule(sched_code)
 
+    # ---- the same step replayed from a CUDA graph: one step captured once
+    # (binding kernel, statistics, Newton-Schulz launches, apply), then K
+    # replays.  The device work is the same; the host-side argument
+    # marshalling and the per-launch enqueue cost are gone.
+    graph_leg = None
+    if not args.no_graph:
+        gs = torch.cuda.Stream()
+        gs.wait_stream(stream)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(gs):
+            with torch.cuda.graph(graph, stream=gs):
+                opt.step(hp, malter=malter, stream=gs)
+        torch.cuda.synchronize()
+        for _ in range(2):
+            graph.replay()
+        torch.cuda.synchronize()
+        barrier()
+        g0 = torch.cuda.Event(enable_timing=True)
+        g1 = torch.cuda.Event(enable_timing=True)
+        g0.record(stream)
+        for _ in range(args.steps):
+            graph.replay()
+        g1.record(stream)
+        torch.cuda.synchronize()
+        tg = max_over_ranks(g0.elapsed_time(g1), dev) / args.steps
+        if opt.check() != malt.MALT_OK:
+            raise SystemExit("graph-replayed step failed")
+        graph_leg = {"ms_per_step": tg, "value": world / (tg / 1e3), "unit": UNIT,
+                     "schedule": args.ns_schedule}
+        del graph
+
     # ---- the same engine as Muon (identity preconditioners, no statistics):
     # the optimizer-only counterpart of the paper's MALT-vs-Muon overhead table.
     muon = None
@@ -572,7 +603,7 @@ def run_malt(args):
            "clocks": clk, "e2e": e2e, "gpu_launches": launches, "roofline": roofline,
            "hbm_kernels": mem, "ms_per_step_by_kernel": breakdown,
            "cpu_baseline": cpu, "muon_same_engine": muon, "ns_schedules": sched,
-           "workspace_bytes": opt.workspace_bytes()}
+           "cuda_graph": graph_leg, "workspace_bytes": opt.workspace_bytes()}
     print(json.dumps(out), flush=True)
     opt.close()
 
@@ -587,6 +618,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-muon", action="store_true")
+    ap.add_argument("--no-graph", action="store_true",
+                    help="skip the CUDA-graph replay of the timed step")
     ap.add_argument("--ns-schedule", choices=("auto", "phased", "persistent", "fused"),
                     default="auto",
                     help="schedule of the timed steps (default: the library's auto)")
