@@ -8,9 +8,11 @@
 // stream and without any host synchronisation:
 //   bind (caller pointers) -> stats -> finalize -> prescale -> norms
 //   -> Newton-Schulz -> scalars -> apply,
-// where Newton-Schulz is one persistent launch per group of up to kMaxClasses
-// classes running all k x (Gram, Poly, BX) products (the default), or one
-// launch per product (the phased schedule).
+// where Newton-Schulz runs, per group of up to kMaxClasses classes, either as
+// one persistent launch over all k x (Gram, Poly, BX) products or as one
+// launch per product (the phased schedule); by default a group whose Gram
+// product is shallow (few tile waves) takes the persistent launch and a deep
+// one the phased launches.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
