@@ -358,7 +358,9 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
                     const float4 q = mq[sub & 1][pass];
                     v0 = Li * q.x * R4.x; v1 = Li * q.y * R4.y;
                     v2 = Li * q.z * R4.z; v3 = Li * q.w * R4.w;
-                    s_mt += v0 * v0 + v1 * v1 + v2 * v2 + v3 * v3;
+                    // explicit fused multiply-adds: the same rounding wherever
+                    // this block is compiled (standalone kernel or fused step)
+                    s_mt = fmaf(v3, v3, fmaf(v2, v2, fmaf(v1, v1, fmaf(v0, v0, s_mt))));
                     if (malter) {
                         float gq[4];
                         if (gbf) {
@@ -374,7 +376,7 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
                         }
                         const float a0 = Li * gq[0] * R4.x, a1 = Li * gq[1] * R4.y;
                         const float a2 = Li * gq[2] * R4.z, a3 = Li * gq[3] * R4.w;
-                        s_lgr += a0 * a0 + a1 * a1 + a2 * a2 + a3 * a3;
+                        s_lgr = fmaf(a3, a3, fmaf(a2, a2, fmaf(a1, a1, fmaf(a0, a0, s_lgr))));
                     }
                 }
                 tile[rr][cc + 0] = v0; tile[rr][cc + 1] = v1;
@@ -476,8 +478,11 @@ __device__ __forceinline__ void scalars_matrix(const MatDesc& d, MatScalars* sc,
         if (hp.malter) {
             // Algorithm 2, nu_t line; alpha_t as displayed in Section 3.5.
             const double t = static_cast<double>(*tcount);
-            const double nu = static_cast<double>(hp.mu2) * s.nu +
-                              (1.0 - static_cast<double>(hp.mu2)) * s.lgr_sq;
+            // One explicit fma, so that no compilation of this block
+            // contracts the two products differently (the fused step runs
+            // it inside the GEMM kernel).
+            const double nu = fma(static_cast<double>(hp.mu2), static_cast<double>(s.nu),
+                                  (1.0 - static_cast<double>(hp.mu2)) * s.lgr_sq);
             const double bc = sqrt(1.0 - pow(static_cast<double>(hp.mu2), t)) /
                               (1.0 - pow(static_cast<double>(hp.mu1), t) + hp.eps);
             alpha = bc * s.norm_mt / (sqrt(nu) + hp.eps);

@@ -48,6 +48,22 @@ def test_ragged_mixed_shapes(variant):
     run.close()
 
 
+@pytest.mark.parametrize("seed,variant", [(1, "malt"), (2, "malter"), (3, "malt")])
+def test_seeded_random_shapes(seed, variant):
+    """Ten seeded random shapes (multiples of 8 up to 776: wide, tall and
+    square, every tile edge ragged), fp32 and bf16 weights side by side,
+    2 steps, every matrix checked against the oracle."""
+    shapes = inputs.random_shapes(seed, 10)
+    wl = inputs.Workload(f"random{seed}", 40 + seed, shapes, "f32", 1.5, 0.02, variant, 2)
+    run = Run(wl, w_dtypes=["f32", "bf16"] * 5)
+    for s in range(wl.steps):
+        run.step()
+        assert run.status() == 0
+    for i in range(len(shapes)):
+        run.assert_close(i, f"seed {seed} {variant}")
+    run.close()
+
+
 def test_bf16_gradients_and_k8():
     """bf16 gradients, 8 Newton-Schulz iterations, strong anisotropy (sigma 3)."""
     wl = inputs.Workload("bf16g", 32, ((512, 768), (768, 256)), "bf16", 3.0, 0.02, "malt", 3,

@@ -65,6 +65,13 @@ def test_two_launch_groups_bitwise():
     run_both(wl, 2)
 
 
+@pytest.mark.parametrize("seed", [4, 5])
+def test_seeded_random_shapes_bitwise(seed):
+    shapes = inputs.random_shapes(seed, 10)
+    wl = inputs.Workload(f"schedrand{seed}", 60 + seed, shapes, "f32", 1.5, 0.02, "malter", 2)
+    run_both(wl, 2, w_dtypes=["f32", "bf16"] * 5)
+
+
 def test_gpt2_large_layers_bitwise():
     wl = inputs.first_layers(inputs.WORKLOADS["gpt2_large"], 2)
     run_both(wl, 2)
