@@ -179,9 +179,10 @@ __device__ __forceinline__ void stats_block(const MatDesc& d, const UserPtrs& up
             for (int j = 0; j < 8; ++j) {
                 const float gj = gv[u][j];
                 nm[j] = fmaf(mu1, mv[u][j], om * gj);
-                const float sq = gj * gj;
-                rs += sq;
-                csum[j] += sq;
+                // explicit fused multiply-adds: the same rounding in every
+                // compilation of this block
+                rs = fmaf(gj, gj, rs);
+                csum[j] = fmaf(gj, gj, csum[j]);
             }
             if (ok[u]) {
                 const size_t off = static_cast<size_t>(row0 + rb4 + u) * n + col;

@@ -64,6 +64,20 @@ def test_seeded_random_shapes(seed, variant):
     run.close()
 
 
+@pytest.mark.parametrize("seed", [11, 12])
+def test_seeded_random_large_shapes(seed):
+    """Five seeded random shapes up to 2056 (up to 9 x 9 GEMM tiles, ragged),
+    bf16 weights, one MALTER step, checked in full against the oracle."""
+    shapes = inputs.random_shapes(seed, 5, max_dim=2056)
+    wl = inputs.Workload(f"random{seed}", 40 + seed, shapes, "bf16", 1.5, 0.02, "malter", 1)
+    run = Run(wl)
+    run.step()
+    assert run.status() == 0
+    for i in range(len(shapes)):
+        run.assert_close(i, f"seed {seed}")
+    run.close()
+
+
 def test_bf16_gradients_and_k8():
     """bf16 gradients, 8 Newton-Schulz iterations, strong anisotropy (sigma 3)."""
     wl = inputs.Workload("bf16g", 32, ((512, 768), (768, 256)), "bf16", 3.0, 0.02, "malt", 3,

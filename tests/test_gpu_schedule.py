@@ -23,10 +23,12 @@ SCHEDULES = [(malt.MALT_NS_PHASED, 0), (malt.MALT_NS_PERSISTENT, 0), (malt.MALT_
              (malt.MALT_NS_FUSED, 1), (malt.MALT_NS_FUSED, 3)]
 
 
-def run_both(wl, steps, w_dtypes=None, ns_coeffs=None, schedules=SCHEDULES):
+def run_both(wl, steps, w_dtypes=None, ns_coeffs=None, schedules=SCHEDULES, g_dtype="f32"):
     """The same steps under every schedule: all results bitwise equal."""
     import torch
-    kw = {} if ns_coeffs is None else {"ns_coeffs": ns_coeffs}
+    kw = {"g_dtype": g_dtype}
+    if ns_coeffs is not None:
+        kw["ns_coeffs"] = ns_coeffs
     out = []
     for sched, groups in schedules:
         run = Run(wl, check=[], w_dtypes=w_dtypes, **kw)
@@ -65,11 +67,13 @@ def test_two_launch_groups_bitwise():
     run_both(wl, 2)
 
 
-@pytest.mark.parametrize("seed", [4, 5])
-def test_seeded_random_shapes_bitwise(seed):
+@pytest.mark.parametrize("seed,variant,g_dtype", [(4, "malter", "f32"), (5, "malter", "f32"),
+                                                  (6, "malt", "bf16"), (7, "muon", "f32"),
+                                                  (8, "malter", "bf16")])
+def test_seeded_random_shapes_bitwise(seed, variant, g_dtype):
     shapes = inputs.random_shapes(seed, 10)
-    wl = inputs.Workload(f"schedrand{seed}", 60 + seed, shapes, "f32", 1.5, 0.02, "malter", 2)
-    run_both(wl, 2, w_dtypes=["f32", "bf16"] * 5)
+    wl = inputs.Workload(f"schedrand{seed}", 60 + seed, shapes, "f32", 1.5, 0.02, variant, 3)
+    run_both(wl, 3, w_dtypes=["f32", "bf16"] * 5, g_dtype=g_dtype)
 
 
 def test_gpt2_large_layers_bitwise():
