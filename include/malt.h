@@ -29,7 +29,12 @@
  * as void*; NULL is the legacy default stream) and returns a status code
  * immediately; only malt_check, malt_get_scalars, malt_set_scalars and
  * malt_debug_scalars wait for the stream.  No call allocates memory except
- * malt_init_state.  All device pointers stay owned by the caller.
+ * malt_init_state and the first step with an ns_steps value other than 5 (or,
+ * on the fused schedule, a new overlap-group count): that step builds the
+ * persistent schedule's work table for it once (a small device allocation
+ * and an upload that completes before the call returns), so it cannot be
+ * the first such step inside a stream capture.  Tables for ns_steps = 5 are
+ * built by malt_init_state.  All device pointers stay owned by the caller.
  */
 #ifndef MALT_H
 #define MALT_H

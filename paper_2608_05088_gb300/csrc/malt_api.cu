@@ -21,6 +21,7 @@
 #include <cstdio>
 #include <cstring>
 #include <map>
+#include <tuple>
 #include <utility>
 #include <vector>
 
@@ -132,14 +133,18 @@ struct malt_state {
     int sched_groups_pad = 0;
     int ns_schedule = MALT_NS_AUTO;
     int overlap_groups = 0;                       // fused schedule: 0 = automatic
-    // Work tables of the persistent launches, per launch group: [0] the
-    // Newton-Schulz products only, [1] the fused step.  Built for one
-    // ns_steps value (and overlap-group count) at a time.
+    // Work tables of the persistent launches, one per launch group, for the
+    // Newton-Schulz products only (kind 0) or the fused step (kind 1).  Every
+    // set built is kept, keyed by (kind, ns_steps, overlap groups), until the
+    // state is destroyed: a launch still queued never loses its table, and
+    // returning to an earlier ns_steps value uploads nothing.
     struct Tables {
         int k = -1, groups = -1;
         std::vector<NsEntry*> dev;
         std::vector<int32_t> len;
-    } tables[2];
+    };
+    std::map<std::tuple<int, int, int>, Tables> table_cache;
+    const Tables* tables[2] = {nullptr, nullptr};   // the sets the next launches use
     int32_t last_timeout[5] = {};   // site record of the last timeout malt_check reported
     cudaStream_t last_stream = nullptr;
     // Profiling: event pairs recorded around launches, folded in on read.
@@ -209,8 +214,8 @@ void free_state(malt_state* st) {
         cudaEventDestroy(p.second.second);
     }
     for (cudaEvent_t e : st->ev_pool) cudaEventDestroy(e);
-    for (auto& t : st->tables)
-        for (NsEntry* p : t.dev)
+    for (auto& kv : st->table_cache)
+        for (NsEntry* p : kv.second.dev)
             if (p != nullptr) cudaFree(p);
     if (st->ws != nullptr) cudaFree(st->ws);
     delete st;
@@ -474,17 +479,27 @@ void build_table(const NsParams& G, const std::vector<int>& slot_class,
     stage_list(appl, groups - 1, out);
 }
 
-// Make the state's work tables of one kind (0 products only, 1 fused step)
-// match ns_steps k (host build, device upload; synchronises).
+// Select the state's work tables of one kind (0 products only, 1 fused step)
+// for ns_steps k, building them on first use (host build, device allocation
+// and upload, complete before return; not allowed inside a stream capture).
 int ensure_tables(malt_state* st, int fused, int k) {
-    malt_state::Tables& T = st->tables[fused];
     int groups = 1;
     if (fused) groups = st->overlap_groups > 0 ? st->overlap_groups : -1;
-    if (T.k == k && T.groups == groups && T.dev.size() == st->ns_groups.size()) return MALT_OK;
-    for (NsEntry* p : T.dev)
-        if (p != nullptr) cudaFree(p);
+    const auto key = std::make_tuple(fused, k, groups);
+    const auto hit = st->table_cache.find(key);
+    if (hit != st->table_cache.end()) {
+        st->tables[fused] = &hit->second;
+        return MALT_OK;
+    }
+    malt_state::Tables T;
+    T.k = k;
+    T.groups = groups;
     T.dev.assign(st->ns_groups.size(), nullptr);
     T.len.assign(st->ns_groups.size(), 0);
+    auto release = [&T]() {
+        for (NsEntry* p : T.dev)
+            if (p != nullptr) cudaFree(p);
+    };
     std::vector<NsEntry> host;
     for (size_t gi = 0; gi < st->ns_groups.size(); ++gi) {
         const NsParams& G = st->ns_groups[gi];
@@ -496,15 +511,25 @@ int ensure_tables(malt_state* st, int fused, int k) {
         if (cudaMalloc(&T.dev[gi], bytes) != cudaSuccess) {
             T.dev[gi] = nullptr;
             cudaGetLastError();
-            T.k = -1;
+            release();
             return MALT_ERR_OUT_OF_MEMORY;
         }
-        MALT_CUDA(cudaMemcpy(T.dev[gi], host.data(), sizeof(NsEntry) * host.size(),
-                             cudaMemcpyHostToDevice), "cudaMemcpy(work table)");
+        const int rc = cuda_fail(cudaMemcpy(T.dev[gi], host.data(), sizeof(NsEntry) * host.size(),
+                                            cudaMemcpyHostToDevice), "cudaMemcpy(work table)");
+        if (rc != MALT_OK) {
+            release();
+            return rc;
+        }
         T.len[gi] = static_cast<int32_t>(host.size());
     }
-    T.k = k;
-    T.groups = groups;
+    // A copy from pageable memory may return before its DMA lands; the
+    // tables are read by launches on any stream, so wait for it here.
+    const int rc = cuda_fail(cudaStreamSynchronize(cudaStreamLegacy), "cudaStreamSynchronize(tables)");
+    if (rc != MALT_OK) {
+        release();
+        return rc;
+    }
+    st->tables[fused] = &st->table_cache.emplace(key, std::move(T)).first->second;
     return MALT_OK;
 }
 
@@ -707,8 +732,8 @@ int run_newton_schulz(malt_state* st, const malt_hparams_t* hp, cudaStream_t s) 
             const NsParams& G = st->ns_groups[gi];
             if (!persistent(G)) continue;
             prepare(G);
-            const int items = st->tables[0].len[gi];
-            P.table = st->tables[0].dev[gi];
+            const int items = st->tables[0]->len[gi];
+            P.table = st->tables[0]->dev[gi];
             P.front = 0;
             P.nstages = 3 * k;
             P.item_begin = 0;
@@ -801,11 +826,11 @@ int run_fused_step(malt_state* st, const malt_param_t* params, const malt_hparam
         P.a = hp->ns_a;
         P.b = hp->ns_b;
         P.c = hp->ns_c;
-        P.table = st->tables[1].dev[gi];
+        P.table = st->tables[1]->dev[gi];
         P.front = kFrontStages;
         P.nstages = nstages;
         P.item_begin = 0;
-        P.item_end = st->tables[1].len[gi];
+        P.item_end = st->tables[1]->len[gi];
         P.ptrs = st->d_ptrs;
         P.tcount = st->d_t;
         P.hp = step_hyper(hp, flavour == kMalter ? 1 : 0);

@@ -117,6 +117,27 @@ def test_persistent_against_oracle_two_groups():
     run.close()
 
 
+@pytest.mark.parametrize("schedule", [malt.MALT_NS_PERSISTENT, malt.MALT_NS_FUSED])
+def test_ns_steps_change_between_steps(schedule):
+    """One state stepped with ns_steps 5, 3, 5, 3: the persistent and fused
+    launches take a work table per value (built on first use, then kept), and
+    every step matches the oracle run with the same sequence."""
+    import dataclasses
+    wl = inputs.Workload("kswitch", 39, ((256, 512), (392, 136), (520, 520)), "f32", 1.0, 0.02,
+                         "malter", 4)
+    run = Run(wl, w_dtypes=["f32", "bf16", "f32"])
+    run.opt.set_ns_schedule(schedule)
+    base_ref = run.hp_ref
+    for s, k in enumerate((5, 3, 5, 3)):
+        run.hp_ref = dataclasses.replace(base_ref, ns_steps=k)
+        run.hp = malt.hparams(lr=wl.lr, ns_steps=k)
+        run.step()
+        assert run.status() == malt.MALT_OK, run.opt.timeout_site()
+        for i in range(len(wl.shapes)):
+            run.assert_close(i, f"step {s} k={k}")
+    run.close()
+
+
 def test_unknown_schedule_rejected():
     wl = inputs.Workload("schedbad", 54, ((256, 512),), "f32", 1.0, 0.02, "malt", 1)
     run = Run(wl, check=[])
