@@ -147,7 +147,9 @@ int muon_step(malt_state_t* st, const malt_param_t* params, int32_t n,
  * pinned) for the copies to overlap.  The copies run on two library-owned
  * streams ordered by events against `stream`: the next call's gradient copy
  * waits only until the last step that read the same device G buffers (same
- * params[0].g) has consumed them -- so a caller that alternates two device
+ * params[0].g) has consumed them (for a set other than the last two used, until
+ * the latest step has consumed its gradients, which on one stream follows
+ * every earlier step) -- so a caller that alternates two device
  * gradient sets gets the copy-in of step i+1 fully overlapped with step i,
  * and a caller with one set still overlaps it with step i's Newton-Schulz
  * work -- and this step's weight copy overlaps the next step, whose weight

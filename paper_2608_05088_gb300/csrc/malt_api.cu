@@ -915,15 +915,28 @@ int ensure_pipe(malt_state* st) {
     return MALT_OK;
 }
 
-// Slot of the "G consumed" event for this device gradient buffer set.
-int g_slot(malt_state* st, const void* key) {
+// Slot of the "G consumed" event for this device gradient buffer set, and
+// the copy stream's wait before gradients are copied into the set: for a set
+// among the last two used, the last step that read it; for any other set
+// (new, or last used further back), the latest consumption recorded in either
+// slot, which on one compute stream follows every earlier step's.
+int g_slot_wait(malt_state* st, const void* key, int* slot) {
+    for (int k = 0; k < malt_state::kGSlots; ++k) {
+        if (st->g_key[k] != key) continue;
+        if (st->g_recorded[k])
+            MALT_CUDA(cudaStreamWaitEvent(st->h2d, st->ev_g_consumed[k], 0), "cudaStreamWaitEvent(G)");
+        *slot = k;
+        return MALT_OK;
+    }
     for (int k = 0; k < malt_state::kGSlots; ++k)
-        if (st->g_key[k] == key) return k;
+        if (st->g_recorded[k])
+            MALT_CUDA(cudaStreamWaitEvent(st->h2d, st->ev_g_consumed[k], 0), "cudaStreamWaitEvent(G)");
     const int k = st->g_next_slot;
     st->g_next_slot = (k + 1) % malt_state::kGSlots;
     st->g_key[k] = key;
     st->g_recorded[k] = false;
-    return k;
+    *slot = k;
+    return MALT_OK;
 }
 
 int run_host_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_hparams_t* hp,
@@ -941,11 +954,11 @@ int run_host_step(malt_state* st, const malt_param_t* params, int32_t n, const m
     MALT_CUDA(cudaSetDevice(st->device), "cudaSetDevice");
     rc = ensure_pipe(st);
     if (rc != MALT_OK) return rc;
-    // Gradients in: wait until the last step that read this device G set has
+    // Gradients in: wait until the steps that read this device G set have
     // consumed it.  (A step whose set differs may still be running.)
-    const int slot = g_slot(st, params[0].g);
-    if (st->g_recorded[slot])
-        MALT_CUDA(cudaStreamWaitEvent(st->h2d, st->ev_g_consumed[slot], 0), "cudaStreamWaitEvent(G)");
+    int slot = 0;
+    rc = g_slot_wait(st, params[0].g, &slot);
+    if (rc != MALT_OK) return rc;
     for (int i = 0; i < n; ++i) {
         const size_t bytes = static_cast<size_t>(params[i].rows) * params[i].cols *
                              elem_bytes(params[i].g_dtype);

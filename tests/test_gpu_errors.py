@@ -88,6 +88,37 @@ def test_host_buffer_step_matches_device_step(schedule):
     b.close()
 
 
+def test_host_buffer_steps_run_ahead_over_three_gradient_sets():
+    """Six malt_step_host calls queued without a synchronisation in between,
+    rotating three device gradient sets (each copy-in must wait for the steps
+    that last read its set, also once the set has left the two remembered
+    slots) and one pinned gradient buffer per step: the final W, M, l, r
+    equal six device steps on the same gradients, bitwise."""
+    import numpy as np
+    import torch
+    wl = inputs.Workload("hostrun", 44, ((256, 512), (392, 136), (520, 1544)), "f32", 1.5, 0.02,
+                         "malter", 6)
+    a = Run(wl, check=[])
+    b = Run(wl, check=[])
+    g_host = [[torch.from_numpy(inputs.gradient(wl, i, step)).pin_memory()
+               for i in range(len(wl.shapes))] for step in range(wl.steps)]
+    w_host = [[torch.empty(s, dtype=torch.float32).pin_memory() for s in wl.shapes]
+              for _ in range(wl.steps)]
+    sets = [b.params] + [list(zip(b.W, [torch.empty_like(g) for g in b.G], b.M, b.l, b.r))
+                         for _ in range(2)]
+    for step in range(wl.steps):
+        a.step(oracle=False)
+        b.opt.step_host(b.hp, g_host[step], w_host[step], malter=True, params=sets[step % 3])
+    assert a.status() == malt.MALT_OK and b.opt.check() == malt.MALT_OK
+    for i in range(len(wl.shapes)):
+        assert torch.equal(a.W[i], b.W[i])
+        assert torch.equal(w_host[-1][i], b.W[i].cpu())
+        for x, y in ((a.M[i], b.M[i]), (a.l[i], b.l[i]), (a.r[i], b.r[i])):
+            assert torch.equal(x, y)
+    a.close()
+    b.close()
+
+
 def test_step_replays_from_a_cuda_graph():
     """A step enqueues no host synchronisation and no allocation, so it can
     be captured into a CUDA graph; replays advance the device-side step
