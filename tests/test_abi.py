@@ -77,3 +77,35 @@ def test_host_validation_without_gpu(lib):
     assert lib.malt_debug_wait_timeout(0, None) == malt.MALT_ERR_INVALID_ARG
     assert lib.malt_workspace_bytes(None) == 0
     lib.malt_destroy_state(None)
+
+
+def test_noalloc_host_validation_without_gpu(lib):
+    """malt_stats_noalloc rejects bad arguments, and matrices whose partial
+    sums would not fit its fixed scratch, before it touches the GPU."""
+    F32, BF16 = malt.MALT_F32, malt.MALT_BF16
+
+    def call(g=16, dt=F32, m=16, l=16, r=16, L=16, R=16, rows=64, cols=64,
+             mu1=0.95, mu2=0.99, eps=1e-8):
+        return lib.malt_stats_noalloc(g, dt, m, l, r, L, R, rows, cols, mu1, mu2, eps, None)
+
+    assert call(g=None) == malt.MALT_ERR_INVALID_ARG
+    assert call(R=None) == malt.MALT_ERR_INVALID_ARG
+    assert call(mu1=1.0) == malt.MALT_ERR_INVALID_ARG
+    assert call(mu2=-0.5) == malt.MALT_ERR_INVALID_ARG
+    assert call(eps=float("nan")) == malt.MALT_ERR_INVALID_ARG
+    assert call(dt=5) == malt.MALT_ERR_UNSUPPORTED
+    assert call(rows=0) == malt.MALT_ERR_UNSUPPORTED
+    assert call(cols=12) == malt.MALT_ERR_UNSUPPORTED
+    assert call(rows=65536, cols=32768) == malt.MALT_ERR_UNSUPPORTED
+    assert call(l=24) == malt.MALT_ERR_MISALIGNED
+    assert call(dt=BF16, g=40) == malt.MALT_ERR_MISALIGNED
+    # ceil(n/256)*m (rounded up to 64) + ceil(m/64)*n floats of scratch
+    limit = 1048576
+
+    def need(rows, cols):
+        return -(-(-(-cols // 256) * rows) // 64) * 64 + (-(-rows // 64)) * cols
+
+    assert need(8192, 8192) > limit
+    assert call(rows=8192, cols=8192) == malt.MALT_ERR_UNSUPPORTED
+    assert need(4096, 12800) <= limit < need(4096, 13312)
+    assert call(rows=4096, cols=13312) == malt.MALT_ERR_UNSUPPORTED
