@@ -35,6 +35,14 @@
  * and an upload that completes before the call returns), so it cannot be
  * the first such step inside a stream capture.  Tables for ns_steps = 5 are
  * built by malt_init_state.  All device pointers stay owned by the caller.
+ *
+ * Steps of one state share its workspace (operand buffers, partial sums,
+ * scalars, counters).  Enqueue them on one stream, or order their streams
+ * with events, so that no two steps of the same state run at once on the
+ * GPU; a step switched to another stream with no such ordering races the
+ * previous one.  A state is not thread-safe: calls on one state from several
+ * host threads must be serialised by the caller.  Separate states share
+ * nothing and may run concurrently.
  */
 #ifndef MALT_H
 #define MALT_H
