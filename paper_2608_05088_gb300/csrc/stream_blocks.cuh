@@ -255,7 +255,10 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
                                                float2* red, Sync sync) {
     constexpr int P = Mut<kL2>::kPath;
     const int m = d.m, n = d.n;
-    const int tr = local / d.pre_tc, tc = local - tr * d.pre_tc;
+    // A tall matrix's blocks walk down a column band first, so the blocks
+    // resident at once write neighbouring pieces of the same X0 rows.
+    const int tr = d.trans ? local % d.pre_tr : local / d.pre_tc;
+    const int tc = d.trans ? local / d.pre_tr : local - tr * d.pre_tc;
     const int r0 = tr * kPreRows, c0 = tc * kPreCols;
     const int t = tid, warp = t >> 5, lane = t & 31;
     const float* __restrict__ Lv = d.L;
