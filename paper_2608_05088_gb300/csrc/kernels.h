@@ -40,7 +40,8 @@ cudaError_t launch_wait_probe(int32_t* status, uint64_t budget_ns, cudaStream_t 
 cudaError_t launch_ns_gemm(const NsParams& P, int mode, int grid_pairs, cudaStream_t s);
 size_t ns_gemm_smem_bytes();
 int ns_gemm_max_pairs();
-// Opt the GEMM kernel into its shared memory and cache the resident pair count.
+// Opt the GEMM kernel into its shared memory and count the resident CTA pairs,
+// once per device (on the current device; later calls only look it up).
 cudaError_t ns_gemm_configure();
 
 }  // namespace malt

@@ -71,8 +71,10 @@
 //  bitwise identical.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
+#include <algorithm>
 #include <cstdint>
 #include <cstdio>
+#include <mutex>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -876,39 +878,60 @@ cudaError_t set_all_smem_attrs() {
     return e;
 }
 
+// Per-device one-time set-up: the shared-memory opt-in of every
+// instantiation (a function attribute holds for the device that was current
+// when it was set) and the number of CTA pairs resident at once.  0 = not
+// yet done on that device.
+constexpr int kMaxDevices = 64;
+std::mutex g_cfg_mu;
+int g_pairs[kMaxDevices] = {};
+
+cudaError_t configure_current_device(int* pairs) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(g_cfg_mu);
+    if (g_pairs[dev] == 0) {
+        e = set_all_smem_attrs();
+        if (e != cudaSuccess) return e;
+        // All instantiations have the same block shape and shared memory.
+        int n = 0;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(2, 1, 1);
+        cfg.blockDim = dim3(kThreads, 1, 1);
+        cfg.dynamicSmemBytes = kSmemBytes;
+        if (cudaOccupancyMaxActiveClusters(&n, ns_gemm_kernel<kNsFused>, &cfg) != cudaSuccess ||
+            n <= 0) {
+            cudaGetLastError();
+            int sms = 0;
+            e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+            if (e != cudaSuccess) return e;
+            n = std::max(1, sms / 2);
+        }
+        g_pairs[dev] = n;
+    }
+    *pairs = g_pairs[dev];
+    return cudaSuccess;
+}
+
 }  // namespace
 
-// Number of CTA pairs that can be resident at once (the persistent grid).
-// All instantiations have the same block shape and shared memory.
+// Number of CTA pairs that can be resident at once on the current device (the
+// persistent grid); 1 if the device cannot be configured (the next launch
+// then reports the error).
 int ns_gemm_max_pairs() {
-    static int cached = -1;
-    if (cached > 0) return cached;
-    int n = 0;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(2, 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = kSmemBytes;
-    if (set_all_smem_attrs() != cudaSuccess ||
-        cudaOccupancyMaxActiveClusters(&n, ns_gemm_kernel<kNsFused>, &cfg) != cudaSuccess || n <= 0) {
+    int pairs = 0;
+    if (configure_current_device(&pairs) != cudaSuccess) {
         cudaGetLastError();
-        int dev = 0, sms = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        n = sms / 2;
+        return 1;
     }
-    cached = n;
-    return cached;
+    return pairs;
 }
 
 cudaError_t ns_gemm_configure() {
-    static bool configured = false;
-    if (!configured) {
-        const cudaError_t e = set_all_smem_attrs();
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
-    ns_gemm_max_pairs();
-    return cudaSuccess;
+    int pairs = 0;
+    return configure_current_device(&pairs);
 }
 
 cudaError_t launch_ns_gemm(const NsParams& P, int mode, int grid_pairs, cudaStream_t s) {
