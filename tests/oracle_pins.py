@@ -319,6 +319,33 @@ def check_zero_gradient(ref):
         assert not np.any(info["O"])
 
 
+def check_decoupled_weight_decay(ref):
+    """Weight decay in the decoupled form (reading: W <- (1 - lr wd) W before
+    the update; the algorithms leave it out).  With G = 0 every step the
+    direction is 0, so t steps shrink W geometrically: W_t = (1 - lr wd)^t W_0.
+    With a gradient, the decay changes neither the statistics, the direction
+    nor the graft scale, only W, and it acts on the weights the step starts
+    from, not on the updated ones."""
+    rng = np.random.default_rng(26)
+    W0 = rng.standard_normal((8, 12))
+    hp = ref.Hyper(lr=0.05, weight_decay=0.3)
+    for variant in ("malt", "malter"):
+        st = ref.State.zeros(8, 12)
+        W = W0
+        for _ in range(5):
+            W, _ = ref.malt_step_ref(W, np.zeros((8, 12)), st, hp, variant=variant)
+        assert _rel(W, (1.0 - 0.05 * 0.3) ** 5 * W0) < 1e-14
+    G = rng.standard_normal((8, 12))
+    a, b = ref.State.zeros(8, 12), ref.State.zeros(8, 12)
+    Wa, ia = ref.malt_step_ref(W0, G, a, hp, variant="malter")
+    Wb, ib = ref.malt_step_ref(W0, G, b, ref.Hyper(lr=0.05), variant="malter")
+    for key in ("O", "D", "L", "R"):
+        assert np.array_equal(ia[key], ib[key])
+    assert ia["scale"] == ib["scale"] and a.nu == b.nu
+    # Wb = W0 - delta; the decayed step removes the same delta from the shrunk W0
+    assert _rel(Wa, (1.0 - 0.05 * 0.3) * W0 - (W0 - Wb)) < 1e-13
+
+
 def check_bf16_rounding(ref):
     """Round-to-nearest-even to bf16 against torch's fp32 -> bf16 conversion
     (a library routine), on random values and on exact ties."""
@@ -370,6 +397,7 @@ ALL_CHECKS = [
     check_malter_first_alpha,
     check_malter_pm1_closed_form,
     check_zero_gradient,
+    check_decoupled_weight_decay,
     check_bf16_rounding,
     check_state_memory_matches_paper,
     check_defaults_match_paper,

@@ -29,6 +29,23 @@ MUTATIONS = {
     "bf16_one_bit_short": ("np.maximum(e - 8, -133)", "np.maximum(e - 9, -133)"),
     "t_not_incremented": ("state.t += 1 ", "state.t += 0 "),
     "lr_twice_in_malter": ("scale *= alpha", "scale *= alpha * hp.lr"),
+    "ns_gram_transposed": ("A = X @ X.T", "A = X.T @ X"),
+    "ns_product_order": ("X = a * X + B @ X", "X = a * X + X @ B"),
+    "ns_linear_coeff_dropped": ("X = a * X + B @ X", "X = X + B @ X"),
+    "eps_outside_root": ("np.power(np.asarray(v, dtype=np.float64) + eps, PRECOND_EXPONENT)",
+                         "np.power(np.asarray(v, dtype=np.float64), PRECOND_EXPONENT) + eps"),
+    "ema_weights_swapped": ("return mu * prev + (1.0 - mu) * new",
+                            "return (1.0 - mu) * prev + mu * new"),
+    "two_sided_diagonals_swapped": ("return Ld[:, None] * X * Rd[None, :]",
+                                    "return Ld[None, :] * X * Rd[:, None]"),
+    "alpha_uses_M_not_Mt": ("* norm_Mt / (math.sqrt(state.nu) + hp.eps))",
+                            "* float(np.linalg.norm(state.M)) / (math.sqrt(state.nu) + hp.eps))"),
+    "weight_decay_sign": ("(1.0 - hp.lr * hp.weight_decay) * W if",
+                          "(1.0 + hp.lr * hp.weight_decay) * W if"),
+    "weight_decay_after_update": ("W_new = W_decayed - delta",
+                                  "W_new = (1.0 - hp.lr * hp.weight_decay) * (W - delta)"),
+    "graft_uses_normD_twice": ("scale = hp.lr * norm_O / (norm_D + hp.eps)",
+                               "scale = hp.lr * norm_D / (norm_D + hp.eps)"),
 }
 
 
