@@ -72,32 +72,55 @@ def max_over_ranks(x: float, device=None) -> float:
 
 # -------------------------------------------------------------------- clocks
 class ClockSampler:
-    """nvidia-smi sampled every 200 ms while the timed region runs."""
+    """nvidia-smi sampled every 50 ms around the timed region; the summary
+    keeps the samples whose timestamps fall inside it (begin() .. end()).
+    The sampler starts before the region so that its own start-up does not
+    eat into it.  If no timestamp can be read, every sample counts."""
 
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    INTERVAL_MS = 50
+    STARTUP_S = 0.5
 
     def __init__(self, gpu_index: int):
         self.idx = gpu_index
         self.proc = None
         self.path = None
+        self.t0 = None
+        self.t1 = None
 
     def start(self):
+        """Start sampling (call before the timed region)."""
         try:
             fd, self.path = tempfile.mkstemp(suffix=".csv")
             os.close(fd)
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", str(self.INTERVAL_MS)],
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(self.STARTUP_S)
         except Exception:
             self.proc = None
+
+    def begin(self):
+        self.t0 = time.time()
+
+    def end(self):
+        self.t1 = time.time()
+
+    @staticmethod
+    def _stamp(v):
+        from datetime import datetime
+        try:
+            return datetime.strptime(v.strip(), "%Y/%m/%d %H:%M:%S.%f").timestamp()
+        except ValueError:
+            return None
 
     def stop(self):
         if self.proc is None:
             return None
-        time.sleep(0.25)
+        time.sleep(2.0 * self.INTERVAL_MS / 1e3)      # the sample after end()
         self.proc.terminate()
         try:
             self.proc.wait(timeout=5)
@@ -107,28 +130,49 @@ class ClockSampler:
         with open(self.path) as f:
             for line in f:
                 parts = [p.strip() for p in line.split(",")]
-                if len(parts) >= 9:
+                if len(parts) >= 10:
                     rows.append(parts)
         os.unlink(self.path)
+        try:
+            return self.summarise(rows, self.t0, self.t1)
+        except Exception:
+            return self.summarise(rows, None, None)
+
+    @classmethod
+    def summarise(cls, rows, t0, t1):
+        """Median SM clock, maximum clock and the throttle reasons seen in the
+        samples taken between t0 and t1 (all samples if none is dated)."""
         if not rows:
             return None
+        window = "timed region"
+        inside = rows
+        stamps = [cls._stamp(r[0]) for r in rows]
+        if t0 is not None and t1 is not None and all(t is not None for t in stamps):
+            inside = [r for r, t in zip(rows, stamps) if t0 <= t <= t1]
+            if not inside:     # region shorter than the interval: the sample nearest its middle
+                mid = 0.5 * (t0 + t1)
+                inside = [min(zip(rows, stamps), key=lambda rt: abs(rt[1] - mid))[0]]
+                window = "nearest sample to the timed region"
+        else:
+            window = "all samples (timestamps unreadable)"
 
         def num(v):
             try:
                 return float(v)
             except ValueError:
                 return float("nan")
-        sm = [num(r[1]) for r in rows]
-        mx = max(num(r[2]) for r in rows)
+        sm = [num(r[2]) for r in inside]
+        mx = max(num(r[3]) for r in rows)
         reasons = set()
-        for r in rows:
+        for r in inside:
             for name, v in zip(("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
-                                "sw_power_cap"), r[5:9]):
+                                "sw_power_cap"), r[6:10]):
                 if v.lower().startswith("active"):
                     reasons.add(name)
-        good = [s for s in sm if not math.isnan(s)]
+        good = [x for x in sm if not math.isnan(x)]
         return {"sm_mhz": statistics.median(good) if good else None, "sm_max_mhz": mx,
-                "reasons": sorted(reasons), "samples": len(rows)}
+                "reasons": sorted(reasons), "samples": len(inside), "samples_total": len(rows),
+                "interval_ms": cls.INTERVAL_MS, "window": window}
 
 
 # -------------------------------------------------------------------- peaks
@@ -405,9 +449,10 @@ def run_malt(args):
     opt.profile(True)
     opt.profile_read()
     clocks = ClockSampler(local)
+    clocks.start()
     barrier()
     torch.cuda.synchronize()
-    clocks.start()
+    clocks.begin()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
@@ -415,6 +460,7 @@ def run_malt(args):
         opt.step(hp, malter=malter)
     e1.record(stream)
     torch.cuda.synchronize()
+    clocks.end()
     barrier()
     clk = clocks.stop()
     prof = opt.profile_read()

@@ -72,3 +72,72 @@ def test_issued_flops_accounting():
     large = inputs.WORKLOADS["gpt2_large"]
     assert abs(large.ns_flops_issued() - 16.307453952e12) < 1e3
     assert large.ns_flops_min() < large.ns_flops_issued() < large.ns_flops_dense()
+
+
+
+FAKE_SMI = r'''#!/usr/bin/env python3
+# Stand-in for nvidia-smi's query loop: one timestamped row every 50 ms,
+# 1700 MHz with the power cap active while the flag file exists ("load"),
+# 2070 MHz otherwise.
+import datetime, os, sys, time
+flag = os.environ["FAKE_SMI_FLAG"]
+while True:
+    busy = os.path.exists(flag)
+    stamp = datetime.datetime.now().strftime("%Y/%m/%d %H:%M:%S.%f")[:-3]
+    cap = "Active" if busy else "Not Active"
+    sys.stdout.write(f"{stamp}, 0, {1700 if busy else 2070}, 2070, 900.0, 0x4, Not Active, "
+                     f"Not Active, Not Active, {cap}\n")
+    sys.stdout.flush()
+    time.sleep(0.05)
+'''
+
+
+def _row(t, mhz, cap):
+    import datetime
+    stamp = datetime.datetime.fromtimestamp(t).strftime("%Y/%m/%d %H:%M:%S.%f")[:-3]
+    return [stamp, "0", str(mhz), "2070", "900.0", "0x4", "Not Active", "Not Active",
+            "Not Active", cap]
+
+
+def test_clock_sampler_keeps_the_timed_region(tmp_path, monkeypatch):
+    """Against a fake nvidia-smi: the clocks summary takes the samples dated
+    inside begin() .. end(), not the idle ones before and after it."""
+    import time
+    sys.path.insert(0, ROOT)
+    import bench
+    smi = tmp_path / "nvidia-smi"
+    smi.write_text(FAKE_SMI)
+    smi.chmod(0o755)
+    flag = tmp_path / "busy"
+    monkeypatch.setenv("PATH", f"{tmp_path}{os.pathsep}{os.environ['PATH']}")
+    monkeypatch.setenv("FAKE_SMI_FLAG", str(flag))
+    s = bench.ClockSampler(0)
+    s.start()
+    flag.write_text("")
+    s.begin()
+    time.sleep(0.6)
+    s.end()
+    flag.unlink()
+    out = s.stop()
+    assert out["window"] == "timed region"
+    assert out["sm_mhz"] == 1700 and out["reasons"] == ["sw_power_cap"]
+    assert out["sm_max_mhz"] == 2070
+    assert out["samples"] >= 5 and out["samples_total"] > out["samples"]
+
+
+def test_clock_summary_fallbacks():
+    sys.path.insert(0, ROOT)
+    import bench
+    t0 = 1.0e9
+    rows = ([_row(t0 - 0.3 + 0.05 * i, 2070, "Not Active") for i in range(6)]
+            + [_row(t0 + 0.05 * i, 1700, "Active") for i in range(1, 11)]
+            + [_row(t0 + 0.6 + 0.05 * i, 2070, "Not Active") for i in range(6)])
+    got = bench.ClockSampler.summarise(rows, t0, t0 + 0.55)
+    assert (got["sm_mhz"], got["samples"], got["samples_total"]) == (1700, 10, 22)
+    # a region shorter than the interval: the sample nearest its middle
+    got = bench.ClockSampler.summarise(rows, t0 + 0.101, t0 + 0.109)
+    assert got["samples"] == 1 and got["sm_mhz"] == 1700 and got["window"].startswith("nearest")
+    # undated rows: every sample counts
+    got = bench.ClockSampler.summarise([["n/a"] + r[1:] for r in rows], t0, t0 + 0.55)
+    assert got["samples"] == 22 and got["window"].startswith("all samples")
+    assert bench.ClockSampler.summarise([], t0, t0 + 1) is None
