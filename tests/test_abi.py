@@ -109,3 +109,44 @@ def test_noalloc_host_validation_without_gpu(lib):
     assert call(rows=8192, cols=8192) == malt.MALT_ERR_UNSUPPORTED
     assert need(4096, 12800) <= limit < need(4096, 13312)
     assert call(rows=4096, cols=13312) == malt.MALT_ERR_UNSUPPORTED
+
+
+C_CLIENT = r"""
+#include <stdio.h>
+#include <string.h>
+#include "malt.h"
+int main(void) {
+    malt_state_t* st = 0;
+    malt_param_t p;
+    memset(&p, 0, sizeof p);
+    if (malt_init_state(0, 0, 0, 0) != MALT_ERR_INVALID_ARG) return 1;
+    if (malt_init_state(&st, 0, -1, 0) != MALT_ERR_INVALID_ARG || st) return 2;
+    if (malt_init_state(&st, &p, 1, 0) != MALT_ERR_INVALID_ARG || st) return 3;
+    if (strcmp(malt_status_string(MALT_OK), malt_status_string(MALT_ERR_CUDA)) == 0) return 4;
+    if (malt_workspace_bytes(0) != 0) return 5;
+    malt_destroy_state(0);
+    printf("%s\n", malt_status_string(MALT_ERR_MISALIGNED));
+    return 0;
+}
+"""
+
+
+def test_header_is_plain_c_and_links_from_c(lib, tmp_path):
+    """include/malt.h is a C header (C99, no C++ constructs) and a C program
+    links against libmalt.so and calls it; only calls that fail argument
+    checks before touching a GPU are made."""
+    import shutil
+    if shutil.which("gcc") is None:
+        pytest.skip("gcc not available")
+    inc = os.path.join(ROOT, "include")
+    subprocess.run(["gcc", "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror",
+                    "-fsyntax-only", "-x", "c", os.path.join(inc, "malt.h")], check=True)
+    src = tmp_path / "client.c"
+    src.write_text(C_CLIENT)
+    exe = tmp_path / "client"
+    libdir = os.path.dirname(build.LIB)
+    subprocess.run(["gcc", "-std=c99", "-Wall", "-Werror", f"-I{inc}", str(src), f"-L{libdir}",
+                    "-lmalt", f"-Wl,-rpath,{libdir}", "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True)
+    assert out.returncode == 0, out
+    assert out.stdout.strip() == "device pointer not 16-byte aligned"
