@@ -57,7 +57,8 @@ extern "C" {
 /* ---- status codes ------------------------------------------------------ */
 #define MALT_OK                   0
 #define MALT_ERR_INVALID_ARG     -1  /* null pointer, n < 0, bad hyperparameter */
-#define MALT_ERR_UNSUPPORTED     -2  /* rows or cols not a positive multiple of 8, bad dtype */
+#define MALT_ERR_UNSUPPORTED     -2  /* rows or cols not a positive multiple of 8,
+                                        rows*cols >= 2^31, bad dtype */
 #define MALT_ERR_MISALIGNED      -3  /* a device pointer is not 16-byte aligned */
 #define MALT_ERR_SHAPE_CHANGED   -4  /* step called with shapes/dtypes other than at init */
 #define MALT_ERR_CUDA            -5  /* a CUDA runtime call failed (see malt_status_string) */
@@ -76,7 +77,8 @@ extern "C" {
  *   m       momentum M, rows x cols fp32, updated in place
  *   l, r    row statistics (rows fp32) and column statistics (cols fp32),
  *           updated in place
- * rows and cols must be positive multiples of 8.  W, G and M must not
+ * rows and cols must be positive multiples of 8, with rows*cols < 2^31 (the
+ * kernels index a matrix's elements with 32-bit offsets).  W, G and M must not
  * overlap each other or another parameter's buffers. */
 typedef struct {
     void*        w;
