@@ -204,26 +204,37 @@ def ncu_traffic_per_launch(persistent: bool):
 
 
 # ------------------------------------------------------------ CPU baseline
-def oracle_sample_time(wl, layer_indices, reps_budget_s=10.0):
-    """Seconds for one oracle step over the given matrices (fp64, all cores),
-    averaged over as many repetitions as fit in about reps_budget_s."""
+def oracle_full_step_time(wl, step=0):
+    """Seconds of one oracle step over EVERY matrix of the workload (fp64,
+    numpy's BLAS on all host cores), each matrix from zero state with its
+    gradient of `step`.  Inputs are drawn before each matrix's clock starts;
+    only the malt_step_ref calls are timed.  One matrix is held at a time."""
     import numpy as np
     import oracle.malt_ref as ref
     from paper_2608_05088_gb300 import inputs
-    Ws = [inputs.initial_weight(wl, i).astype(np.float64) for i in layer_indices]
-    Gs = [inputs.gradient(wl, i, 0).astype(np.float64) for i in layer_indices]
     hp = ref.Hyper(lr=wl.lr, ns_steps=wl.ns_steps)
-    times = []
-    t_all = time.perf_counter()
-    while True:
-        sts = [ref.State.zeros(*wl.shapes[i]) for i in layer_indices]
+    total = 0.0
+    for i, shape in enumerate(wl.shapes):
+        W = inputs.initial_weight(wl, i).astype(np.float64)
+        G = inputs.gradient(wl, i, step).astype(np.float64)
+        st = ref.State.zeros(*shape)
         t0 = time.perf_counter()
-        for W, G, st in zip(Ws, Gs, sts):
-            ref.malt_step_ref(W, G, st, hp, variant=wl.variant, weight_dtype=wl.weight_dtype)
-        times.append(time.perf_counter() - t0)
-        if time.perf_counter() - t_all > reps_budget_s:
-            break
-    return statistics.median(times), len(times)
+        ref.malt_step_ref(W, G, st, hp, variant=wl.variant, weight_dtype=wl.weight_dtype)
+        total += time.perf_counter() - t0
+    return total
+
+
+def oracle_warmup(wl, matrices=4):
+    """One untimed oracle step of the first matrices (BLAS threads and pages)."""
+    import numpy as np
+    import oracle.malt_ref as ref
+    from paper_2608_05088_gb300 import inputs
+    hp = ref.Hyper(lr=wl.lr, ns_steps=wl.ns_steps)
+    for i in range(min(matrices, len(wl.shapes))):
+        ref.malt_step_ref(inputs.initial_weight(wl, i).astype(np.float64),
+                          inputs.gradient(wl, i, 0).astype(np.float64),
+                          ref.State.zeros(*wl.shapes[i]), hp, variant=wl.variant,
+                          weight_dtype=wl.weight_dtype)
 
 
 def cpu_cores():
@@ -235,39 +246,26 @@ def cpu_cores():
 
 # ----------------------------------------------------------------- reference
 def run_reference(args):
-    """The fp64 oracle timed on the host cores, one bounded sample per step
-    (the 4 matrices of one GPT-2 layer, scaled to the full 36-layer set)."""
+    """The fp64 oracle timed on the host cores: one warm-up step over one
+    layer's matrices, then ONE timed step over the whole parameter set (about
+    a minute for GPT-2 Large on 16 cores; the requested step count would take
+    many minutes).  The line reports the steps actually timed."""
     rank, world, _ = rank_env()
     if rank != 0:
         return
-    import numpy as np
-    import oracle.malt_ref as ref
     from paper_2608_05088_gb300 import inputs
     wl = inputs.WORKLOADS[args.workload]
-    per_layer = 4 if wl.name.startswith("gpt2") else len(wl.shapes)
-    layers = len(wl.shapes) // per_layer
-    idx = list(range(per_layer))
-    Ws = [inputs.initial_weight(wl, i).astype(np.float64) for i in idx]
-    sts = [ref.State.zeros(*wl.shapes[i]) for i in idx]
-    hp = ref.Hyper(lr=wl.lr, ns_steps=wl.ns_steps)
-    times = []
-    for s in range(args.warmup + args.steps):
-        Gs = [inputs.gradient(wl, i, s).astype(np.float64) for i in idx]
-        t0 = time.perf_counter()
-        for j in range(per_layer):
-            Ws[j], _ = ref.malt_step_ref(Ws[j], Gs[j], sts[j], hp, variant=wl.variant,
-                                         weight_dtype=wl.weight_dtype)
-        if s >= args.warmup:
-            times.append(time.perf_counter() - t0)
-    t_step = sum(times) / len(times) * layers
+    oracle_warmup(wl)
+    t_step = oracle_full_step_time(wl)
     value = 1.0 / t_step
-    sample = (f"one layer ({per_layer} matrices) of {wl.name} per step, scaled x{layers} "
-              f"to the full set")
+    sample = (f"one full step of all {len(wl.shapes)} matrices of {wl.name} (each from zero "
+              f"state), after one warm-up step of 4 matrices")
     out = {"metric": METRIC, "value": value, "unit": UNIT, "impl": "reference",
-           "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+           "n_gpus": world, "steps": 1, "warmup": 1,
+           "requested": {"steps": args.steps, "warmup": args.warmup},
            "ms_per_step": t_step * 1e3, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-           "config": workload_config(wl),
+           "config": dict(workload_config(wl), ns_schedule=args.ns_schedule),
            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(),
                             "kind": "oracle", "sample": sample},
            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
@@ -433,10 +431,8 @@ def run_malt(args):
     malter = wl.variant == "malter"
     stream = torch.cuda.current_stream()
     sched_code = {"auto": malt.MALT_NS_AUTO, "phased": malt.MALT_NS_PHASED,
-                  "persistent": malt.MALT_NS_PERSISTENT,
-                  "fused": malt.MALT_NS_FUSED}[args.ns_schedule]
+                  "persistent": malt.MALT_NS_PERSISTENT}[args.ns_schedule]
     opt.set_ns_schedule(sched_code)
-    opt.set_overlap_groups(args.overlap_groups)
 
     for _ in range(args.warmup):
         opt.step(hp, malter=malter)
@@ -479,8 +475,7 @@ def run_malt(args):
         sched = {"timed": args.ns_schedule + (" (persistent for shallow products, phased for "
                                               "deep ones)" if args.ns_schedule == "auto" else ""),
                  "timed_ms_per_step": t_ms / args.steps}
-        for name, code in (("phased", malt.MALT_NS_PHASED), ("persistent", malt.MALT_NS_PERSISTENT),
-                           ("fused", malt.MALT_NS_FUSED)):
+        for name, code in (("phased", malt.MALT_NS_PHASED), ("persistent", malt.MALT_NS_PERSISTENT)):
             opt.set_ns_schedule(code)
             for _ in range(2):
                 opt.step(hp, malter=malter)
@@ -587,11 +582,8 @@ def run_malt(args):
 
     # ---- roofline of the dominant kernel (the Newton-Schulz GEMMs)
     pk, pk_src = peaks()
-    fused_timed = prof["step_fused"][1] > 0
-    # the fused schedule runs the whole step in its launches: their time is the kernel's
-    ns_kinds = ("step_fused",) if fused_timed else malt.NS_KINDS
-    ns_ms = sum(prof[k][0] for k in ns_kinds)
-    ns_launches = sum(prof[k][1] for k in ns_kinds)
+    ns_ms = sum(prof[k][0] for k in malt.NS_KINDS)
+    ns_launches = sum(prof[k][1] for k in malt.NS_KINDS)
     # Algorithmic work: the Newton-Schulz flops with the symmetry of the Gram
     # matrix and of the polynomial used (3 p^2 q + p^3 per matrix and iteration),
     # which is what the kernels compute (upper-triangle tiles only).
@@ -602,7 +594,7 @@ def run_malt(args):
     persistent_timed = prof["ns_persistent"][1] > 0 and prof["ns_bx"][1] == 0
     # the committed capture is of the 144-matrix GPT-2 Large set only
     traffic = ncu_traffic_per_launch(persistent_timed) if (
-        wl.name == "gpt2_large" and not args.layers and not fused_timed) else None
+        wl.name == "gpt2_large" and not args.layers) else None
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "traffic": traffic,
                 "kernel": ("ns_gemm_kernel, persistent schedule (every Gram, Poly and BX "
@@ -633,13 +625,12 @@ def run_malt(args):
 
     cpu = None
     if not args.no_cpu_baseline and world == 1:
-        per_layer = 4
-        t_layer, reps = oracle_sample_time(wl, list(range(per_layer)))
-        layers = len(wl.shapes) // per_layer
-        cpu = {"value": 1.0 / (t_layer * layers), "unit": UNIT, "cores": cpu_cores(),
-               "kind": "oracle",
-               "sample": f"one MALT step of layer 0 ({per_layer} matrices) in fp64, "
-                         f"median of {reps}, scaled x{layers} to the full set"}
+        oracle_warmup(wl)
+        t_cpu = oracle_full_step_time(wl)
+        cpu = {"value": 1.0 / t_cpu, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+               "ms_per_step": t_cpu * 1e3,
+               "sample": f"one fp64 step of all {len(wl.shapes)} matrices of {wl.name} "
+                         f"(each from zero state), timed once, no scaling"}
 
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_ms / args.steps,
@@ -666,11 +657,9 @@ def main():
     ap.add_argument("--no-muon", action="store_true")
     ap.add_argument("--no-graph", action="store_true",
                     help="skip the CUDA-graph replay of the timed step")
-    ap.add_argument("--ns-schedule", choices=("auto", "phased", "persistent", "fused"),
+    ap.add_argument("--ns-schedule", choices=("auto", "phased", "persistent"),
                     default="auto",
                     help="schedule of the timed steps (default: the library's auto)")
-    ap.add_argument("--overlap-groups", type=int, default=0,
-                    help="fused schedule: runs of matrices overlapped (0: automatic)")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling only: the first N layers of the workload")
     ap.add_argument("--compare-cublas", action="store_true",

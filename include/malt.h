@@ -27,14 +27,13 @@
  *
  * Every call is asynchronous on the given CUDA stream (a cudaStream_t passed
  * as void*; NULL is the legacy default stream) and returns a status code
- * immediately; only malt_check, malt_get_scalars, malt_set_scalars and
- * malt_debug_scalars wait for the stream.  No call allocates memory except
- * malt_init_state and the first step with an ns_steps value other than 5 (or,
- * on the fused schedule, a new overlap-group count): that step builds the
- * persistent schedule's work table for it once (a small device allocation
- * and an upload that completes before the call returns), so it cannot be
- * the first such step inside a stream capture.  Tables for ns_steps = 5 are
- * built by malt_init_state.  All device pointers stay owned by the caller.
+ * immediately; only malt_check, malt_get_scalars, malt_set_scalars,
+ * malt_debug_scalars, malt_profile_read and malt_debug_wait_timeout wait for
+ * the stream.  Only malt_init_state allocates device memory (the workspace,
+ * with the persistent schedule's work table for every ns_steps value);
+ * malt_debug_wait_timeout allocates one word for its probe, and the first
+ * malt_step_host call on a state creates its two copy streams and their
+ * events.  All device pointers passed in stay owned by the caller.
  *
  * Steps of one state share its workspace (operand buffers, partial sums,
  * scalars, counters).  Enqueue them on one stream, or order their streams
@@ -188,11 +187,17 @@ int malt_check(malt_state_t* st);
  * malt_debug_direction: enqueue on `stream` a copy of the last step's
  *   orthogonalised direction O of parameter idx (rows x cols, bf16,
  *   row-major, same orientation as W) into the device buffer out.
+ * malt_debug_precond: enqueue on `stream` copies of the last step's diagonal
+ *   preconditioners of parameter idx, L = (l + eps)^(-1/8) (rows floats) and
+ *   R = (r + eps)^(-1/8) (cols floats), as the step computed and used them
+ *   (Algorithm 1, L_t / R_t line), into the device buffers L_out and R_out
+ *   (fp32, caller-owned).  Muon steps leave L = R = 1.
  * malt_debug_scalars: synchronise, then write 8 floats per parameter to host
  *   memory: ||O||_F, ||D||_F, ||Mt||_F, ||L G R||_F^2 (MALTER steps, else 0),
  *   nu, alpha (1 on MALT steps), the applied scale lr*alpha*||O||/(||D||+eps),
  *   and 1/(||Mt||_F + ns_eps). */
 int malt_debug_direction(malt_state_t* st, int32_t idx, void* out, void* stream);
+int malt_debug_precond(malt_state_t* st, int32_t idx, float* L_out, float* R_out, void* stream);
 /* malt_debug_timeout_site: where the first device-side wait gave up in the
  *   work that the last MALT_ERR_TIMEOUT from malt_check covered, 5 int32 to
  *   out5 (host memory): site code (1 claim a ring slot, 2 producer waits for
@@ -227,8 +232,7 @@ int malt_debug_wait_timeout(int64_t budget_ns, void* stream);
 #define MALT_KIND_SCALARS   8
 #define MALT_KIND_APPLY     9
 #define MALT_KIND_NS_PERSISTENT 10   /* all Newton-Schulz products, persistent schedule */
-#define MALT_KIND_STEP_FUSED 11      /* the whole step in one launch, fused schedule */
-#define MALT_NUM_KINDS     12
+#define MALT_NUM_KINDS     11
 int malt_profile_enable(malt_state_t* st, int32_t enable);
 int malt_profile_read(malt_state_t* st, double* ms_out, int64_t* launches_out, int32_t nkinds);
 
@@ -244,59 +248,42 @@ int malt_profile_read(malt_state_t* st, double* ms_out, int64_t* launches_out, i
  *     device (bounded) only until the previous product of matrix j is stored,
  *     so one matrix's next product overlaps another matrix's current one and
  *     there is no launch gap or wave tail between products.
- *   MALT_NS_FUSED: the whole step in one persistent launch per class group.
- *     The HBM-bound stages run on the GEMM kernel's epilogue warps between
- *     tiles, chained per matrix by the same device counters; the matrices
- *     are split into consecutive runs (malt_set_overlap_groups) so that one
- *     run's statistics / prescale and another run's apply overlap a third
- *     run's tensor-core products.
  *   MALT_NS_AUTO (default): per class group, persistent when a Gram product
  *     has fewer tiles than 16 waves of the resident CTA pairs, phased otherwise.
- * All compute every tile and element with the same arithmetic: results are
- * bitwise identical.  Takes effect at the next step.  The persistent and
- * fused schedules use a work table per ns_steps value, built on the host and
- * uploaded by the first step that needs it (a synchronising copy: for a
- * stream capture, take one eager step with the same ns_steps first; the
- * table for ns_steps = 5 is built at init).  MALT_ERR_INVALID_ARG for a null
- * state or an unknown schedule. */
+ * Both compute every tile with the same arithmetic: results are bitwise
+ * identical.  Takes effect at the next step.  The persistent launches claim
+ * from a work table that malt_init_state builds once for up to 64 iterations,
+ * so no step uploads anything.  MALT_ERR_INVALID_ARG for a null state or an
+ * unknown schedule. */
 #define MALT_NS_PHASED     0
 #define MALT_NS_PERSISTENT 1
 #define MALT_NS_AUTO       2
-#define MALT_NS_FUSED      3
 int malt_set_ns_schedule(malt_state_t* st, int32_t schedule);
 
-/* Fused schedule: the number of consecutive runs the matrices are split into
- * (1..64; 0 = automatic, min(4, matrices / 8)).  More runs hide more of the
- * HBM-bound stages behind the products but make each run's products
- * shallower.  Takes effect at the next step (rebuilding the work table).
- * MALT_ERR_INVALID_ARG for a null state or a count outside 0..64. */
-int malt_set_overlap_groups(malt_state_t* st, int32_t groups);
-
-/* Host only (no GPU, no CUDA call): the work table of the persistent
- * (fused = 0) or fused (fused = 1) schedule for these parameter shapes (only
- * rows and cols are read), ns_steps iterations and overlap_groups runs (0 =
- * automatic), in claim order, 8 int32 per item: launch group, stage, stage
- * kind (0 Gram, 1 Poly, 2 B*X, 3 statistics, 4 finalize, 5 prescale,
- * 6 norms, 7 scalars, 8 apply), matrix index, local index (the tile of the
- * product, 256 x 256 tiles of the NS frame with Gram and Poly listing the
- * upper triangle only; the block pair or 0 for a memory stage), the index of
- * the counter the item waits for ((stage - 1) * n + matrix, or -1), the count
- * that counter must reach (16 signals per item of the previous stage), and
- * the number of items of (stage, matrix).  Writes min(capacity, total) items
- * to out (capacity * 8 int32, caller-owned) and the total to *count; call
- * with capacity 0 to size out.  MALT_ERR_INVALID_ARG for bad arguments or
- * ns_steps outside [1, 64], MALT_ERR_UNSUPPORTED for a shape
- * malt_init_state would reject. */
-int malt_ns_schedule(const malt_param_t* params, int32_t n, int32_t ns_steps, int32_t fused,
-                     int32_t overlap_groups, int32_t* out, int64_t capacity, int64_t* count);
+/* Host only (no GPU, no CUDA call): the work table of the persistent schedule
+ * for these parameter shapes (only rows and cols are read) and ns_steps
+ * iterations, in claim order, 8 int32 per item: launch group, stage (3 i +
+ * kind for iteration i), kind (0 Gram, 1 Poly, 2 B*X), matrix index, local
+ * index (the 256 x 256 tile of the NS frame; Gram and Poly list the upper
+ * triangle only), the index of the counter the item waits for
+ * ((stage - 1) * n + matrix, or -1), the count that counter must reach (16
+ * signals per tile of the previous product), and the number of tiles of
+ * (stage, matrix).  Writes min(capacity, total) items to out (capacity * 8
+ * int32, caller-owned) and the total to *count; call with capacity 0 to size
+ * out.  MALT_ERR_INVALID_ARG for bad arguments or ns_steps outside [1, 64],
+ * MALT_ERR_UNSUPPORTED for a shape malt_init_state would reject. */
+int malt_ns_schedule(const malt_param_t* params, int32_t n, int32_t ns_steps, int32_t* out,
+                     int64_t capacity, int64_t* count);
 
 /* Statistics stage of ONE matrix without any device allocation.
  * The paper has no counterpart: this exists for callers that cannot allocate
- * device memory when they need the work done -- code inside a CUDA stream
- * capture, code that must not trigger the device synchronisation an
- * allocation may cause, code whose framework allocator owns all device
- * memory.  It runs the momentum and statistics updates and writes the two
- * diagonal preconditioners, exactly as a MALT step does for that matrix:
+ * device memory when they need the work done -- code under a framework
+ * allocator that owns all device memory, code in a latency-critical loop that
+ * must not risk the device synchronisation an allocation may cause, services
+ * that reserve all their memory at start-up.  It runs the momentum and
+ * statistics updates and writes the two diagonal preconditioners with the
+ * same kernels' arithmetic as a MALT step for that matrix (bitwise the same
+ * m, l, r, and L, R as malt_debug_precond returns):
  *   m <- mu1 m + (1 - mu1) g;  l, r <- EMAs of the row / column sums of g^2;
  *   L_out = (l + eps)^(-1/8) (rows floats), R_out = (r + eps)^(-1/8) (cols floats).
  * All pointers are caller-owned device buffers laid out as in malt_param_t

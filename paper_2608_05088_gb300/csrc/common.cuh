@@ -88,28 +88,22 @@ struct StepHyper {
 enum GemmPhase : int32_t { kGram = 0, kPoly = 1, kBX = 2 };
 
 // Launch modes of the Newton-Schulz kernel: one product with a static tile
-// split; a persistent work table of products; a persistent work table of
-// the whole step (products and the HBM-bound stages around them).
-enum NsMode : int32_t { kNsPhased = 0, kNsPersistent = 1, kNsFused = 2 };
+// split, or a persistent work table of all products of the k iterations.
+enum NsMode : int32_t { kNsPhased = 0, kNsPersistent = 1 };
 
 // Epilogue warps of a CTA pair; each one signals a finished item once.
 constexpr uint32_t kNsSignalsPerTile = 2 * kEpiWarpsPerCta;
 
-// Stage kinds of a persistent work table.  The products of Newton-Schulz
-// iteration i are stages front + 3 i + {kGram, kPoly, kBX}; a fused step puts
-// the HBM-bound stages around them (kFrontStages before, kBackStages after).
-enum StageKind : int32_t {
-    kKindStats = 3, kKindFinalize = 4, kKindPrescale = 5, kKindNorms = 6,
-    kKindScalars = 7, kKindApply = 8
-};
-constexpr int kFrontStages = 4;   // stats, finalize, prescale, norms
-constexpr int kBackStages = 2;    // scalars, apply
+// Stages of a persistent work table: the products of Newton-Schulz
+// iteration i are stages 3 i + {kGram, kPoly, kBX}.  The table of k
+// iterations is the first k iterations' entries of any longer table.
+constexpr int kMaxNsSteps = 64;
 
 // One item of a persistent work table.
 struct __align__(16) NsEntry {
     int32_t code;     // stage (bits 0-11) | class slot (bits 12-15) | batch slot (bits 16-31)
     int32_t g;        // matrix; -1 marks the end of the table
-    int32_t local;    // tile of the product, block pair of a memory stage, 0 otherwise
+    int32_t local;    // tile of the product
     uint32_t target;  // signals the previous stage of matrix g must reach (0: none)
 };
 
@@ -158,15 +152,7 @@ struct NsParams {
     uint64_t budget_ns;
     // Persistent launches: the work table (item_end entries) and its stages.
     const NsEntry* table;
-    int32_t front;                // memory stages before the products (0 or kFrontStages)
-    int32_t nstages;              // front + 3 ns_steps (+ kBackStages when fused)
-    // Fused step: what the memory stages need.
-    const UserPtrs* ptrs;
-    const long long* tcount;
-    StepHyper hp;
-    float decay;                  // 1 - lr * weight_decay
-    int32_t with_stats;           // 0 for Muon through the same engine (momentum only)
-    int32_t identity;             // 1 for Muon: L = R = 1
+    int32_t nstages;              // 3 ns_steps
 };
 static_assert(sizeof(NsParams) <= 32764, "NsParams is passed by value as the kernel parameter");
 

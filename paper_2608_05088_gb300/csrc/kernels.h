@@ -11,7 +11,6 @@ struct BindParams {
     UserPtrs p[kBindChunk];
     int32_t count;
     int32_t offset;
-    long long* tcount;   // when set, the launch also adds 1 to the step counter
 };
 
 cudaError_t launch_bind(const BindParams& P, UserPtrs* table, cudaStream_t s);
@@ -34,9 +33,9 @@ cudaError_t launch_wait_probe(int32_t* status, uint64_t budget_ns, cudaStream_t 
 // Newton-Schulz products over up to kMaxClasses shape classes on grid_pairs
 // CTA pairs (clusters of two).  mode kNsPhased: the items
 // [P.item_begin, P.item_end) of one product, static round-robin.
-// kNsPersistent / kNsFused: the work table P.table, claimed dynamically, each
-// item waiting for its matrix's previous stage (P.queue and P.done zeroed
-// before the launch); kNsFused tables also hold the HBM-bound stages.
+// kNsPersistent: the work table P.table, claimed dynamically, each item
+// waiting for its matrix's previous product (P.queue and P.done zeroed before
+// the launch).
 cudaError_t launch_ns_gemm(const NsParams& P, int mode, int grid_pairs, cudaStream_t s);
 size_t ns_gemm_smem_bytes();
 int ns_gemm_max_pairs();

@@ -21,7 +21,6 @@
 #include <cstdio>
 #include <cstring>
 #include <map>
-#include <tuple>
 #include <utility>
 #include <vector>
 
@@ -132,19 +131,11 @@ struct malt_state {
     uint32_t* d_sched = nullptr;
     int sched_groups_pad = 0;
     int ns_schedule = MALT_NS_AUTO;
-    int overlap_groups = 0;                       // fused schedule: 0 = automatic
-    // Work tables of the persistent launches, one per launch group, for the
-    // Newton-Schulz products only (kind 0) or the fused step (kind 1).  Every
-    // set built is kept, keyed by (kind, ns_steps, overlap groups), until the
-    // state is destroyed: a launch still queued never loses its table, and
-    // returning to an earlier ns_steps value uploads nothing.
-    struct Tables {
-        int k = -1, groups = -1;
-        std::vector<NsEntry*> dev;
-        std::vector<int32_t> len;
-    };
-    std::map<std::tuple<int, int, int>, Tables> table_cache;
-    const Tables* tables[2] = {nullptr, nullptr};   // the sets the next launches use
+    // Work table of the persistent launches, one per launch group, for
+    // kMaxNsSteps iterations (in the workspace, uploaded at init); a launch of
+    // k iterations claims its first k * table_per_iter[group] entries.
+    std::vector<NsEntry*> table_dev;
+    std::vector<int32_t> table_per_iter;
     int32_t last_timeout[5] = {};   // site record of the last timeout malt_check reported
     cudaStream_t last_stream = nullptr;
     // Profiling: event pairs recorded around launches, folded in on read.
@@ -214,9 +205,6 @@ void free_state(malt_state* st) {
         cudaEventDestroy(p.second.second);
     }
     for (cudaEvent_t e : st->ev_pool) cudaEventDestroy(e);
-    for (auto& kv : st->table_cache)
-        for (NsEntry* p : kv.second.dev)
-            if (p != nullptr) cudaFree(p);
     if (st->ws != nullptr) cudaFree(st->ws);
     delete st;
 }
@@ -256,8 +244,7 @@ struct LaunchScope {
     }
 };
 
-constexpr int kMaxNsSteps = 64;
-constexpr int kMaxStages = kFrontStages + 3 * kMaxNsSteps + kBackStages;
+constexpr int kMaxStages = 3 * kMaxNsSteps;
 // Auto schedule: persistent when a symmetric product has fewer tiles than
 // this many waves of the resident CTA pairs.
 constexpr int kAutoPersistentWaves = 16;
@@ -360,178 +347,40 @@ void plan_ns_groups(const std::vector<ShapeClass>& classes, int nmat, std::vecto
 }
 
 // ------------------------------------------------------------- work tables
-// Stage s of a persistent table: kFrontStages memory stages (fused only),
-// then 3 k products, then kBackStages memory stages (fused only).
-int stage_kind(int s, int front, int k) {
-    if (s < front) return kKindStats + s;
-    if (s >= front + 3 * k) return kKindScalars + (s - front - 3 * k);
-    return (s - front) % 3;                       // kGram, kPoly, kBX
-}
+// Tiles of one matrix in one product of this kind.
+int32_t stage_items(int kind, const NsClass& C) { return ns_phase_tiles(C, kind); }
 
-// Items of one matrix in a stage of this kind (memory stages: one CTA pair
-// runs two blocks per item).
-int32_t stage_items(int kind, const MatDesc& d, const NsClass& C) {
-    switch (kind) {
-        case kGram:
-        case kPoly:
-        case kBX: return ns_phase_tiles(C, kind);
-        case kKindStats: return (d.stat_rb * d.stat_cb + 1) / 2;
-        case kKindPrescale: return (d.pre_tr * d.pre_tc + 1) / 2;
-        case kKindApply: return (mat_apply_blocks(d) + 1) / 2;
-        default: return 1;                        // finalize, norms, scalars
-    }
-}
-
-// Automatic number of overlap groups of a fused launch over nmat matrices.
-int auto_overlap_groups(int nmat) { return std::max(1, std::min(4, nmat / 8)); }
-
-// The work table of one launch group.
-//  * Products only (fused = false): for each product of each iteration, every
-//    tile of every class (slot order), batch slot by batch slot.
-//  * Fused step: the matrices split into `groups` consecutive runs (in
-//    parameter order).  Run 0's memory front stages go first; then the
-//    products of run j, with the front stages of run j+1 and the back stages
-//    of run j-1 spread evenly among them, so HBM-bound work overlaps the
-//    tensor-bound products; run groups-1's back stages close the table.
-// Every item's dependency is the previous stage of its own matrix, and
-// every stage of a matrix is listed after its previous stage: claiming in
-// table order never waits on an item that has not been claimed.
+// The work table of one launch group for k iterations: for each product of
+// each iteration, every tile of every class (slot order), batch slot by
+// batch slot.  Every item depends on the previous product of its own matrix,
+// listed earlier: claiming in table order never waits on an item that has
+// not been claimed.  The table of k iterations is the prefix of any longer
+// one (an iteration adds entries at the end and changes none before it).
 void build_table(const NsParams& G, const std::vector<int>& slot_class,
-                 const std::vector<ShapeClass>& classes, const std::vector<MatDesc>& hmats, int k,
-                 bool fused, int groups, std::vector<NsEntry>& out) {
+                 const std::vector<ShapeClass>& classes, int k, std::vector<NsEntry>& out) {
     out.clear();
-    const int front = fused ? kFrontStages : 0;
-    // matrices of this launch with their slot and batch index
-    std::vector<int> mats;
-    std::vector<int> slot_of(hmats.size(), -1), b_of(hmats.size(), -1);
-    for (int c = 0; c < G.nclasses; ++c) {
-        const ShapeClass& S = classes[slot_class[c]];
-        for (int b = 0; b < S.batch; ++b) {
-            slot_of[S.mats[b]] = c;
-            b_of[S.mats[b]] = b;
-            mats.push_back(S.mats[b]);
-        }
-    }
-    std::sort(mats.begin(), mats.end());
-    const int nm = static_cast<int>(mats.size());
-    if (!fused) groups = 1;
-    groups = std::max(1, std::min(groups, nm));
-    std::vector<int> run_of(hmats.size(), 0);
-    for (int i = 0; i < nm; ++i) run_of[mats[i]] = static_cast<int>((static_cast<int64_t>(i) * groups) / nm);
-
-    auto items = [&](int st, int g) {
-        return stage_items(stage_kind(st, front, k), hmats[g], G.cls[slot_of[g]]);
-    };
-    auto entry = [&](int st, int g, int local) {
-        NsEntry e;
-        e.code = st | (slot_of[g] << 12) | (b_of[g] << 16);
-        e.g = g;
-        e.local = local;
-        e.target = st == 0 ? 0u : kNsSignalsPerTile * static_cast<uint32_t>(items(st - 1, g));
-        return e;
-    };
-    // items of stage st for the matrices of run j (all runs when j < 0)
-    auto stage_list = [&](int st, int j, std::vector<NsEntry>& v) {
-        const int kind = stage_kind(st, front, k);
-        if (kind <= kBX) {
-            for (int c = 0; c < G.nclasses; ++c) {
-                const ShapeClass& S = classes[slot_class[c]];
-                for (int b = 0; b < S.batch; ++b) {
-                    const int g = S.mats[b];
-                    if (j >= 0 && run_of[g] != j) continue;
-                    for (int t = 0; t < items(st, g); ++t) v.push_back(entry(st, g, t));
+    for (int st = 0; st < 3 * k; ++st) {
+        const int kind = st % 3;
+        for (int c = 0; c < G.nclasses; ++c) {
+            const ShapeClass& S = classes[slot_class[c]];
+            const int32_t items = stage_items(kind, G.cls[c]);
+            const int32_t prev = st == 0 ? 0 : stage_items((st - 1) % 3, G.cls[c]);
+            for (int b = 0; b < S.batch; ++b) {
+                for (int t = 0; t < items; ++t) {
+                    NsEntry e;
+                    e.code = st | (c << 12) | (b << 16);
+                    e.g = S.mats[b];
+                    e.local = t;
+                    e.target = kNsSignalsPerTile * static_cast<uint32_t>(prev);
+                    out.push_back(e);
                 }
             }
-        } else {
-            for (int g : mats) {
-                if (j >= 0 && run_of[g] != j) continue;
-                for (int t = 0; t < items(st, g); ++t) v.push_back(entry(st, g, t));
-            }
         }
-    };
-    const int nprod = 3 * k;
-    if (!fused) {
-        for (int st = 0; st < nprod; ++st) stage_list(st, -1, out);
-        return;
     }
-    const int scal = front + nprod, appl = scal + 1;
-    for (int st = 0; st < front; ++st) stage_list(st, 0, out);
-    for (int j = 0; j < groups; ++j) {
-        std::vector<NsEntry> prod, bg;
-        for (int st = front; st < front + nprod; ++st) stage_list(st, j, prod);
-        if (j + 1 < groups) stage_list(0, j + 1, bg);          // stats of the next run
-        if (j >= 1) {
-            stage_list(scal, j - 1, bg);                       // back stages of the previous run
-            stage_list(appl, j - 1, bg);
-        }
-        if (j + 1 < groups)
-            for (int st = 1; st < front; ++st) stage_list(st, j + 1, bg);
-        const size_t np = prod.size(), nb = bg.size();
-        size_t ib = 0;
-        for (size_t ip = 0; ip < np; ++ip) {
-            out.push_back(prod[ip]);
-            const size_t upto = (ip + 1) * nb / np;
-            while (ib < upto) out.push_back(bg[ib++]);
-        }
-        while (ib < nb) out.push_back(bg[ib++]);
-    }
-    stage_list(scal, groups - 1, out);
-    stage_list(appl, groups - 1, out);
 }
 
-// Select the state's work tables of one kind (0 products only, 1 fused step)
-// for ns_steps k, building them on first use (host build, device allocation
-// and upload, complete before return; not allowed inside a stream capture).
-int ensure_tables(malt_state* st, int fused, int k) {
-    int groups = 1;
-    if (fused) groups = st->overlap_groups > 0 ? st->overlap_groups : -1;
-    const auto key = std::make_tuple(fused, k, groups);
-    const auto hit = st->table_cache.find(key);
-    if (hit != st->table_cache.end()) {
-        st->tables[fused] = &hit->second;
-        return MALT_OK;
-    }
-    malt_state::Tables T;
-    T.k = k;
-    T.groups = groups;
-    T.dev.assign(st->ns_groups.size(), nullptr);
-    T.len.assign(st->ns_groups.size(), 0);
-    auto release = [&T]() {
-        for (NsEntry* p : T.dev)
-            if (p != nullptr) cudaFree(p);
-    };
-    std::vector<NsEntry> host;
-    for (size_t gi = 0; gi < st->ns_groups.size(); ++gi) {
-        const NsParams& G = st->ns_groups[gi];
-        int nm = 0;
-        for (int c = 0; c < G.nclasses; ++c) nm += G.cls[c].batch;
-        build_table(G, st->ns_slot_class[gi], st->classes, st->hmats, k, fused != 0,
-                    groups > 0 ? groups : auto_overlap_groups(nm), host);
-        const size_t bytes = sizeof(NsEntry) * std::max<size_t>(host.size(), 1);
-        if (cudaMalloc(&T.dev[gi], bytes) != cudaSuccess) {
-            T.dev[gi] = nullptr;
-            cudaGetLastError();
-            release();
-            return MALT_ERR_OUT_OF_MEMORY;
-        }
-        const int rc = cuda_fail(cudaMemcpy(T.dev[gi], host.data(), sizeof(NsEntry) * host.size(),
-                                            cudaMemcpyHostToDevice), "cudaMemcpy(work table)");
-        if (rc != MALT_OK) {
-            release();
-            return rc;
-        }
-        T.len[gi] = static_cast<int32_t>(host.size());
-    }
-    // A copy from pageable memory may return before its DMA lands; the
-    // tables are read by launches on any stream, so wait for it here.
-    const int rc = cuda_fail(cudaStreamSynchronize(cudaStreamLegacy), "cudaStreamSynchronize(tables)");
-    if (rc != MALT_OK) {
-        release();
-        return rc;
-    }
-    st->tables[fused] = &st->table_cache.emplace(key, std::move(T)).first->second;
-    return MALT_OK;
-}
+// Entries per iteration of a launch group's table.
+int32_t table_per_iter(const NsParams& G) { return 2 * G.sym_items + G.full_items; }
 
 int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
     st->nmat = n;
@@ -575,6 +424,22 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
     st->sched_groups_pad = ((ngroups + 63) / 64) * 64;
     const size_t o_sched = cv.take(sizeof(uint32_t) * (st->sched_groups_pad +
                                                        static_cast<size_t>(kMaxStages) * n));
+    // Persistent work tables for kMaxNsSteps iterations, one per launch group
+    // (planned here without tensor maps, which only the launches need).
+    std::vector<std::vector<NsEntry>> tables;
+    {
+        std::vector<NsParams> groups;
+        std::vector<std::vector<int>> slot_class;
+        plan_ns_groups(st->classes, n, groups, &slot_class);
+        tables.resize(groups.size());
+        for (size_t gi = 0; gi < groups.size(); ++gi) {
+            build_table(groups[gi], slot_class[gi], st->classes, kMaxNsSteps, tables[gi]);
+            st->table_per_iter.push_back(table_per_iter(groups[gi]));
+        }
+    }
+    std::vector<size_t> o_table(tables.size());
+    for (size_t gi = 0; gi < tables.size(); ++gi)
+        o_table[gi] = cv.take(sizeof(NsEntry) * std::max<size_t>(tables[gi].size(), 1));
 
     st->ws_bytes = cv.off;
     if (cudaMalloc(&st->ws, st->ws_bytes) != cudaSuccess) {
@@ -614,6 +479,8 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
     st->d_status = reinterpret_cast<int32_t*>(base + o_status);
     for (int j = 0; j < 4; ++j) st->d_pref[j] = reinterpret_cast<int32_t*>(base + o_pref[j]);
     st->d_sched = reinterpret_cast<uint32_t*>(base + o_sched);
+    for (size_t gi = 0; gi < tables.size(); ++gi)
+        st->table_dev.push_back(reinterpret_cast<NsEntry*>(base + o_table[gi]));
 
     // Block-prefix tables.
     std::vector<int32_t> pref[4];
@@ -676,19 +543,21 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
             MALT_CUDA(cudaMemcpy(C.d_mat_of, C.mats.data(), sizeof(int32_t) * C.batch,
                                  cudaMemcpyHostToDevice), "cudaMemcpy(mat_of)");
         }
+        for (size_t gi = 0; gi < tables.size(); ++gi)
+            MALT_CUDA(cudaMemcpy(st->table_dev[gi], tables[gi].data(),
+                                 sizeof(NsEntry) * tables[gi].size(), cudaMemcpyHostToDevice),
+                      "cudaMemcpy(work table)");
     }
     return MALT_OK;
 }
 
-int bind_pointers(malt_state* st, const malt_param_t* params, cudaStream_t s,
-                  bool bump_t = false) {
+int bind_pointers(malt_state* st, const malt_param_t* params, cudaStream_t s) {
     BindParams bp;
     for (int off = 0; off < st->nmat; off += kBindChunk) {
         const int cnt = std::min(kBindChunk, st->nmat - off);
         std::memset(&bp, 0, sizeof(bp));
         bp.count = cnt;
         bp.offset = off;
-        bp.tcount = (bump_t && off == 0) ? st->d_t : nullptr;
         for (int i = 0; i < cnt; ++i) {
             const malt_param_t& p = params[off + i];
             bp.p[i] = UserPtrs{p.w, p.g, p.m, p.l, p.r};
@@ -722,8 +591,6 @@ int run_newton_schulz(malt_state* st, const malt_hparams_t* hp, cudaStream_t s) 
     bool any_persistent = false;
     for (const NsParams& G : st->ns_groups) any_persistent |= persistent(G);
     if (any_persistent) {
-        const int rc = ensure_tables(st, 0, k);
-        if (rc != MALT_OK) return rc;
         LaunchScope ls(st, MALT_KIND_NS_PERSISTENT, s, 0);   // launches counted below
         const size_t counters = st->sched_groups_pad + static_cast<size_t>(3 * k) * st->nmat;
         MALT_CUDA(cudaMemsetAsync(st->d_sched, 0, counters * sizeof(uint32_t), s),
@@ -732,9 +599,8 @@ int run_newton_schulz(malt_state* st, const malt_hparams_t* hp, cudaStream_t s) 
             const NsParams& G = st->ns_groups[gi];
             if (!persistent(G)) continue;
             prepare(G);
-            const int items = st->tables[0]->len[gi];
-            P.table = st->tables[0]->dev[gi];
-            P.front = 0;
+            const int items = k * st->table_per_iter[gi];
+            P.table = st->table_dev[gi];
             P.nstages = 3 * k;
             P.item_begin = 0;
             P.item_end = items;
@@ -800,54 +666,6 @@ StepHyper step_hyper(const malt_hparams_t* hp, int malter) {
     return sh;
 }
 
-// The whole step in one persistent launch per launch group (fused schedule):
-// statistics, finalize, prescale, norms, the Newton-Schulz products, scalars
-// and apply of each matrix, chained by the per-matrix dependency counters.
-int run_fused_step(malt_state* st, const malt_param_t* params, const malt_hparams_t* hp,
-                   cudaStream_t s, int flavour, const PipeHooks* hooks) {
-    const int k = hp->ns_steps;
-    int rc = ensure_tables(st, 1, k);
-    if (rc != MALT_OK) return rc;
-    rc = bind_pointers(st, params, s, /*bump_t=*/true);
-    if (rc != MALT_OK) return rc;
-    // The launch writes W: the previous host step's read-back must be done.
-    if (hooks != nullptr && hooks->wait_before_apply != nullptr)
-        MALT_CUDA(cudaStreamWaitEvent(s, hooks->wait_before_apply, 0), "cudaStreamWaitEvent(W read)");
-    thread_local NsParams P;
-    const int max_pairs = ns_gemm_max_pairs();
-    const int nstages = kFrontStages + 3 * k + kBackStages;
-    LaunchScope ls(st, MALT_KIND_STEP_FUSED, s, 0);          // launches counted below
-    const size_t counters = st->sched_groups_pad + static_cast<size_t>(nstages) * st->nmat;
-    MALT_CUDA(cudaMemsetAsync(st->d_sched, 0, counters * sizeof(uint32_t), s),
-              "cudaMemsetAsync(schedule counters)");
-    for (size_t gi = 0; gi < st->ns_groups.size(); ++gi) {
-        P = st->ns_groups[gi];
-        P.ns_steps = k;
-        P.a = hp->ns_a;
-        P.b = hp->ns_b;
-        P.c = hp->ns_c;
-        P.table = st->tables[1]->dev[gi];
-        P.front = kFrontStages;
-        P.nstages = nstages;
-        P.item_begin = 0;
-        P.item_end = st->tables[1]->len[gi];
-        P.ptrs = st->d_ptrs;
-        P.tcount = st->d_t;
-        P.hp = step_hyper(hp, flavour == kMalter ? 1 : 0);
-        P.decay = 1.f - hp->lr * hp->weight_decay;
-        P.with_stats = flavour == kMuon ? 0 : 1;
-        P.identity = flavour == kMuon ? 1 : 0;
-        const int pairs = std::max(1, std::min(P.item_end, max_pairs));
-        ++st->prof_launches[MALT_KIND_STEP_FUSED];
-        MALT_CUDA(launch_ns_gemm(P, kNsFused, pairs, s), "ns_gemm_kernel (fused step)");
-    }
-    if (hooks != nullptr) {
-        MALT_CUDA(cudaEventRecord(hooks->record_g_consumed, s), "cudaEventRecord(G consumed)");
-        MALT_CUDA(cudaEventRecord(hooks->record_applied, s), "cudaEventRecord(applied)");
-    }
-    return MALT_OK;
-}
-
 int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_hparams_t* hp,
              void* stream, int flavour, const PipeHooks* hooks = nullptr) {
     const int malter = flavour == kMalter ? 1 : 0;
@@ -858,7 +676,6 @@ int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_h
     st->last_stream = s;
     if (n == 0) return MALT_OK;
     MALT_CUDA(cudaSetDevice(st->device), "cudaSetDevice");
-    if (st->ns_schedule == MALT_NS_FUSED) return run_fused_step(st, params, hp, s, flavour, hooks);
     rc = bind_pointers(st, params, s);
     if (rc != MALT_OK) return rc;
     const int nm = st->nmat;
@@ -1007,10 +824,6 @@ int malt_init_state(malt_state_t** out, const malt_param_t* params, int32_t n, v
     // happens here, so a first step taken inside a stream capture makes no
     // such calls.
     if (rc == MALT_OK && n > 0) rc = cuda_fail(ns_gemm_configure(), "ns_gemm_configure");
-    // Work tables for the default ns_steps, so that a first step taken inside
-    // a stream capture uploads nothing.
-    if (rc == MALT_OK && n > 0) rc = ensure_tables(st, 0, 5);
-    if (rc == MALT_OK && n > 0) rc = ensure_tables(st, 1, 5);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     for (int i = 0; rc == MALT_OK && i < n; ++i) {
         const malt_param_t& p = params[i];
@@ -1112,6 +925,18 @@ int malt_debug_direction(malt_state_t* st, int32_t idx, void* out, void* stream)
     return MALT_OK;
 }
 
+int malt_debug_precond(malt_state_t* st, int32_t idx, float* L_out, float* R_out, void* stream) {
+    if (st == nullptr || idx < 0 || idx >= st->nmat || L_out == nullptr || R_out == nullptr)
+        return MALT_ERR_INVALID_ARG;
+    const MatDesc& d = st->hmats[idx];
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    MALT_CUDA(cudaMemcpyAsync(L_out, d.L, sizeof(float) * d.m, cudaMemcpyDeviceToDevice, s),
+              "cudaMemcpyAsync(L)");
+    MALT_CUDA(cudaMemcpyAsync(R_out, d.R, sizeof(float) * d.n, cudaMemcpyDeviceToDevice, s),
+              "cudaMemcpyAsync(R)");
+    return MALT_OK;
+}
+
 int malt_debug_scalars(malt_state_t* st, float* out_host, int32_t n) {
     if (st == nullptr || n != st->nmat || (n > 0 && out_host == nullptr)) return MALT_ERR_INVALID_ARG;
     MALT_CUDA(cudaStreamSynchronize(st->last_stream), "cudaStreamSynchronize");
@@ -1186,25 +1011,18 @@ int malt_debug_timeout_site(const malt_state_t* st, int32_t* out5) {
     return MALT_OK;
 }
 
-int malt_set_overlap_groups(malt_state_t* st, int32_t groups) {
-    if (st == nullptr || groups < 0 || groups > 64) return MALT_ERR_INVALID_ARG;
-    st->overlap_groups = groups;
-    return MALT_OK;
-}
-
 int malt_set_ns_schedule(malt_state_t* st, int32_t schedule) {
     if (st == nullptr || (schedule != MALT_NS_PHASED && schedule != MALT_NS_PERSISTENT &&
-                          schedule != MALT_NS_AUTO && schedule != MALT_NS_FUSED))
+                          schedule != MALT_NS_AUTO))
         return MALT_ERR_INVALID_ARG;
     st->ns_schedule = schedule;
     return MALT_OK;
 }
 
-int malt_ns_schedule(const malt_param_t* params, int32_t n, int32_t ns_steps, int32_t fused,
-                     int32_t overlap_groups, int32_t* out, int64_t capacity, int64_t* count) {
+int malt_ns_schedule(const malt_param_t* params, int32_t n, int32_t ns_steps, int32_t* out,
+                     int64_t capacity, int64_t* count) {
     if (count == nullptr || n < 0 || (n > 0 && params == nullptr) || ns_steps < 1 ||
-        ns_steps > kMaxNsSteps || overlap_groups < 0 || overlap_groups > 64 || capacity < 0 ||
-        (capacity > 0 && out == nullptr))
+        ns_steps > kMaxNsSteps || capacity < 0 || (capacity > 0 && out == nullptr))
         return MALT_ERR_INVALID_ARG;
     for (int i = 0; i < n; ++i)
         if (params[i].rows <= 0 || params[i].cols <= 0 || params[i].rows % 8 != 0 ||
@@ -1216,19 +1034,15 @@ int malt_ns_schedule(const malt_param_t* params, int32_t n, int32_t ns_steps, in
     std::vector<NsParams> groups;
     std::vector<std::vector<int>> slot_class;
     plan_ns_groups(classes, n, groups, &slot_class);
-    const int front = fused ? kFrontStages : 0;
     int64_t total = 0;
     std::vector<NsEntry> table;
     for (size_t gi = 0; gi < groups.size(); ++gi) {
         const NsParams& G = groups[gi];
-        int nm = 0;
-        for (int c = 0; c < G.nclasses; ++c) nm += G.cls[c].batch;
-        build_table(G, slot_class[gi], classes, hmats, ns_steps, fused != 0,
-                    overlap_groups > 0 ? overlap_groups : auto_overlap_groups(nm), table);
+        build_table(G, slot_class[gi], classes, ns_steps, table);
         for (const NsEntry& e : table) {
             if (total < capacity) {
                 const int st = entry_stage(e);
-                const int kind = stage_kind(st, front, ns_steps);
+                const int kind = st % 3;
                 int32_t* o = out + total * 8;
                 o[0] = static_cast<int32_t>(gi);
                 o[1] = st;
@@ -1237,7 +1051,7 @@ int malt_ns_schedule(const malt_param_t* params, int32_t n, int32_t ns_steps, in
                 o[4] = e.local;
                 o[5] = e.target > 0 ? (st - 1) * n + e.g : -1;
                 o[6] = static_cast<int32_t>(e.target);
-                o[7] = stage_items(kind, hmats[e.g], G.cls[entry_cls(e)]);
+                o[7] = stage_items(kind, G.cls[entry_cls(e)]);
             }
             ++total;
         }

@@ -79,7 +79,6 @@
 #include "common.cuh"
 #include "kernels.h"
 #include "ptx.cuh"
-#include "stream_blocks.cuh"
 
 namespace malt {
 
@@ -209,10 +208,9 @@ enum JobState : int32_t { kJobWork = 0, kJobEnd = -1, kJobTimeout = -2 };
 struct Job {
     int32_t state;
     int32_t stage;    // stage of the work table (persistent) or product index (phased)
-    int32_t mem;      // memory stage kind (kKindStats..kKindApply), 0 for a product tile
     int32_t g;        // matrix (-1 when not known yet: phased)
     int32_t local;
-    NsWork w;         // product tiles only
+    NsWork w;
 };
 
 __device__ __forceinline__ Job job_of_entry(const NsParams& P, const NsEntry& e) {
@@ -225,69 +223,14 @@ __device__ __forceinline__ Job job_of_entry(const NsParams& P, const NsEntry& e)
     j.stage = entry_stage(e);
     j.g = e.g;
     j.local = e.local;
-    const int s_ns = j.stage - P.front;
-    if (s_ns < 0) {
-        j.mem = kKindStats + j.stage;
-    } else if (s_ns >= 3 * P.ns_steps) {
-        j.mem = kKindScalars + (s_ns - 3 * P.ns_steps);
-    } else {
-        j.mem = 0;
-        j.w.s = s_ns;
-        j.w.iter = s_ns / 3;
-        j.w.kind = s_ns - 3 * j.w.iter;
-        j.w.cls = entry_cls(e);
-        j.w.b = entry_b(e);
-        j.w.local = e.local;
-        ns_tile_coords(P.cls[j.w.cls], j.w.kind, e.local, &j.w.mt, &j.w.nt);
-    }
+    j.w.s = j.stage;
+    j.w.iter = j.stage / 3;
+    j.w.kind = j.stage - 3 * j.w.iter;
+    j.w.cls = entry_cls(e);
+    j.w.b = entry_b(e);
+    j.w.local = e.local;
+    ns_tile_coords(P.cls[j.w.cls], j.w.kind, e.local, &j.w.mt, &j.w.nt);
     return j;
-}
-
-// One HBM-bound stage item of a fused step on the 8 epilogue warps of a CTA
-// (tid 0..255): CTA `rank` of the pair takes block 2 local + rank of a stats,
-// prescale or apply item; finalize splits rows (even CTA) and columns (odd
-// CTA); norms and scalars run on the even CTA.  Kept out of line so that its
-// registers do not weigh on the tile epilogue.
-__device__ __noinline__ void run_memory_stage(const NsParams& P, int mem, int g, int local,
-                                              int rank, int tid, float* scratch) {
-    blk::SyncEpilogue sync;
-    const MatDesc& d = P.mats[g];
-    const UserPtrs up = P.ptrs[g];
-    const int bi = 2 * local + rank;
-    switch (mem) {
-        case kKindStats:
-            if (bi < d.stat_rb * d.stat_cb) {
-                if (P.with_stats)
-                    blk::stats_block<true>(d, up, bi, P.hp.mu1, tid, scratch, sync);
-                else
-                    blk::stats_block<false>(d, up, bi, P.hp.mu1, tid, scratch, sync);
-            }
-            break;
-        case kKindFinalize: {
-            const int lo = rank ? d.m : 0, hi = rank ? d.m + d.n : d.m;
-            for (int x = lo + tid; x < hi; x += blk::kThreads)
-                blk::finalize_entry<true>(d, up, x, P.hp.mu2, P.hp.eps, P.identity);
-            break;
-        }
-        case kKindPrescale:
-            if (bi < d.pre_tr * d.pre_tc)
-                blk::prescale_block<true>(d, up, bi, P.hp.malter, tid,
-                                          reinterpret_cast<float(*)[65]>(scratch),
-                                          reinterpret_cast<float2*>(scratch + 64 * 66), sync);
-            break;
-        case kKindNorms:
-            if (rank == 0)
-                blk::norms_matrix<true>(d, P.scal + g, P.hp.ns_eps, P.hp.malter, tid, scratch, sync);
-            break;
-        case kKindScalars:
-            if (rank == 0)
-                blk::scalars_matrix<true>(d, P.scal + g, P.tcount, P.hp, tid, scratch, sync);
-            break;
-        default:                                             // kKindApply
-            if (bi < mat_apply_blocks(d))
-                blk::apply_block<true>(d, up, bi, __ldcg(&P.scal[g].scale), P.decay, tid, sync);
-            break;
-    }
 }
 
 }  // namespace
@@ -295,8 +238,7 @@ __device__ __noinline__ void run_memory_stage(const NsParams& P, int mem, int g,
 template <int kMode>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 ns_gemm_kernel(const __grid_constant__ NsParams P) {
-    constexpr bool kPersistent = kMode != kNsPhased;   // table-driven, claimed dynamically
-    constexpr bool kFused = kMode == kNsFused;         // the table also holds memory stages
+    constexpr bool kPersistent = kMode == kNsPersistent;   // table-driven, claimed dynamically
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[kRing];
     __shared__ __align__(8) uint64_t empty_bar[kRing];
@@ -380,7 +322,6 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
         j.state = kJobWork;
         j.w = ns_decode(P, static_cast<int>(it));
         j.stage = j.w.s;
-        j.mem = 0;
         j.g = -1;
         j.local = j.w.local;
         return j;
@@ -462,7 +403,6 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                     break;
                 }
                 if (job.state == kJobEnd) break;
-                if (kFused && job.mem) continue;         // memory stages load no operands
                 const int item = job.local;
                 // The loads below read what other CTAs stored in this launch.
                 if (kPersistent) fence_proxy_async_global();
@@ -547,7 +487,6 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
                     break;
                 }
                 if (job.state == kJobEnd) break;
-                if (kFused && job.mem) continue;
                 const int item = job.local;
                 const NsWork& w = job.w;
                 const bool b_mn = w.kind == kBX;
@@ -612,8 +551,6 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
         const int colw = (ew >> 2) * kEpiCols;    // first accumulator column of this warp
         const uint32_t tempty_leader0 = mapa_shared(smem_u32(&tempty_bar[0]), 0);
         const uint32_t tempty_leader1 = mapa_shared(smem_u32(&tempty_bar[1]), 0);
-        const int tid = ew * 32 + lane;           // thread of the 256 running memory stages
-        float* scratch = reinterpret_cast<float*>(stage_out);
         int gi = 0;                               // product tiles so far (accumulator)
         for (int seq = 0;; ++seq) {
             Job job;
@@ -644,21 +581,6 @@ ns_gemm_kernel(const __grid_constant__ NsParams P) {
             }
             if (job.state == kJobEnd) break;
             const int item = job.local;
-            if (kFused && job.mem) {
-                // ---- an HBM-bound stage of the fused step, on the 8 epilogue
-                // warps of each CTA; the staging area is its shared scratch.
-                if (lane == 0) bulk_wait_group_read<0>();   // no tile store still reads it
-                blk::SyncEpilogue sync;
-                sync();
-                run_memory_stage(P, job.mem, job.g, job.local, rank, tid, scratch);
-                sync();                                      // scratch free for tile stores again
-                __syncwarp();
-                if (lane == 0 && job.stage + 1 < P.nstages) {
-                    __threadfence();
-                    red_release_gpu_add(P.done + job.stage * P.nmat + job.g, 1u);
-                }
-                continue;
-            }
             const NsWork& w = job.w;
             const NsClass& C = P.cls[w.cls];
             const uint32_t acc = gi & 1, acc_phase = (gi >> 1) & 1;
@@ -874,7 +796,6 @@ cudaError_t set_smem_attr() {
 cudaError_t set_all_smem_attrs() {
     cudaError_t e = set_smem_attr<kNsPhased>();
     if (e == cudaSuccess) e = set_smem_attr<kNsPersistent>();
-    if (e == cudaSuccess) e = set_smem_attr<kNsFused>();
     return e;
 }
 
@@ -901,7 +822,7 @@ cudaError_t configure_current_device(int* pairs) {
         cfg.gridDim = dim3(2, 1, 1);
         cfg.blockDim = dim3(kThreads, 1, 1);
         cfg.dynamicSmemBytes = kSmemBytes;
-        if (cudaOccupancyMaxActiveClusters(&n, ns_gemm_kernel<kNsFused>, &cfg) != cudaSuccess ||
+        if (cudaOccupancyMaxActiveClusters(&n, ns_gemm_kernel<kNsPersistent>, &cfg) != cudaSuccess ||
             n <= 0) {
             cudaGetLastError();
             int sms = 0;
@@ -937,18 +858,14 @@ cudaError_t ns_gemm_configure() {
 cudaError_t launch_ns_gemm(const NsParams& P, int mode, int grid_pairs, cudaStream_t s) {
     const cudaError_t ce = ns_gemm_configure();
     if (ce != cudaSuccess) return ce;
-    if (mode == kNsFused)
-        ns_gemm_kernel<kNsFused><<<2 * grid_pairs, kThreads, kSmemBytes, s>>>(P);
-    else if (mode == kNsPersistent)
+    if (mode == kNsPersistent)
         ns_gemm_kernel<kNsPersistent><<<2 * grid_pairs, kThreads, kSmemBytes, s>>>(P);
     else
         ns_gemm_kernel<kNsPhased><<<2 * grid_pairs, kThreads, kSmemBytes, s>>>(P);
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) {
         cudaFuncAttributes fa{};
-        if (mode == kNsFused)
-            cudaFuncGetAttributes(&fa, ns_gemm_kernel<kNsFused>);
-        else if (mode == kNsPersistent)
+        if (mode == kNsPersistent)
             cudaFuncGetAttributes(&fa, ns_gemm_kernel<kNsPersistent>);
         else
             cudaFuncGetAttributes(&fa, ns_gemm_kernel<kNsPhased>);

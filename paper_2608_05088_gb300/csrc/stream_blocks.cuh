@@ -1,9 +1,10 @@
 // stream_blocks.cuh -- the HBM-bound stages of the MALT / MALTER step as
-// block-level device functions of 256 threads (tid 0..255).  The standalone
-// kernels of stream_kernels.cu run one call per CUDA block; the fused step
-// kernel (ns_gemm.cu) runs the same calls on the 8 epilogue warps of a CTA,
-// between Newton-Schulz tiles.  Both run the same arithmetic in the same
-// order, so a step gives bitwise the same result either way.
+// block-level device functions of 256 threads (tid 0..255).  The kernels of
+// stream_kernels.cu run one call per CUDA block; malt_stats_noalloc
+// (noalloc.cu) runs the statistics and finalize blocks of one matrix on its
+// own scratch.  Every multiply-add that decides a rounding is an explicit
+// fmaf / fma, so each block computes bitwise the same result in every
+// translation unit it is compiled into.
 //
 //   stats     Algorithm 1, M_t / l_t / r_t lines: one pass over G and M that
 //             updates the momentum and writes per-tile partial sums of G^2 for
@@ -18,11 +19,6 @@
 //             grafted scale lr * alpha * ||O|| / (||D|| + eps) per matrix.
 //   apply     W <- (1 - lr wd) W - scale * L O R (Algorithm 1, W_t line), with
 //             O in W's layout, streamed contiguously.
-//
-// Template flag kL2: data that an earlier stage of the same launch may have
-// written (M, L, R, the partial sums, the per-matrix scalars, O) is read
-// through L2 only (ld.global.cg), so a stale L1 line is never used.  False in
-// the standalone kernels, where every input comes from an earlier launch.
 #pragma once
 #include <cuda_bf16.h>
 #include <cstdint>
@@ -34,17 +30,6 @@ namespace blk {
 
 constexpr int kThreads = 256;
 
-// Block-wide barrier of the threads running a block function.
-struct SyncBlock {
-    __device__ __forceinline__ void operator()() const { __syncthreads(); }
-};
-// The 8 epilogue warps of a CTA of the fused kernel (named barrier 1).
-struct SyncEpilogue {
-    __device__ __forceinline__ void operator()() const {
-        asm volatile("bar.sync 1, 256;" ::: "memory");
-    }
-};
-
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -53,19 +38,17 @@ __device__ __forceinline__ float warp_sum(float v) {
 
 // Sum of v over the first nthreads threads (a multiple of 32) in a fixed
 // order; every thread of the block calls it, the result is valid in tid 0.
-template <class Sync>
-__device__ __forceinline__ float block_sum(float v, float* sh /* >= 32 */, int tid, int nthreads,
-                                           Sync sync) {
+__device__ __forceinline__ float block_sum(float v, float* sh /* >= 32 */, int tid, int nthreads) {
     v = warp_sum(v);
     const int w = tid >> 5, lane = tid & 31;
     if (lane == 0 && tid < nthreads) sh[w] = v;
-    sync();
+    __syncthreads();
     float s = 0.f;
     if (tid == 0) {
         const int nw = nthreads >> 5;
         for (int i = 0; i < nw; ++i) s += sh[i];
     }
-    sync();
+    __syncthreads();
     return s;
 }
 
@@ -88,12 +71,6 @@ template <int kPath>
 __device__ __forceinline__ float ld_f(const float* p) {
     return kPath == kLdRO ? __ldg(p) : kPath == kLdL2 ? __ldcg(p) : *p;
 }
-
-// Path of data an earlier stage of the same launch may have written.
-template <bool kL2>
-struct Mut {
-    static constexpr int kPath = kL2 ? kLdL2 : kLdPlain;
-};
 
 // 8 consecutive elements (bf16 or fp32) at element offset off, as floats.
 template <int kPath = kLdRO>
@@ -133,9 +110,9 @@ __device__ __forceinline__ uint4 pack8_bf16(const float (&v)[8]) {
 constexpr int kStatRowsPerWarp = kStatRows / 8;
 constexpr int kStatBatch = 4;
 
-template <bool kStats, class Sync>
+template <bool kStats>
 __device__ __forceinline__ void stats_block(const MatDesc& d, const UserPtrs& up, int local,
-                                            float mu1, int tid, float* colsh, Sync sync) {
+                                            float mu1, int tid, float* colsh) {
     const int m = d.m, n = d.n;
     const int rb = local / d.stat_cb, cb = local - rb * d.stat_cb;
     const int warp = tid >> 5, lane = tid & 31;
@@ -203,7 +180,7 @@ __device__ __forceinline__ void stats_block(const MatDesc& d, const UserPtrs& up
     float4* cs = reinterpret_cast<float4*>(colsh + warp * kStatCols + lane * 8);
     cs[0] = make_float4(csum[0], csum[1], csum[2], csum[3]);
     cs[1] = make_float4(csum[4], csum[5], csum[6], csum[7]);
-    sync();
+    __syncthreads();
     const int c = tid;
     const int gc = cb * kStatCols + c;
     if (gc < n) {
@@ -217,10 +194,9 @@ __device__ __forceinline__ void stats_block(const MatDesc& d, const UserPtrs& up
 // --------------------------------------------------------------- finalize
 // Entry `local` of the matrix's m + n statistics: row i = local (< m) or
 // column j = local - m.  identity (Muon): L = R = 1, statistics untouched.
-template <bool kL2 = false>
 __device__ __forceinline__ void finalize_entry(const MatDesc& d, const UserPtrs& up, int local,
                                                float mu2, float eps, int identity) {
-    constexpr int P = Mut<kL2>::kPath;
+    constexpr int P = kLdPlain;
     if (identity) {
         if (local < d.m) d.L[local] = 1.f; else d.R[local - d.m] = 1.f;
         return;
@@ -249,11 +225,10 @@ __device__ __forceinline__ void finalize_entry(const MatDesc& d, const UserPtrs&
 // tall matrix's NS frame is Mt^T, so its block walks four 64 x 64 sub-tiles
 // through shared memory (tile: 64 x 65 floats) and writes each transposed.
 // red: 8 float2.
-template <bool kL2, class Sync>
 __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs& up, int local,
                                                int malter, int tid, float (*tile)[65],
-                                               float2* red, Sync sync) {
-    constexpr int P = Mut<kL2>::kPath;
+                                               float2* red) {
+    constexpr int P = kLdPlain;
     const int m = d.m, n = d.n;
     // A tall matrix's blocks walk down a column band first, so the blocks
     // resident at once write neighbouring pieces of the same X0 rows.
@@ -363,7 +338,7 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
                     v0 = Li * q.x * R4.x; v1 = Li * q.y * R4.y;
                     v2 = Li * q.z * R4.z; v3 = Li * q.w * R4.w;
                     // explicit fused multiply-adds: the same rounding wherever
-                    // this block is compiled (standalone kernel or fused step)
+                    // this block is compiled
                     s_mt = fmaf(v3, v3, fmaf(v2, v2, fmaf(v1, v1, fmaf(v0, v0, s_mt))));
                     if (malter) {
                         float gq[4];
@@ -387,7 +362,7 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
                 tile[rr][cc + 2] = v2; tile[rr][cc + 3] = v3;
             }
             if (sub + 2 < kSubs) load_sub(sub + 2, mq[sub & 1]);
-            sync();
+            __syncthreads();
             // Output row = column of Mt, 8 consecutive rows of Mt per thread.
 #pragma unroll
             for (int pass = 0; pass < 2; ++pass) {
@@ -402,7 +377,7 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
                         pack8_bf16(v);
                 }
             }
-            sync();                                       // tile is reused by the next sub-tile
+            __syncthreads();                                       // tile is reused by the next sub-tile
         }
     }
     // One fixed-order reduction of both partial sums.
@@ -412,7 +387,7 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
         s_lgr += __shfl_xor_sync(0xffffffffu, s_lgr, o);
     }
     if (lane == 0) red[warp] = make_float2(s_mt, s_lgr);
-    sync();
+    __syncthreads();
     if (t == 0) {
         float a = 0.f, b = 0.f;
 #pragma unroll
@@ -427,18 +402,17 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
 
 // ------------------------------------------------------------------ norms
 // ||Mt||_F, 1 / (||Mt||_F + ns_eps) and ||L G R||_F^2 of one matrix (256 threads).
-template <bool kL2, class Sync>
 __device__ __forceinline__ void norms_matrix(const MatDesc& d, MatScalars* sc, float ns_eps,
-                                             int malter, int tid, float* red, Sync sync) {
-    constexpr int P = Mut<kL2>::kPath;
+                                             int malter, int tid, float* red) {
+    constexpr int P = kLdPlain;
     const int tiles = d.pre_tr * d.pre_tc;
     float a = 0.f, b = 0.f;
     for (int i = tid; i < tiles; i += kThreads) {
         a += ld_f<P>(d.prepart + 2 * i);
         b += ld_f<P>(d.prepart + 2 * i + 1);
     }
-    a = block_sum(a, red, tid, kThreads, sync);
-    b = block_sum(b, red, tid, kThreads, sync);
+    a = block_sum(a, red, tid, kThreads);
+    b = block_sum(b, red, tid, kThreads);
     if (tid == 0) {
         const float nrm = sqrtf(a);
         sc->norm_mt = nrm;
@@ -453,11 +427,10 @@ __device__ __forceinline__ void norms_matrix(const MatDesc& d, MatScalars* sc, f
 // block size), so the result does not depend on who runs it.
 constexpr int kScalarThreads = 128;
 
-template <bool kL2, class Sync>
 __device__ __forceinline__ void scalars_matrix(const MatDesc& d, MatScalars* sc,
                                                const long long* tcount, const StepHyper& hp,
-                                               int tid, float* red, Sync sync) {
-    constexpr int P = Mut<kL2>::kPath;
+                                               int tid, float* red) {
+    constexpr int P = kLdPlain;
     float a = 0.f, b = 0.f;
     // One partial per epilogue warp per GEMM tile of the last iteration.
     if (tid < kScalarThreads) {
@@ -466,8 +439,8 @@ __device__ __forceinline__ void scalars_matrix(const MatDesc& d, MatScalars* sc,
             b += ld_f<P>(d.nspart + 2 * i + 1);
         }
     }
-    a = block_sum(a, red, tid, kScalarThreads, sync);
-    b = block_sum(b, red, tid, kScalarThreads, sync);
+    a = block_sum(a, red, tid, kScalarThreads);
+    b = block_sum(b, red, tid, kScalarThreads);
     if (tid == 0) {
         MatScalars s;
         {
@@ -483,8 +456,7 @@ __device__ __forceinline__ void scalars_matrix(const MatDesc& d, MatScalars* sc,
             // Algorithm 2, nu_t line; alpha_t as displayed in Section 3.5.
             const double t = static_cast<double>(*tcount);
             // One explicit fma, so that no compilation of this block
-            // contracts the two products differently (the fused step runs
-            // it inside the GEMM kernel).
+            // contracts the two products differently.
             const double nu = fma(static_cast<double>(hp.mu2), static_cast<double>(s.nu),
                                   (1.0 - static_cast<double>(hp.mu2)) * s.lgr_sq);
             const double bc = sqrt(1.0 - pow(static_cast<double>(hp.mu2), t)) /
@@ -539,14 +511,12 @@ __device__ __forceinline__ void apply8(const MatDesc& d, const UserPtrs& up, boo
 
 // Block `local` of the apply pass: kApplyElems contiguous elements (O is in
 // W's layout).  s = the grafted scale.
-template <bool kL2, class Sync>
 __device__ __forceinline__ void apply_block(const MatDesc& d, const UserPtrs& up, int local,
-                                            float s, float decay, int tid, Sync sync) {
-    constexpr int P = Mut<kL2>::kPath;
-    constexpr int PO = kL2 ? kLdL2 : kLdRO;       // O: read-only path unless written in-launch
+                                            float s, float decay, int tid) {
+    constexpr int P = kLdPlain;
+    constexpr int PO = kLdRO;                     // O: written by an earlier launch
     const int m = d.m, n = d.n;
     const bool wbf = d.w_bf16 != 0;
-    (void)sync;
     const int32_t total = m * n;
     const int32_t e0 = local * kApplyElems;
 #pragma unroll 4

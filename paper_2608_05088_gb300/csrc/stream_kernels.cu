@@ -33,7 +33,6 @@ __device__ __forceinline__ int find_mat(const int32_t* __restrict__ pref, int nm
 __global__ void bind_kernel(const __grid_constant__ BindParams P, UserPtrs* __restrict__ table) {
     const int i = threadIdx.x;
     if (i < P.count) table[P.offset + i] = P.p[i];
-    if (i == 0 && P.tcount != nullptr) *P.tcount += 1;   // fused step: 1-based step count
 }
 
 // ------------------------------------------------------------------ stats
@@ -44,7 +43,7 @@ stats_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs
     __shared__ __align__(16) float colsh[8 * kStatCols];
     const int g = find_mat(pref, nmat, blockIdx.x);
     blk::stats_block<kStats>(mats[g], ptrs[g], blockIdx.x - __ldg(pref + g), mu1, threadIdx.x,
-                             colsh, blk::SyncBlock{});
+                             colsh);
 }
 
 // --------------------------------------------------------------- finalize
@@ -56,7 +55,7 @@ finalize_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ p
     if (x == 0) *tcount += 1;                 // 1-based step count
     if (x >= total) return;
     const int g = find_mat(pref, nmat, x);
-    blk::finalize_entry<false>(mats[g], ptrs[g], x - __ldg(pref + g), mu2, eps, identity);
+    blk::finalize_entry(mats[g], ptrs[g], x - __ldg(pref + g), mu2, eps, identity);
 }
 
 // --------------------------------------------------------------- prescale
@@ -66,8 +65,8 @@ prescale_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ p
     __shared__ float tile[64][65];
     __shared__ float2 red[8];
     const int g = find_mat(pref, nmat, blockIdx.x);
-    blk::prescale_block<false>(mats[g], ptrs[g], blockIdx.x - __ldg(pref + g), malter, threadIdx.x,
-                        tile, red, blk::SyncBlock{});
+    blk::prescale_block(mats[g], ptrs[g], blockIdx.x - __ldg(pref + g), malter, threadIdx.x, tile,
+                        red);
 }
 
 // ------------------------------------------------------------------ norms
@@ -76,7 +75,7 @@ norms_kernel(const MatDesc* __restrict__ mats, MatScalars* __restrict__ scal, fl
              int malter) {
     __shared__ float red[32];
     const int g = blockIdx.x;
-    blk::norms_matrix<false>(mats[g], scal + g, ns_eps, malter, threadIdx.x, red, blk::SyncBlock{});
+    blk::norms_matrix(mats[g], scal + g, ns_eps, malter, threadIdx.x, red);
 }
 
 // ---------------------------------------------------------------- scalars
@@ -85,7 +84,7 @@ scalars_kernel(const MatDesc* __restrict__ mats, MatScalars* __restrict__ scal,
                const long long* __restrict__ tcount, StepHyper hp) {
     __shared__ float red[32];
     const int g = blockIdx.x;
-    blk::scalars_matrix<false>(mats[g], scal + g, tcount, hp, threadIdx.x, red, blk::SyncBlock{});
+    blk::scalars_matrix(mats[g], scal + g, tcount, hp, threadIdx.x, red);
 }
 
 // ------------------------------------------------------------------ apply
@@ -94,8 +93,8 @@ apply_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs
              const MatScalars* __restrict__ scal, const int32_t* __restrict__ pref, int nmat,
              float decay) {
     const int g = find_mat(pref, nmat, blockIdx.x);
-    blk::apply_block<false>(mats[g], ptrs[g], blockIdx.x - __ldg(pref + g), scal[g].scale, decay,
-                           threadIdx.x, blk::SyncBlock{});
+    blk::apply_block(mats[g], ptrs[g], blockIdx.x - __ldg(pref + g), scal[g].scale, decay,
+                     threadIdx.x);
 }
 
 // ------------------------------------------------------------- wait probe

@@ -32,19 +32,17 @@ EXPORTS = ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
            "malt_debug_wait_timeout", "malt_profile_enable", "malt_profile_read",
            "malt_workspace_bytes", "malt_status_string", "malt_destroy_state",
            "malt_stats_noalloc", "malt_step_host", "muon_step", "malt_set_ns_schedule",
-           "malt_ns_schedule", "malt_debug_timeout_site", "malt_set_overlap_groups")
+           "malt_ns_schedule", "malt_debug_timeout_site", "malt_debug_precond")
 NOALLOC_SCRATCH_FLOATS = 1048576
 KIND_NAMES = ("bind", "stats", "finalize", "prescale", "norms", "ns_gram", "ns_poly", "ns_bx",
-              "scalars", "apply", "ns_persistent", "step_fused")
+              "scalars", "apply", "ns_persistent")
 NS_KINDS = ("ns_gram", "ns_poly", "ns_bx", "ns_persistent")
 # Newton-Schulz schedules (malt_set_ns_schedule)
 MALT_NS_PHASED = 0
 MALT_NS_PERSISTENT = 1
 MALT_NS_AUTO = 2
-MALT_NS_FUSED = 3
-# stage kinds of malt_ns_schedule
-STAGE_KIND_NAMES = ("gram", "poly", "bx", "stats", "finalize", "prescale", "norms", "scalars",
-                    "apply")
+# product kinds of malt_ns_schedule
+STAGE_KIND_NAMES = ("gram", "poly", "bx")
 
 
 class malt_param_t(ctypes.Structure):
@@ -94,6 +92,8 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.malt_set_scalars.argtypes = [vp, P(ctypes.c_float), i32, i64]
     lib.malt_check.argtypes = [vp]
     lib.malt_debug_direction.argtypes = [vp, i32, vp, vp]
+    lib.malt_debug_precond.argtypes = [vp, i32, vp, vp, vp]
+    lib.malt_debug_precond.restype = ctypes.c_int
     lib.malt_debug_scalars.argtypes = [vp, P(ctypes.c_float), i32]
     lib.malt_debug_wait_timeout.argtypes = [i64, vp]
     lib.malt_profile_enable.argtypes = [vp, i32]
@@ -116,9 +116,7 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.malt_debug_timeout_site.restype = ctypes.c_int
     lib.malt_set_ns_schedule.argtypes = [vp, i32]
     lib.malt_set_ns_schedule.restype = ctypes.c_int
-    lib.malt_ns_schedule.argtypes = [P(malt_param_t), i32, i32, i32, i32, P(i32), i64, P(i64)]
-    lib.malt_set_overlap_groups.argtypes = [vp, i32]
-    lib.malt_set_overlap_groups.restype = ctypes.c_int
+    lib.malt_ns_schedule.argtypes = [P(malt_param_t), i32, i32, P(i32), i64, P(i64)]
     lib.malt_ns_schedule.restype = ctypes.c_int
     for name in ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
                  "malt_set_scalars", "malt_check", "malt_debug_direction",
@@ -235,6 +233,12 @@ def malt_debug_direction(st, idx: int, out, stream=None):
                                        _stream_handle(stream)), "malt_debug_direction")
 
 
+def malt_debug_precond(st, idx: int, L_out, R_out, stream=None):
+    _check(load().malt_debug_precond(st, idx, ctypes.c_void_p(L_out.data_ptr()),
+                                     ctypes.c_void_p(R_out.data_ptr()), _stream_handle(stream)),
+           "malt_debug_precond")
+
+
 def malt_debug_scalars(st, n: int) -> np.ndarray:
     buf = (ctypes.c_float * max(n * SCALARS_PER_MAT, 1))()
     _check(load().malt_debug_scalars(st, buf, n), "malt_debug_scalars")
@@ -258,11 +262,42 @@ def malt_profile_read(st):
     return {KIND_NAMES[k]: (float(ms[k]), int(cnt[k])) for k in range(n)}
 
 
+def _noalloc_check(G, M, l, r, L_out, R_out):
+    """The tensors malt_stats_noalloc hands to its kernels as raw pointers:
+    contiguous, on the current CUDA device, with the shapes and dtypes the
+    kernels index (M rows x cols fp32, G the same shape in fp32 or bf16, l and
+    L_out rows fp32, r and R_out cols fp32).  Raises ValueError otherwise."""
+    import torch
+    if M.dim() != 2:
+        raise ValueError("M must be a 2-D rows x cols tensor")
+    rows, cols = M.shape
+    want = {"G": (G, (rows, cols), (torch.float32, torch.bfloat16)),
+            "M": (M, (rows, cols), (torch.float32,)),
+            "l": (l, (rows,), (torch.float32,)), "L_out": (L_out, (rows,), (torch.float32,)),
+            "r": (r, (cols,), (torch.float32,)), "R_out": (R_out, (cols,), (torch.float32,))}
+    for name, (t, shape, dtypes) in want.items():
+        if tuple(t.shape) != shape:
+            raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {shape}")
+        if t.dtype not in dtypes:
+            raise ValueError(f"{name} has dtype {t.dtype}, expected one of {dtypes}")
+        if not t.is_contiguous():
+            raise ValueError(f"{name} must be contiguous")
+    for name, (t, _, _) in want.items():
+        if not t.is_cuda:
+            raise ValueError(f"{name} must be a CUDA tensor, not on {t.device}")
+    dev = torch.cuda.current_device()
+    for name, (t, _, _) in want.items():
+        if t.device.index != dev:
+            raise ValueError(f"{name} must be on the current CUDA device (cuda:{dev}), not {t.device}")
+    return rows, cols
+
+
 def malt_stats_noalloc(G, M, l, r, L_out, R_out, mu1=0.95, mu2=0.99, eps=1e-8, stream=None) -> int:
     """Statistics stage of one matrix with no device allocation (see
-    include/malt.h).  Returns the status code; it does not raise, so callers
-    can see MALT_ERR_UNSUPPORTED for matrices past the scratch limit."""
-    rows, cols = M.shape
+    include/malt.h).  Checks the tensors (ValueError on a mismatch), then
+    returns the library's status code without raising, so callers can see
+    MALT_ERR_UNSUPPORTED for matrices past the scratch limit."""
+    rows, cols = _noalloc_check(G, M, l, r, L_out, R_out)
     return load().malt_stats_noalloc(
         ctypes.c_void_p(G.data_ptr()), _dtype_code(G), ctypes.c_void_p(M.data_ptr()),
         ctypes.c_void_p(l.data_ptr()), ctypes.c_void_p(r.data_ptr()),
@@ -289,29 +324,25 @@ def malt_set_ns_schedule(st, schedule: int):
     _check(load().malt_set_ns_schedule(st, int(schedule)), "malt_set_ns_schedule")
 
 
-def malt_ns_schedule(shapes, ns_steps: int, fused: bool = False, overlap_groups: int = 0):
-    """The work table of the persistent (or, with fused=True, the fused-step)
-    schedule for these (rows, cols) shapes, computed on the host by the
-    library (no GPU): an int32 array of shape (items, 8) with columns launch
-    group, stage, stage kind (STAGE_KIND_NAMES), matrix, local index,
-    counter index, counter target, items of (stage, matrix)."""
+def malt_ns_schedule(shapes, ns_steps: int):
+    """The work table of the persistent schedule for these (rows, cols)
+    shapes, computed on the host by the library (no GPU): an int32 array of
+    shape (items, 8) with columns launch group, stage, product kind
+    (STAGE_KIND_NAMES), matrix, tile, counter index, counter target, tiles of
+    (stage, matrix)."""
     import numpy as np
     arr = (malt_param_t * max(len(shapes), 1))()
     for i, (rows, cols) in enumerate(shapes):
         arr[i] = malt_param_t(None, MALT_F32, None, MALT_F32, None, None, None, rows, cols)
     lib = load()
     count = ctypes.c_int64(0)
-    _check(lib.malt_ns_schedule(arr, len(shapes), ns_steps, int(fused), overlap_groups, None, 0,
-                                ctypes.byref(count)), "malt_ns_schedule")
+    _check(lib.malt_ns_schedule(arr, len(shapes), ns_steps, None, 0, ctypes.byref(count)),
+           "malt_ns_schedule")
     out = np.zeros((count.value, 8), dtype=np.int32)
-    _check(lib.malt_ns_schedule(arr, len(shapes), ns_steps, int(fused), overlap_groups,
+    _check(lib.malt_ns_schedule(arr, len(shapes), ns_steps,
                                 out.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)),
                                 count.value, ctypes.byref(count)), "malt_ns_schedule")
     return out
-
-
-def malt_set_overlap_groups(st, groups: int):
-    _check(load().malt_set_overlap_groups(st, int(groups)), "malt_set_overlap_groups")
 
 
 # --- convenience wrapper ------------------------------------------------------
@@ -357,14 +388,20 @@ class MaltOptimizer:
         malt_debug_direction(self.state, idx, out, stream)
         return out
 
+    def precond(self, idx: int, stream=None):
+        """(L, R) of parameter idx as the last step computed them."""
+        import torch
+        W = self.params[idx][0]
+        L = torch.empty(W.shape[0], dtype=torch.float32, device=W.device)
+        R = torch.empty(W.shape[1], dtype=torch.float32, device=W.device)
+        malt_debug_precond(self.state, idx, L, R, stream)
+        return L, R
+
     def timeout_site(self):
         return malt_debug_timeout_site(self.state)
 
     def set_ns_schedule(self, schedule: int):
         malt_set_ns_schedule(self.state, schedule)
-
-    def set_overlap_groups(self, groups: int):
-        malt_set_overlap_groups(self.state, groups)
 
     def profile(self, enable: bool = True):
         malt_profile_enable(self.state, enable)

@@ -27,6 +27,35 @@ def bf16_ulp(x: np.ndarray) -> np.ndarray:
     return np.ldexp(1.0, np.maximum(e - 8, -133))
 
 
+def bf16_rounding(W_gpu, x_gpu, x_ref, slack, dW_ref):
+    """Rounding checks of a bf16 weight update against the oracle.
+
+    x_gpu: the GPU's pre-rounding value rebuilt in fp64 (exact up to `slack`,
+    the kernel's own fp32 rounding); x_ref: the oracle's.  An entry
+    "straddles" when a bf16 rounding boundary lies between the two values
+    (the interval widened by the slack); elsewhere both must round alike.
+      own_mismatch: entries with W_gpu != rn(x_gpu) although no boundary lies
+        within the slack of x_gpu (must be 0);
+      oracle_mismatch_off_boundary: entries with W_gpu != rn(x_ref) that do
+        not straddle (must be 0);
+      straddle: the fraction of entries that straddle;
+      straddle_allowed: the fraction the update tolerance would allow, the
+        mean over entries of min(1, TOL_DW |dW_ref| / ulp) -- the chance that
+        a boundary falls between two values that far apart.
+    """
+    rn = ref.round_to_bf16
+    near = rn(x_gpu - slack) != rn(x_gpu + slack)            # within slack of a boundary
+    own_mismatch = int(np.sum((W_gpu != rn(x_gpu)) & ~near))
+    lo = np.minimum(x_gpu, x_ref) - slack
+    hi = np.maximum(x_gpu, x_ref) + slack
+    straddle = rn(lo) != rn(hi)
+    off = int(np.sum((W_gpu != rn(x_ref)) & ~straddle))
+    ulp = bf16_ulp(np.maximum(np.abs(x_ref), np.abs(x_gpu)))
+    allowed = float(np.mean(np.minimum(1.0, TOL_DW * np.abs(dW_ref) / ulp)))
+    return dict(own_mismatch=own_mismatch, oracle_mismatch_off_boundary=off,
+                straddle=float(np.mean(straddle)), straddle_allowed=allowed)
+
+
 class Run:
     """One optimizer state on the GPU plus oracle states for `check` matrices."""
 
@@ -84,7 +113,6 @@ class Run:
         """One step on the GPU (and the oracle for checked matrices)."""
         s = self.steps_done
         self.W_prev = {i: self.host(self.W[i]) for i in self.check if self.w_dtypes[i] == "bf16"}
-        self.W_prev_ref = {i: self.W_ref[i].copy() for i in self.W_prev}
         for i in range(len(self.wl.shapes)):
             G = grads[i] if grads is not None else self.gradient(i, s)
             self.G[i].copy_(self.torch.from_numpy(np.ascontiguousarray(G)))
@@ -109,32 +137,38 @@ class Run:
         info = self.info[i]
         W = self.host(self.W[i])
         O = self.host(self.opt.direction(i))
+        Lg, Rg = (self.host(t) for t in self.opt.precond(i))
         sc = self.opt.debug_scalars()[i]
+        out = dict(W_gpu=W, W_pre=None, W_pre_ref=None, slack=None)
         if self.w_dtypes[i] == "bf16":
             # bf16 rounding decides most entries of W_0 - W_t, so compare the
-            # pre-rounding update rebuilt from the GPU's own l, r, O and scale.
-            eps = self.hp_ref.eps
-            if self.variant == "muon":
-                Lg, Rg = np.ones(W.shape[0]), np.ones(W.shape[1])
-            else:
-                Lg = (self.host(self.l[i]) + eps) ** -0.125
-                Rg = (self.host(self.r[i]) + eps) ** -0.125
+            # pre-rounding update, rebuilt exactly (fp64) from the step's own
+            # L, R, bf16 O and fp32 scale, with the oracle's.
             dW = float(sc[6]) * Lg[:, None] * O * Rg[None, :]
             dW_ref = info["delta"]
-            # the GPU's own pre-rounding value, decoupled decay included
-            W_pre = self.decay_gpu * self.W_prev[i] - dW
             hp = self.hp_ref
-            W_pre_ref = (1.0 - hp.lr * hp.weight_decay) * self.W_prev_ref[i] - dW_ref
+            # Both pre-rounding values start from the GPU's previous W (the
+            # oracle teacher-forced), so their gap is this step's only.
+            W_pre = self.decay_gpu * self.W_prev[i] - dW
+            W_pre_ref = (1.0 - hp.lr * hp.weight_decay) * self.W_prev[i] - dW_ref
+            # the apply kernel's own fp32 arithmetic (s L_i, its product with
+            # O_ij, decay * W, one fma) moves its value from W_pre by at most a
+            # few fp32 ulps of the terms
+            out.update(W_pre=W_pre, W_pre_ref=W_pre_ref,
+                       slack=2.0 ** -21 * (np.abs(W_pre) + np.abs(dW)))
         else:
             dW = self.W0[i] - W
             dW_ref = self.W0[i] - self.W_ref[i]
         stats_used = self.variant != "muon"      # Muon leaves l and r untouched
-        return dict(
+
+        def elem(a, b):
+            return float(np.max(np.abs(a - b) / np.maximum(np.abs(b), 1e-30)))
+        out.update(
             M=rel(self.host(self.M[i]), st.M),
-            l=float(np.max(np.abs(self.host(self.l[i]) - st.l) / np.maximum(st.l, 1e-30)))
-            if stats_used else 0.0,
-            r=float(np.max(np.abs(self.host(self.r[i]) - st.r) / np.maximum(st.r, 1e-30)))
-            if stats_used else 0.0,
+            l=elem(self.host(self.l[i]), st.l) if stats_used else 0.0,
+            r=elem(self.host(self.r[i]), st.r) if stats_used else 0.0,
+            L=elem(Lg, info["L"]),
+            R=elem(Rg, info["R"]),
             O=rel(O, info["O"]),
             W=rel(W, self.W_ref[i]),
             dW=rel(dW, dW_ref),
@@ -143,34 +177,36 @@ class Run:
             norm_d=abs(sc[1] - info["norm_D"]) / max(info["norm_D"], 1e-30),
             alpha=abs(sc[5] - info["alpha"]) / max(abs(info["alpha"]), 1e-30),
             nu=(abs(sc[4] - info["nu"]) / max(info["nu"], 1e-30)) if self.variant == "malter" else 0.0,
-            W_gpu=W,
-            W_pre=W_pre if self.w_dtypes[i] == "bf16" else None,
-            W_pre_ref=W_pre_ref if self.w_dtypes[i] == "bf16" else None,
         )
+        if self.w_dtypes[i] == "bf16":
+            out.update(bf16_rounding(W, out["W_pre"], out["W_pre_ref"], out["slack"], dW_ref))
+        return out
 
     def assert_close(self, i, ctx=""):
         e = self.compare(i)
+        arrays = ("W_gpu", "W_pre", "W_pre_ref", "slack")
         msg = f"{ctx} matrix {i} {self.wl.shapes[i]}: " + ", ".join(
-            f"{k}={v:.3g}" for k, v in e.items() if k not in ("W_gpu", "W_pre", "W_pre_ref"))
+            f"{k}={v:.3g}" for k, v in e.items() if k not in arrays)
         assert e["M"] < TOL_STATS and e["l"] < TOL_STATS and e["r"] < TOL_STATS, msg
+        assert e["L"] < TOL_STATS and e["R"] < TOL_STATS, msg
         assert e["norm_mt"] < TOL_STATS, msg
         assert e["O"] < TOL_DIR and e["norm_o"] < TOL_DIR and e["norm_d"] < TOL_DIR, msg
         assert e["W"] < TOL_W and e["dW"] < TOL_DW, msg
         if self.variant == "malter":
             assert e["nu"] < 1e-4 and e["alpha"] < 1e-4, msg
         if self.w_dtypes[i] == "bf16":
-            # Rounding x and y to nearest bf16 moves them apart by at most
-            # |x - y| + one ulp, with x, y the GPU's and the oracle's
-            # pre-rounding values; and the stored W is the round-to-nearest-
-            # even of the GPU's own pre-rounding value (fp32 arithmetic decides
-            # a few near-ties).
-            Wr = self.W_ref[i]
-            diff = np.abs(e["W_gpu"] - Wr)
-            gap = np.abs(e["W_pre"] - e["W_pre_ref"])
-            ulp = bf16_ulp(np.maximum(np.abs(e["W_pre"]), np.abs(e["W_pre_ref"])))
-            assert np.all(diff <= gap * 1.001 + ulp * 1.0001), msg
-            own = ref.round_to_bf16(e["W_pre"])
-            assert np.mean(own != e["W_gpu"]) < 5e-3, msg + f", rne mismatch={np.mean(own != e['W_gpu']):.3g}"
+            # The stored bf16 W is the round-to-nearest-even of the GPU's own
+            # pre-rounding value, and equals the oracle's rounding wherever no
+            # rounding boundary lies between the two pre-rounding values.
+            assert e["own_mismatch"] == 0, msg
+            assert e["oracle_mismatch_off_boundary"] == 0, msg
+            # Where a boundary does lie between them the two roundings may
+            # differ.  That happens on a fraction of the entries set by the
+            # pre-rounding gap: at most the fraction the update tolerance
+            # allows, and at most 1 % at the paper's GPT-2 learning rates.
+            assert e["straddle"] <= e["straddle_allowed"] + 1e-3, msg
+            if self.wl.name.startswith("gpt2"):
+                assert e["straddle"] <= 0.01, msg
         return e
 
     def close(self):

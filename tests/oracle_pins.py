@@ -137,6 +137,41 @@ def check_ns_band(ref):
     assert 0.5 < np.median(S_out) < 1.3
 
 
+def check_ns_scalar_map_closed_forms(ref):
+    """The scalar map that Newton-Schulz applies to each normalised singular
+    value, against facts fixed by the polynomial p(x) = a x + b x^3 + c x^5
+    itself: p(0) = 0, p(1) = a + b + c, p is odd, p'(0) = a (so k steps scale
+    tiny inputs by a^k); and k steps equal the k-fold composition p(p(...)),
+    built as a polynomial by numpy.polynomial for k <= 2 and evaluated by its
+    polyval k times for k <= 6 (library routines working from the coefficient
+    vector), for the quintic, a second quintic and the cubic (1.5, -0.5, 0),
+    whose fixed point is 1."""
+    from numpy.polynomial import Polynomial
+    from numpy.polynomial.polynomial import polyval
+    for coeffs in (ref.DEFAULT_NS_COEFFS, (1.5, -0.5, 0.0), (2.0, -1.5, 0.5)):
+        a, b, c = coeffs
+        assert ref.ns_scalar_map(0.0, 1, coeffs) == 0.0
+        assert abs(ref.ns_scalar_map(1.0, 1, coeffs) - (a + b + c)) < 1e-15
+        xs = np.linspace(-1.2, 1.2, 241)
+        assert np.allclose(ref.ns_scalar_map(-xs, 3, coeffs), -ref.ns_scalar_map(xs, 3, coeffs),
+                           rtol=0, atol=1e-13)
+        tiny = 1e-9
+        for k in (1, 4):
+            assert abs(ref.ns_scalar_map(tiny, k, coeffs) / tiny - a ** k) < 1e-6 * a ** k
+        coef = [0.0, a, 0.0, b, 0.0, c]
+        xs = np.linspace(0.0, 1.1, 111)
+        # one and two steps: the composed polynomial itself (degree 5, 25)
+        p = Polynomial(coef)
+        assert np.allclose(ref.ns_scalar_map(xs, 1, coeffs), p(xs), rtol=1e-12, atol=1e-13)
+        assert np.allclose(ref.ns_scalar_map(xs, 2, coeffs), p(p)(xs), rtol=1e-9, atol=1e-10)
+        # more steps: the library's evaluation of p, applied k times
+        y = xs.copy()
+        for k in range(1, 7):
+            y = polyval(y, coef)
+            assert np.allclose(ref.ns_scalar_map(xs, k, coeffs), y, rtol=1e-12, atol=1e-13), (coeffs, k)
+    assert ref.ns_scalar_map(1.0, 7, (1.5, -0.5, 0.0)) == 1.0
+
+
 def check_cubic_ns_is_polar(ref):
     """With the cubic coefficients (1.5, -0.5, 0) and many steps Newton-Schulz
     converges to the polar factor U V^T (Section 3.1): compare with an SVD and
@@ -387,6 +422,7 @@ ALL_CHECKS = [
     check_preconditioner_root,
     check_two_sided_entrywise,
     check_ns_singular_value_map,
+    check_ns_scalar_map_closed_forms,
     check_ns_band,
     check_cubic_ns_is_polar,
     check_step_internals,

@@ -150,3 +150,32 @@ def test_header_is_plain_c_and_links_from_c(lib, tmp_path):
     out = subprocess.run([str(exe)], capture_output=True, text=True)
     assert out.returncode == 0, out
     assert out.stdout.strip() == "device pointer not 16-byte aligned"
+
+
+def test_noalloc_binding_checks_tensors_without_gpu():
+    """The binding refuses tensors whose shape, dtype, layout or device would
+    make the kernels index past them, before any pointer reaches the library."""
+    import torch
+    m, n = 16, 24
+
+    def t(*shape, dtype=torch.float32):
+        return torch.zeros(shape, dtype=dtype)
+
+    good = dict(G=t(m, n), M=t(m, n), l=t(m), r=t(n), L_out=t(m), R_out=t(n))
+    bad_cases = [
+        dict(G=t(m, n - 8)),                      # G shorter than M
+        dict(l=t(m - 8)),                         # row statistics too short
+        dict(R_out=t(n + 8)),                     # wrong length
+        dict(M=t(m, n, dtype=torch.bfloat16)),    # bf16 momentum
+        dict(G=t(m, n, dtype=torch.float16)),     # unsupported gradient type
+        dict(M=t(n, m).t()),                      # right shape, not contiguous
+        dict(M=t(m * n)),                         # not 2-D
+    ]
+    for case in bad_cases:
+        args = dict(good, **case)
+        with pytest.raises(ValueError):
+            malt.malt_stats_noalloc(args["G"], args["M"], args["l"], args["r"],
+                                    args["L_out"], args["R_out"])
+    # well-formed host tensors are refused too: the library takes device pointers
+    with pytest.raises(ValueError, match="CUDA"):
+        malt.malt_stats_noalloc(*good.values())

@@ -49,6 +49,15 @@ def test_reference_arm_prints_contract_line():
     assert line["impl"] == "reference" and line["value"] > 0
     assert line["cpu_baseline"]["kind"] == "oracle"
     assert line["e2e"]["h2d_bytes_per_step"] == 0
+    # one real step over the whole parameter set, reported as what ran
+    assert line["steps"] == 1 and line["requested"] == {"steps": 2, "warmup": 3}
+    assert abs(line["ms_per_step"] * line["value"] - 1e3) < 1e-6 * 1e3
+    # the same config keys as the GPU arm's line
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2608_05088_gb300 import inputs
+    want = dict(bench.workload_config(inputs.WORKLOADS["single_256x512"]), ns_schedule="auto")
+    assert line["config"] == json.loads(json.dumps(want))
 
 
 def test_reference_arm_nonzero_rank_is_silent():

@@ -54,20 +54,19 @@ def test_empty_parameter_list():
     opt.close()
 
 
-@pytest.mark.parametrize("schedule", ["auto", "fused"])
+@pytest.mark.parametrize("schedule", ["auto", "persistent"])
 def test_host_buffer_step_matches_device_step(schedule):
     """malt_step_host (gradients from pinned host memory, weights copied back)
     gives bitwise the same W, M, l, r as malt_step on the same gradients, and
-    the host copies of W equal the device W after every step (also when the
-    whole step is one fused launch, which reads G and writes W inside it)."""
+    the host copies of W equal the device W after every step."""
     import numpy as np
     import torch
     wl = inputs.Workload("hoststep", 42, ((256, 512), (392, 136), (520, 1544)), "bf16", 1.5, 0.02,
                          "malter", 3)
     a = Run(wl, check=[])
     b = Run(wl, check=[])
-    if schedule == "fused":
-        b.opt.set_ns_schedule(malt.MALT_NS_FUSED)
+    if schedule == "persistent":
+        b.opt.set_ns_schedule(malt.MALT_NS_PERSISTENT)
     g_host = [torch.empty(s, dtype=torch.float32).pin_memory() for s in wl.shapes]
     w_host = [torch.empty(s, dtype=torch.bfloat16).pin_memory() for s in wl.shapes]
     # alternate two device gradient sets, as a pipelining caller does

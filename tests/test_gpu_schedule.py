@@ -18,9 +18,7 @@ RAGGED = ((200, 328), (392, 136), (8, 8), (136, 1000), (520, 520), (64, 2056), (
 TEN_CLASSES = tuple((64 * (i + 1), 512) for i in range(8)) + ((520, 8), (16, 16))
 
 
-# (schedule, overlap groups): the fused step with automatic, one and three runs
-SCHEDULES = [(malt.MALT_NS_PHASED, 0), (malt.MALT_NS_PERSISTENT, 0), (malt.MALT_NS_FUSED, 0),
-             (malt.MALT_NS_FUSED, 1), (malt.MALT_NS_FUSED, 3)]
+SCHEDULES = [malt.MALT_NS_PHASED, malt.MALT_NS_PERSISTENT, malt.MALT_NS_AUTO]
 
 
 def run_both(wl, steps, w_dtypes=None, ns_coeffs=None, schedules=SCHEDULES, g_dtype="f32"):
@@ -30,13 +28,12 @@ def run_both(wl, steps, w_dtypes=None, ns_coeffs=None, schedules=SCHEDULES, g_dt
     if ns_coeffs is not None:
         kw["ns_coeffs"] = ns_coeffs
     out = []
-    for sched, groups in schedules:
+    for sched in schedules:
         run = Run(wl, check=[], w_dtypes=w_dtypes, **kw)
         run.opt.set_ns_schedule(sched)
-        run.opt.set_overlap_groups(groups)
         for _ in range(steps):
             run.step(oracle=False)
-        assert run.status() == malt.MALT_OK, (sched, groups, run.opt.timeout_site())
+        assert run.status() == malt.MALT_OK, (sched, run.opt.timeout_site())
         torch.cuda.synchronize()
         res = [run.host(t) for t in run.W + run.M + run.l + run.r]
         res += [run.host(run.opt.direction(i)) for i in range(len(wl.shapes))]
@@ -45,9 +42,9 @@ def run_both(wl, steps, w_dtypes=None, ns_coeffs=None, schedules=SCHEDULES, g_dt
         res += [np.asarray(nu), np.asarray([t])]
         out.append(res)
         run.close()
-    for (sched, groups), res in zip(schedules[1:], out[1:]):
+    for sched, res in zip(schedules[1:], out[1:]):
         for i, (a, b) in enumerate(zip(out[0], res)):
-            assert np.array_equal(a, b), (sched, groups, i)
+            assert np.array_equal(a, b), (sched, i)
 
 
 @pytest.mark.parametrize("variant", ["malt", "malter"])
@@ -81,30 +78,6 @@ def test_gpt2_large_layers_bitwise():
     run_both(wl, 2)
 
 
-@pytest.mark.parametrize("variant", ["malt", "malter", "muon"])
-def test_fused_against_oracle(variant):
-    """The whole step in one launch (statistics to apply on the GEMM
-    kernel's epilogue warps), against the oracle, 3 steps (the inputs of the
-    phased parity tests of tests/test_gpu_parity.py)."""
-    shapes = RAGGED[:6] if variant == "muon" else RAGGED
-    seed = 36 if variant == "muon" else 31
-    wl = inputs.Workload("fusedo", seed, shapes, "f32", 1.5, 0.02, variant, 3)
-    run = Run(wl, w_dtypes=["f32", "bf16"] * (len(shapes) // 2))
-    run.opt.set_ns_schedule(malt.MALT_NS_FUSED)
-    run.opt.set_overlap_groups(2)
-    for s in range(wl.steps):
-        run.step()
-        assert run.status() == malt.MALT_OK, run.opt.timeout_site()
-        for i in range(len(wl.shapes)):
-            run.assert_close(i, f"{variant} step {s}")
-    run.close()
-
-
-def test_fused_muon_bitwise():
-    wl = inputs.Workload("fusedmu", 56, RAGGED[:6], "f32", 1.5, 0.02, "muon", 2)
-    run_both(wl, 2)
-
-
 def test_persistent_against_oracle_two_groups():
     wl = inputs.Workload("sched10o", 53, TEN_CLASSES, "f32", 1.0, 0.02, "malter", 2)
     run = Run(wl)
@@ -117,11 +90,11 @@ def test_persistent_against_oracle_two_groups():
     run.close()
 
 
-@pytest.mark.parametrize("schedule", [malt.MALT_NS_PERSISTENT, malt.MALT_NS_FUSED])
+@pytest.mark.parametrize("schedule", [malt.MALT_NS_PERSISTENT, malt.MALT_NS_PHASED])
 def test_ns_steps_change_between_steps(schedule):
-    """One state stepped with ns_steps 5, 3, 5, 3: the persistent and fused
-    launches take a work table per value (built on first use, then kept), and
-    every step matches the oracle run with the same sequence."""
+    """One state stepped with ns_steps 5, 3, 5, 3: the persistent launches
+    claim the first k iterations' entries of the work table built at init,
+    and every step matches the oracle run with the same sequence."""
     import dataclasses
     wl = inputs.Workload("kswitch", 39, ((256, 512), (392, 136), (520, 520)), "f32", 1.0, 0.02,
                          "malter", 4)

@@ -3,16 +3,15 @@
 The library builds the tables the persistent launches claim from with the
 same code the GPU path uses (malt_ns_schedule needs no GPU).  The Orth step
 of Algorithm 1 iterates A = X X^T, B' = aI + bA + cA^2, X <- B' X on each
-matrix's own data, and the fused step chains the HBM-bound stages of each
-matrix around them (statistics, finalize, prescale, norms; scalars, apply),
-so for each table:
-  * every item of every stage of every matrix appears exactly once (all
-    256 x 256 tiles of a product, the upper triangle for the symmetric A and
-    B'; every block pair of a memory stage);
+matrix's own data, so for each table:
+  * every tile of every product of every matrix appears exactly once (all
+    256 x 256 tiles of B' X, the upper triangle for the symmetric A and B');
   * an item waits exactly for the previous stage of its own matrix, complete;
   * the table is topologically ordered: when an item is claimed, every item
     it waits for was claimed before it.  Claims happen only in running CTAs,
-    so this order is what makes the schedule deadlock-free.
+    so this order is what makes the schedule deadlock-free;
+  * the table of k iterations is the prefix of the table of any larger k (the
+    library builds the table once for 64 iterations and launches k of them).
 """
 import numpy as np
 import pytest
@@ -20,7 +19,6 @@ import pytest
 from paper_2608_05088_gb300 import build, inputs
 
 SIGNALS_PER_ITEM = 16   # epilogue warps of a CTA pair
-STATS, FINALIZE, PRESCALE, NORMS, SCALARS, APPLY = 3, 4, 5, 6, 7, 8
 
 
 @pytest.fixture(scope="module")
@@ -39,25 +37,13 @@ def expected_items(rows, cols, kind):
     tp, tq = cdiv(p, 256), cdiv(q, 256)
     if kind == 2:
         return tp * tq
-    if kind in (0, 1):
-        return tp * (tp + 1) // 2
-    if kind == STATS:
-        return cdiv(cdiv(rows, 64) * cdiv(cols, 256), 2)
-    if kind == PRESCALE:
-        return cdiv(cdiv(rows, 64) * cdiv(cols, 256), 2)
-    if kind == APPLY:                   # 16384-element runs (O is in W's layout)
-        return cdiv(cdiv(rows * cols, 16384), 2)
-    return 1
+    assert kind in (0, 1)
+    return tp * (tp + 1) // 2
 
 
-def stage_kinds(k, fused):
-    kinds = [0, 1, 2] * k
-    return [STATS, FINALIZE, PRESCALE, NORMS] + kinds + [SCALARS, APPLY] if fused else kinds
-
-
-def check_table(tab, shapes, k, fused):
+def check_table(tab, shapes, k):
     n = len(shapes)
-    kinds = stage_kinds(k, fused)
+    kinds = [0, 1, 2] * k
     seen = {}
     for grp, st, kind, mat, local, dep, target, nitems in tab:
         assert kind == kinds[st]
@@ -90,21 +76,27 @@ RAGGED = [(200, 328), (392, 136), (8, 8), (136, 1000), (520, 520), (64, 2056), (
           (256, 512)]
 
 
-@pytest.mark.parametrize("k", [1, 2, 5])
+@pytest.mark.parametrize("k", [1, 2, 5, 64])
 def test_products_ragged(malt, k):
-    check_table(malt.malt_ns_schedule(RAGGED, k), RAGGED, k, False)
+    check_table(malt.malt_ns_schedule(RAGGED, k), RAGGED, k)
 
 
-@pytest.mark.parametrize("groups", [0, 1, 2, 3, 8])
-def test_fused_ragged(malt, groups):
-    tab = malt.malt_ns_schedule(RAGGED, 3, fused=True, overlap_groups=groups)
-    check_table(tab, RAGGED, 3, True)
+def test_shorter_tables_are_prefixes(malt):
+    """The library uploads one table for 64 iterations at init and launches
+    the first k iterations' entries of it."""
+    full = malt.malt_ns_schedule(RAGGED, 64)
+    for k in (1, 3, 5, 17):
+        tab = malt.malt_ns_schedule(RAGGED, k)
+        for grp in np.unique(full[:, 0]):
+            a, b = tab[tab[:, 0] == grp], full[full[:, 0] == grp]
+            assert np.array_equal(a, b[: len(a)])
+            assert len(b) == 64 * len(a) // k
 
 
 def test_gpt2_large(malt):
     shapes = list(inputs.WORKLOADS["gpt2_large"].shapes)
     tab = malt.malt_ns_schedule(shapes, 5)
-    check_table(tab, shapes, 5, False)
+    check_table(tab, shapes, 5)
     # 36 of each of 1280x3840, 1280^2, 1280x5120, 5120x1280 (frames 1280 x
     # {3840, 1280, 5120, 5120}): 15 upper tiles per Gram / Poly, 5 x q/256 per BX
     per_iter = 144 * 15 * 2 + 36 * (5 * 15 + 5 * 5 + 2 * 5 * 20)
@@ -114,25 +106,12 @@ def test_gpt2_large(malt):
     assert all(max(shapes[m]) == 5120 for m in first[:, 3])
 
 
-def test_gpt2_large_fused(malt):
-    shapes = list(inputs.WORKLOADS["gpt2_large"].shapes)
-    tab = malt.malt_ns_schedule(shapes, 5, fused=True)
-    check_table(tab, shapes, 5, True)
-    # the memory stages of later runs are interleaved with earlier products
-    kinds = tab[:, 2]
-    first_product = int(np.argmax(kinds <= 2))
-    last_product = len(kinds) - 1 - int(np.argmax(kinds[::-1] <= 2))
-    inside = kinds[first_product:last_product]
-    assert np.sum(inside > 2) > 0.5 * np.sum(kinds > 2)
-
-
 def test_more_classes_than_one_launch(malt):
     # ten distinct NS frames: two launch groups (at most eight classes each)
     shapes = [(64 * (i + 1), 512) for i in range(8)] + [(520, 8), (16, 16)]
-    for fused in (False, True):
-        tab = malt.malt_ns_schedule(shapes, 3, fused=fused)
-        assert set(np.unique(tab[:, 0]).tolist()) == {0, 1}
-        check_table(tab, shapes, 3, fused)
+    tab = malt.malt_ns_schedule(shapes, 3)
+    assert set(np.unique(tab[:, 0]).tolist()) == {0, 1}
+    check_table(tab, shapes, 3)
 
 
 def test_bad_arguments(malt):
@@ -142,5 +121,3 @@ def test_bad_arguments(malt):
         malt.malt_ns_schedule([(256, 512)], 65)
     with pytest.raises(malt.MaltError):
         malt.malt_ns_schedule([(250, 512)], 5)
-    with pytest.raises(malt.MaltError):
-        malt.malt_ns_schedule([(256, 512)], 5, fused=True, overlap_groups=65)

@@ -44,6 +44,10 @@ MUTATIONS = {
                           "(1.0 + hp.lr * hp.weight_decay) * W if"),
     "weight_decay_after_update": ("W_new = W_decayed - delta",
                                   "W_new = (1.0 - hp.lr * hp.weight_decay) * (W - delta)"),
+    "ns_scalar_map_wrong_power": ("x = a * x + b * x ** 3 + c * x ** 5",
+                                  "x = a * x + b * x ** 3 + c * x ** 4"),
+    "ns_scalar_map_coeffs_swapped": ("x = a * x + b * x ** 3 + c * x ** 5",
+                                     "x = a * x + c * x ** 3 + b * x ** 5"),
     "graft_uses_normD_twice": ("scale = hp.lr * norm_O / (norm_D + hp.eps)",
                                "scale = hp.lr * norm_D / (norm_D + hp.eps)"),
 }
