@@ -202,10 +202,12 @@ class Run:
             assert e["oracle_mismatch_off_boundary"] == 0, msg
             # Where a boundary does lie between them the two roundings may
             # differ.  That happens on a fraction of the entries set by the
-            # pre-rounding gap: at most the fraction the update tolerance
-            # allows, and at most 1 % at the paper's GPT-2 learning rates.
+            # pre-rounding gap, which grows with the update (so with the
+            # learning rate): at most the fraction the update tolerance
+            # allows, and at most 1 % for the GPT-2 sets at the paper's MALT
+            # learning rates (MALTER's tuned rates are ten times larger).
             assert e["straddle"] <= e["straddle_allowed"] + 1e-3, msg
-            if self.wl.name.startswith("gpt2"):
+            if self.wl.name.startswith("gpt2") and self.variant == "malt":
                 assert e["straddle"] <= 0.01, msg
         return e
 
