@@ -17,6 +17,7 @@ timed region).  Prints one JSON line on rank 0.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import math
@@ -400,6 +401,98 @@ def run_stress_sweep(args):
                 torch.cuda.empty_cache()
 
 
+# ----------------------------------------------------------- whole optimizer
+ADAMW_BYTES_PER_ELEM = 30.0     # g 4, w 4+4, m 4+4, v 4+4, bf16 copy 2
+
+
+def run_whole_optimizer_leg(args, wl, G, dev, stream):
+    """The whole optimizer step of the model (Section 5.1 parameter grouping):
+    MALT on the 2-D matrices with fp32 master weights, their bf16 copies and
+    decoupled weight decay 0.1 (appendix table), plus AdamW on the other
+    tensors (embeddings, tied head, LayerNorms, biases) at the AdamW learning
+    rate, both on one stream.  The matrices read the timed workload's
+    gradients G.  Reports ms per whole step, the AdamW launch's own time and
+    HBM rate, and the apply pass (which now also writes the copies)."""
+    import torch
+    import paper_2608_05088_gb300.malt as malt
+    from paper_2608_05088_gb300 import inputs
+    base = wl.name.split("_first")[0]
+    if base not in inputs.ADAMW_SETS:
+        return None
+    aset = inputs.ADAMW_SETS[base]
+    W = [torch.from_numpy(w).to(dev) for w in inputs.initial_weights(
+        dataclasses.replace(wl, weight_dtype="f32"))]
+    copies = [torch.empty(s_, dtype=torch.bfloat16, device=dev) for s_ in wl.shapes]
+    M = [torch.empty(s_, dtype=torch.float32, device=dev) for s_ in wl.shapes]
+    l = [torch.empty(s_[0], dtype=torch.float32, device=dev) for s_ in wl.shapes]
+    r = [torch.empty(s_[1], dtype=torch.float32, device=dev) for s_ in wl.shapes]
+    others = []
+    for i, (_, shape, wd) in enumerate(aset.tensors):
+        w = torch.from_numpy(inputs.adamw_initial(aset, i)).to(dev)
+        others.append((w, torch.empty(shape, dtype=torch.bfloat16, device=dev),
+                       torch.from_numpy(inputs.adamw_gradient(aset, i, 0)).to(dev),
+                       torch.empty(shape, dtype=torch.float32, device=dev),
+                       torch.empty(shape, dtype=torch.float32, device=dev), wd))
+    whole = malt.WholeOptimizer(list(zip(W, G, M, l, r)), others, copies=copies)
+    hp = malt.hparams(lr=wl.lr, ns_steps=wl.ns_steps, weight_decay=0.1)
+    ahp = malt.adamw_hparams(lr=aset.lr)
+    malter = wl.variant == "malter"
+    for _ in range(args.warmup):
+        whole.step(hp, ahp, malter=malter)
+    torch.cuda.synchronize()
+    if whole.check() != malt.MALT_OK:
+        raise SystemExit("whole-optimizer warm-up step failed")
+    barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        whole.step(hp, ahp, malter=malter)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    t_whole = max_over_ranks(e0.elapsed_time(e1), dev) / args.steps
+    # the AdamW launches alone, and the MALT apply pass, from their own events
+    whole.malt.profile(True)
+    whole.malt.profile_read()
+    a0 = torch.cuda.Event(enable_timing=True)
+    a1 = torch.cuda.Event(enable_timing=True)
+    t_adam = 0.0
+    for _ in range(args.steps):
+        whole.malt.step(hp, malter=malter)
+        a0.record(stream)
+        whole.adamw.step(ahp)
+        a1.record(stream)
+        torch.cuda.synchronize()
+        t_adam += a0.elapsed_time(a1)
+    prof = whole.malt.profile_read()
+    whole.malt.profile(False)
+    if whole.check() != malt.MALT_OK:
+        raise SystemExit("whole-optimizer step failed")
+    t_adam /= args.steps
+    pk, pk_src = peaks()
+    gbs = ADAMW_BYTES_PER_ELEM * aset.elements / (t_adam / 1e3) / 1e9
+    apply_ms = prof["apply"][0] / args.steps
+    apply_bpe = 4.0 + 4.0 + 2.0 + 2.0            # W fp32 read+write, O read, copy write
+    out = {"ms_per_step": t_whole, "value": world_size() / (t_whole / 1e3), "unit": UNIT,
+           "matrices": len(wl.shapes), "matrix_elements": wl.elements,
+           "adamw_tensors": len(aset.tensors), "adamw_elements": aset.elements,
+           "parameters": wl.elements + aset.elements,
+           "malt": f"{wl.variant}, fp32 master weights with bf16 copies, weight decay 0.1, lr {wl.lr}",
+           "adamw": f"betas (0.9, 0.95), eps 1e-8, lr {aset.lr}, weight decay 0.1 on the "
+                    f"embeddings, 0 on vectors, bf16 copies",
+           "adamw_kernel": {"ms_per_step": t_adam, "bytes_per_elem": ADAMW_BYTES_PER_ELEM,
+                            "achieved_gbs": gbs, "frac_of_hbm": gbs / float(pk["hbm_gbs"])},
+           "apply_with_copies": {"ms_per_step": apply_ms, "bytes_per_elem": apply_bpe,
+                                 "achieved_gbs": apply_bpe * wl.elements / (apply_ms / 1e3) / 1e9},
+           "peaks": pk_src}
+    whole.close()
+    return out
+
+
+def world_size():
+    return rank_env()[1]
+
+
 # --------------------------------------------------------------------- MALT
 def run_malt(args):
     import numpy as np
@@ -545,6 +638,11 @@ def run_malt(args):
         if opt.check() != malt.MALT_OK:
             raise SystemExit("muon step failed")
 
+    # ---- the whole optimizer (MALT on the matrices + AdamW on the rest)
+    whole = None
+    if not args.no_whole:
+        whole = run_whole_optimizer_leg(args, wl, G, dev, stream)
+
     # ---- end to end through the C ABI with host buffers (malt_step_host):
     # every step copies all gradients in from pinned host memory and all
     # updated weights back out; the library overlaps those copies with the
@@ -640,6 +738,7 @@ def run_malt(args):
            "clocks": clk, "e2e": e2e, "gpu_launches": launches, "roofline": roofline,
            "hbm_kernels": mem, "ms_per_step_by_kernel": breakdown,
            "cpu_baseline": cpu, "muon_same_engine": muon, "ns_schedules": sched,
+           "whole_optimizer": whole,
            "cuda_graph": graph_leg, "workspace_bytes": opt.workspace_bytes()}
     print(json.dumps(out), flush=True)
     opt.close()
@@ -655,6 +754,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-muon", action="store_true")
+    ap.add_argument("--no-whole", action="store_true",
+                    help="skip the whole-optimizer leg (MALT + AdamW on every parameter)")
     ap.add_argument("--no-graph", action="store_true",
                     help="skip the CUDA-graph replay of the timed step")
     ap.add_argument("--ns-schedule", choices=("auto", "phased", "persistent"),

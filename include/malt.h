@@ -305,6 +305,75 @@ int malt_stats_noalloc(const void* g, int32_t g_dtype, float* m, float* l, float
                        float* L_out, float* R_out, int64_t rows, int64_t cols,
                        float mu1, float mu2, float eps, void* stream);
 
+/* Whole-optimizer step, 2-D matrices: register bf16 copies of fp32 master
+ * weights.  copies[i] is a caller-owned device buffer of rows x cols bf16
+ * (16-byte aligned) that every later step's weight update fills with the
+ * round-to-nearest-even of the updated fp32 W of parameter i (the weights a
+ * bf16 model computes with), or NULL for none; copies = NULL clears all.
+ * Only parameters with w_dtype MALT_F32 may have a copy
+ * (MALT_ERR_UNSUPPORTED otherwise).  n must equal the state's parameter
+ * count.  Takes effect at the next step. */
+int malt_set_weight_copies(malt_state_t* st, void* const* copies, int32_t n);
+
+/* ---- Whole-optimizer step: AdamW for the other parameters --------------
+ * The paper updates only the 2-D weight matrices with MALT / MALTER and hands
+ * the vectors, scalars, embeddings and output head to AdamW (Section 5.1,
+ * parameter grouping; appendix table: betas (0.9, 0.95), weight decay 0.1).
+ * Per tensor at step t (1-based, counted on the device):
+ *   m <- beta1 m + (1 - beta1) g,  v <- beta2 v + (1 - beta2) g^2,
+ *   w <- (1 - lr wd) w - lr (m / (1 - beta1^t)) / (sqrt(v / (1 - beta2^t)) + eps),
+ * decoupled weight decay wd per tensor.  One grouped streaming launch (plus
+ * a pointer-binding launch) covers every tensor.  A whole-optimizer step is
+ * malt_step (or malter_step) on the matrices and malt_adamw_step on the rest,
+ * enqueued on the same stream. */
+typedef struct {
+    float*       w;             /* fp32 master weights, numel, updated in place     */
+    void*        w_copy;        /* bf16 copy of the updated w (numel), or NULL      */
+    const void*  g;             /* gradient, numel, MALT_F32 or MALT_BF16, read only */
+    int32_t      g_dtype;
+    float*       m;             /* first moment, numel fp32, in place               */
+    float*       v;             /* second moment, numel fp32, in place              */
+    int64_t      numel;         /* elements (any positive count)                   */
+    float        weight_decay;  /* decoupled decay of this tensor (0 for none)      */
+} malt_adamw_param_t;
+/* All pointers are caller-owned DEVICE pointers, 16-byte aligned, not
+ * overlapping one another or another tensor's. */
+
+typedef struct {
+    float lr;      /* learning rate                                     */
+    float beta1;   /* first-moment EMA, 0 <= beta1 < 1 (table: 0.9)      */
+    float beta2;   /* second-moment EMA, 0 <= beta2 < 1 (table: 0.95)    */
+    float eps;     /* added to sqrt(v_hat), >= 0 (1e-8 suggested)        */
+} malt_adamw_hparams_t;
+
+/* Opaque: the tensor table, block-prefix table and step counter t. */
+typedef struct malt_adamw_state malt_adamw_state_t;
+
+/* Plan the launches for these n tensors (sizes and gradient types fixed from
+ * here on), allocate the small state on the current device and zero m and v
+ * of every tensor on `stream` (m_0 = v_0 = 0, t = 0).  n = 0 is allowed.
+ * Errors: MALT_ERR_INVALID_ARG (null pointer, n < 0, NaN decay),
+ * MALT_ERR_UNSUPPORTED (numel <= 0, bad g_dtype), MALT_ERR_MISALIGNED,
+ * MALT_ERR_OUT_OF_MEMORY; on failure *out is NULL. */
+int malt_adamw_init_state(malt_adamw_state_t** out, const malt_adamw_param_t* params, int32_t n,
+                          void* stream);
+
+/* One AdamW step of all n tensors, enqueued on `stream` (no host
+ * synchronisation).  The tensors must have the sizes and gradient types of
+ * init, in the same order (MALT_ERR_SHAPE_CHANGED); pointers, w_copy and
+ * weight_decay may change.  MALT_ERR_INVALID_ARG for hyperparameters out of
+ * range. */
+int malt_adamw_step(malt_adamw_state_t* st, const malt_adamw_param_t* params, int32_t n,
+                    const malt_adamw_hparams_t* hp, void* stream);
+
+/* Checkpoint support: read or set the step counter t (both synchronise with
+ * the stream of the state's last call).  m, v and w are caller-owned. */
+int malt_adamw_get_step(malt_adamw_state_t* st, int64_t* t_host);
+int malt_adamw_set_step(malt_adamw_state_t* st, int64_t t_host);
+
+/* Free the state (synchronises with its last stream first). */
+void malt_adamw_destroy_state(malt_adamw_state_t* st);
+
 /* Bytes of device workspace the state holds. */
 size_t malt_workspace_bytes(const malt_state_t* st);
 

@@ -12,10 +12,12 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(OUT_DIR, "libmalt.so")
-SOURCES = ["stream_kernels.cu", "ns_gemm.cu", "malt_api.cu", "noalloc.cu"]
+SOURCES = ["stream_kernels.cu", "ns_gemm.cu", "malt_api.cu", "noalloc.cu", "adamw.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
+# Host code is compiled without floating-point contraction, so the few
+# scalars it derives (decay factors) round the same on x86 and Arm hosts.
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
-         "-Xcompiler", "-fno-strict-aliasing"]
+         "-Xcompiler", "-fno-strict-aliasing", "-Xcompiler", "-ffp-contract=off"]
 
 
 def nvcc() -> str:

@@ -46,6 +46,7 @@ struct UserPtrs {
     float* m;
     float* l;
     float* r;
+    void* wcopy;    // bf16 copy of an fp32 W written by the apply pass, or null
 };
 
 // Static per-matrix description, built at init and kept on the device.

@@ -112,6 +112,7 @@ struct malt_state {
     int nmat = 0;
     int num_sms = 0;
     std::vector<malt_param_t> shape0;      // shapes / dtypes fixed at init
+    std::vector<void*> wcopy;              // bf16 copies of fp32 weights (malt_set_weight_copies)
     std::vector<MatDesc> hmats;
     std::vector<ShapeClass> classes;
     void* ws = nullptr;
@@ -385,6 +386,7 @@ int32_t table_per_iter(const NsParams& G) { return 2 * G.sym_items + G.full_item
 int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
     st->nmat = n;
     st->shape0.assign(params, params + n);
+    st->wcopy.assign(n, nullptr);
     build_classes(params, n, st->hmats, st->classes);
 
     // Workspace layout.
@@ -560,7 +562,7 @@ int bind_pointers(malt_state* st, const malt_param_t* params, cudaStream_t s) {
         bp.offset = off;
         for (int i = 0; i < cnt; ++i) {
             const malt_param_t& p = params[off + i];
-            bp.p[i] = UserPtrs{p.w, p.g, p.m, p.l, p.r};
+            bp.p[i] = UserPtrs{p.w, p.g, p.m, p.l, p.r, st->wcopy[off + i]};
         }
         LaunchScope ls(st, MALT_KIND_BIND, s);
         MALT_CUDA(launch_bind(bp, st->d_ptrs, s), "bind_kernel");
@@ -1008,6 +1010,17 @@ size_t malt_workspace_bytes(const malt_state_t* st) { return st == nullptr ? 0 :
 int malt_debug_timeout_site(const malt_state_t* st, int32_t* out5) {
     if (st == nullptr || out5 == nullptr) return MALT_ERR_INVALID_ARG;
     std::memcpy(out5, st->last_timeout, sizeof(st->last_timeout));
+    return MALT_OK;
+}
+
+int malt_set_weight_copies(malt_state_t* st, void* const* copies, int32_t n) {
+    if (st == nullptr || n != st->nmat) return MALT_ERR_INVALID_ARG;
+    for (int i = 0; copies != nullptr && i < n; ++i) {
+        if (copies[i] == nullptr) continue;
+        if (st->shape0[i].w_dtype != MALT_F32) return MALT_ERR_UNSUPPORTED;
+        if (!aligned16(copies[i])) return MALT_ERR_MISALIGNED;
+    }
+    for (int i = 0; i < n; ++i) st->wcopy[i] = copies != nullptr ? copies[i] : nullptr;
     return MALT_OK;
 }
 

@@ -143,7 +143,7 @@ extern "C" int malt_stats_noalloc(const void* g, int32_t g_dtype, float* m, floa
     d.colpart = scratch + row_floats;
     d.L = L_out;
     d.R = R_out;
-    const UserPtrs up{nullptr, g, m, l, r};
+    const UserPtrs up{nullptr, g, m, l, r, nullptr};
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     noalloc_stats_kernel<<<static_cast<unsigned>(cb_count * rb_count), 256, 0, s>>>(d, up, mu1);
     cudaError_t e = cudaGetLastError();

@@ -18,7 +18,8 @@
 //   scalars   ||O||_F, ||D||_F, MALTER's nu and alpha (Section 3.5) and the
 //             grafted scale lr * alpha * ||O|| / (||D|| + eps) per matrix.
 //   apply     W <- (1 - lr wd) W - scale * L O R (Algorithm 1, W_t line), with
-//             O in W's layout, streamed contiguously.
+//             O in W's layout, streamed contiguously; for fp32 master weights
+//             also their bf16 copy, when the caller registered one.
 #pragma once
 #include <cuda_bf16.h>
 #include <cstdint>
@@ -506,6 +507,9 @@ __device__ __forceinline__ void apply8(const MatDesc& d, const UserPtrs& up, boo
         float4* wp = reinterpret_cast<float4*>(static_cast<float*>(up.w) + e);
         wp[0] = make_float4(w[0], w[1], w[2], w[3]);
         wp[1] = make_float4(w[4], w[5], w[6], w[7]);
+        // fp32 master weights: the bf16 copy the model computes with
+        if (up.wcopy != nullptr)
+            *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(up.wcopy) + e) = pack8_bf16(w);
     }
 }
 

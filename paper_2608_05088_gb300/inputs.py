@@ -173,6 +173,81 @@ def initial_weights(wl: Workload, indices=None, workers: int = 8):
         return list(ex.map(lambda i: initial_weight(wl, i), idxs))
 
 
+# ---------------------------------------------------------------------------
+# The rest of a GPT-2 model: the tensors AdamW updates in the paper's
+# parameter grouping (Section 5.1: vectors, scalars, embeddings, output head).
+# NanoGPT's layout: token embedding with its padded vocabulary of 50304 rows,
+# tied with the output head (one tensor); position embedding over the block
+# size 1024; per layer the two LayerNorms' gains and biases and the four
+# Linear biases; the final LayerNorm.  Weight decay (appendix table: 0.1)
+# goes to the 2-D tensors and not to the vectors, NanoGPT's convention.
+# Learning rates: the AdamW column of the Section 5.1 table.
+# ---------------------------------------------------------------------------
+GPT2_VOCAB = 50304
+GPT2_BLOCK = 1024
+_TAG_ADAM_SCALES, _TAG_ADAM_GRAD, _TAG_ADAM_INIT = 5, 6, 7
+
+
+@dataclasses.dataclass(frozen=True)
+class AdamWSet:
+    name: str
+    wid: int                     # seed component
+    tensors: tuple               # ((name, shape, weight_decay), ...)
+    lr: float
+    steps: int
+    sigma: float = 1.5
+
+    @property
+    def elements(self) -> int:
+        return int(sum(int(np.prod(shape)) for _, shape, _ in self.tensors))
+
+
+def _gpt2_adamw(layers, d):
+    t = [("wte", (GPT2_VOCAB, d), 0.1), ("wpe", (GPT2_BLOCK, d), 0.1)]
+    for i in range(layers):
+        t += [(f"h{i}.ln_1.weight", (d,), 0.0), (f"h{i}.ln_1.bias", (d,), 0.0),
+              (f"h{i}.attn.c_attn.bias", (3 * d,), 0.0), (f"h{i}.attn.c_proj.bias", (d,), 0.0),
+              (f"h{i}.ln_2.weight", (d,), 0.0), (f"h{i}.ln_2.bias", (d,), 0.0),
+              (f"h{i}.mlp.c_fc.bias", (4 * d,), 0.0), (f"h{i}.mlp.c_proj.bias", (d,), 0.0)]
+    t += [("ln_f.weight", (d,), 0.0), ("ln_f.bias", (d,), 0.0)]
+    return tuple(t)
+
+
+ADAMW_SETS = {
+    "gpt2_small": AdamWSet("gpt2_small_adamw", 12, _gpt2_adamw(12, 768), 0.0013, 10),
+    "gpt2_medium": AdamWSet("gpt2_medium_adamw", 13, _gpt2_adamw(24, 1024), 0.0009, 10),
+    "gpt2_large": AdamWSet("gpt2_large_adamw", 14, _gpt2_adamw(36, 1280), 0.0009, 10),
+}
+
+
+def adamw_initial(aset: AdamWSet, idx: int) -> np.ndarray:
+    """Initial value of tensor idx (fp32): embeddings ~ N(0, 0.02^2), LayerNorm
+    gains 1, biases 0 (the GPT-2 / NanoGPT initialisation)."""
+    name, shape, _ = aset.tensors[idx]
+    if len(shape) == 2:
+        w = _rng(aset.wid, idx, 0, _TAG_ADAM_INIT).standard_normal(shape, dtype=np.float32)
+        w *= np.float32(0.02)
+        return w
+    if name.endswith("ln_1.weight") or name.endswith("ln_2.weight") or name == "ln_f.weight":
+        return np.ones(shape, dtype=np.float32)
+    return np.zeros(shape, dtype=np.float32)
+
+
+def adamw_gradient(aset: AdamWSet, idx: int, step: int) -> np.ndarray:
+    """fp32 gradient of tensor idx at step (0-based): z times log-normal
+    scales drawn once per tensor (per row and column for the embeddings, per
+    entry for a vector)."""
+    _, shape, _ = aset.tensors[idx]
+    srng = _rng(aset.wid, idx, -1, _TAG_ADAM_SCALES)
+    z = _rng(aset.wid, idx, step, _TAG_ADAM_GRAD).standard_normal(shape, dtype=np.float32)
+    if len(shape) == 2:
+        z *= np.exp(aset.sigma * srng.standard_normal(shape[0])).astype(np.float32)[:, None]
+        z *= np.exp(aset.sigma * srng.standard_normal(shape[1])).astype(np.float32)[None, :]
+    else:
+        z *= np.exp(aset.sigma * srng.standard_normal(shape)).astype(np.float32)
+    return z
+
+
 def toy_quadratic_problem(kappa: float, n: int = 50, r: int = 5, seed: int = 0):
     """(A, B, C) of the matrix quadratic regression min_X 1/2 ||A X B^T - C||_F^2
     (Appendix B): C = U* S* V*^T of rank r with orthonormal U*, V* (n x r) and a

@@ -32,7 +32,9 @@ EXPORTS = ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
            "malt_debug_wait_timeout", "malt_profile_enable", "malt_profile_read",
            "malt_workspace_bytes", "malt_status_string", "malt_destroy_state",
            "malt_stats_noalloc", "malt_step_host", "muon_step", "malt_set_ns_schedule",
-           "malt_ns_schedule", "malt_debug_timeout_site", "malt_debug_precond")
+           "malt_ns_schedule", "malt_debug_timeout_site", "malt_debug_precond",
+           "malt_set_weight_copies", "malt_adamw_init_state", "malt_adamw_step",
+           "malt_adamw_get_step", "malt_adamw_set_step", "malt_adamw_destroy_state")
 NOALLOC_SCRATCH_FLOATS = 1048576
 KIND_NAMES = ("bind", "stats", "finalize", "prescale", "norms", "ns_gram", "ns_poly", "ns_bx",
               "scalars", "apply", "ns_persistent")
@@ -57,6 +59,17 @@ class malt_hparams_t(ctypes.Structure):
                 ("eps", ctypes.c_float), ("weight_decay", ctypes.c_float),
                 ("ns_steps", ctypes.c_int32), ("ns_a", ctypes.c_float),
                 ("ns_b", ctypes.c_float), ("ns_c", ctypes.c_float), ("ns_eps", ctypes.c_float)]
+
+
+class malt_adamw_param_t(ctypes.Structure):
+    _fields_ = [("w", ctypes.c_void_p), ("w_copy", ctypes.c_void_p), ("g", ctypes.c_void_p),
+                ("g_dtype", ctypes.c_int32), ("m", ctypes.c_void_p), ("v", ctypes.c_void_p),
+                ("numel", ctypes.c_int64), ("weight_decay", ctypes.c_float)]
+
+
+class malt_adamw_hparams_t(ctypes.Structure):
+    _fields_ = [("lr", ctypes.c_float), ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
+                ("eps", ctypes.c_float)]
 
 
 class MaltError(RuntimeError):
@@ -117,6 +130,18 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.malt_set_ns_schedule.argtypes = [vp, i32]
     lib.malt_set_ns_schedule.restype = ctypes.c_int
     lib.malt_ns_schedule.argtypes = [P(malt_param_t), i32, i32, P(i32), i64, P(i64)]
+    lib.malt_set_weight_copies.argtypes = [vp, P(vp), i32]
+    lib.malt_set_weight_copies.restype = ctypes.c_int
+    lib.malt_adamw_init_state.argtypes = [P(vp), P(malt_adamw_param_t), i32, vp]
+    lib.malt_adamw_init_state.restype = ctypes.c_int
+    lib.malt_adamw_step.argtypes = [vp, P(malt_adamw_param_t), i32, P(malt_adamw_hparams_t), vp]
+    lib.malt_adamw_step.restype = ctypes.c_int
+    lib.malt_adamw_get_step.argtypes = [vp, P(i64)]
+    lib.malt_adamw_get_step.restype = ctypes.c_int
+    lib.malt_adamw_set_step.argtypes = [vp, i64]
+    lib.malt_adamw_set_step.restype = ctypes.c_int
+    lib.malt_adamw_destroy_state.argtypes = [vp]
+    lib.malt_adamw_destroy_state.restype = None
     lib.malt_ns_schedule.restype = ctypes.c_int
     for name in ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
                  "malt_set_scalars", "malt_check", "malt_debug_direction",
@@ -305,6 +330,72 @@ def malt_stats_noalloc(G, M, l, r, L_out, R_out, mu1=0.95, mu2=0.99, eps=1e-8, s
         rows, cols, mu1, mu2, eps, _stream_handle(stream))
 
 
+def malt_set_weight_copies(st, copies, n: int):
+    """copies: one bf16 CUDA tensor (the shape of its fp32 W) or None for each
+    of the state's n parameters, or None to clear all."""
+    if copies is None:
+        _check(load().malt_set_weight_copies(st, None, n), "malt_set_weight_copies")
+        return
+    for c in copies:
+        if c is not None and (not c.is_contiguous() or _dtype_code(c) != MALT_BF16):
+            raise ValueError("weight copies must be contiguous bf16 tensors")
+    arr = (ctypes.c_void_p * max(len(copies), 1))(
+        *[None if c is None else c.data_ptr() for c in copies])
+    _check(load().malt_set_weight_copies(st, arr, len(copies)), "malt_set_weight_copies")
+
+
+def adamw_hparams(lr=1e-3, betas=(0.9, 0.95), eps=1e-8) -> malt_adamw_hparams_t:
+    return malt_adamw_hparams_t(lr, betas[0], betas[1], eps)
+
+
+def adamw_params_array(params):
+    """params: sequence of (w, w_copy or None, g, m, v, weight_decay) CUDA
+    tensors (w, m, v fp32; w_copy bf16) -> ctypes array."""
+    arr = (malt_adamw_param_t * max(len(params), 1))()
+    for i, (w, wc, g, m, v, wd) in enumerate(params):
+        for t in (w, g, m, v) + (() if wc is None else (wc,)):
+            if not t.is_contiguous():
+                raise ValueError("all tensors must be contiguous")
+        n = w.numel()
+        if any(t.numel() != n for t in (g, m, v)) or (wc is not None and wc.numel() != n):
+            raise ValueError("w, w_copy, g, m and v must have the same number of elements")
+        import torch
+        if w.dtype != torch.float32 or m.dtype != torch.float32 or v.dtype != torch.float32:
+            raise ValueError("w, m and v must be float32")
+        if wc is not None and wc.dtype != torch.bfloat16:
+            raise ValueError("w_copy must be bfloat16")
+        arr[i] = malt_adamw_param_t(w.data_ptr(), None if wc is None else wc.data_ptr(),
+                                    g.data_ptr(), _dtype_code(g), m.data_ptr(), v.data_ptr(),
+                                    n, float(wd))
+    return arr
+
+
+def malt_adamw_init_state(params, stream=None) -> ctypes.c_void_p:
+    st = ctypes.c_void_p()
+    _check(load().malt_adamw_init_state(ctypes.byref(st), adamw_params_array(params), len(params),
+                                        _stream_handle(stream)), "malt_adamw_init_state")
+    return st
+
+
+def malt_adamw_step(st, params, hp: malt_adamw_hparams_t, stream=None):
+    _check(load().malt_adamw_step(st, adamw_params_array(params), len(params), ctypes.byref(hp),
+                                  _stream_handle(stream)), "malt_adamw_step")
+
+
+def malt_adamw_get_step(st) -> int:
+    t = ctypes.c_int64()
+    _check(load().malt_adamw_get_step(st, ctypes.byref(t)), "malt_adamw_get_step")
+    return int(t.value)
+
+
+def malt_adamw_set_step(st, t: int):
+    _check(load().malt_adamw_set_step(st, int(t)), "malt_adamw_set_step")
+
+
+def malt_adamw_destroy_state(st):
+    load().malt_adamw_destroy_state(st)
+
+
 def malt_workspace_bytes(st) -> int:
     return int(load().malt_workspace_bytes(st))
 
@@ -403,6 +494,9 @@ class MaltOptimizer:
     def set_ns_schedule(self, schedule: int):
         malt_set_ns_schedule(self.state, schedule)
 
+    def set_weight_copies(self, copies):
+        malt_set_weight_copies(self.state, copies, self.n)
+
     def profile(self, enable: bool = True):
         malt_profile_enable(self.state, enable)
 
@@ -422,3 +516,59 @@ class MaltOptimizer:
             self.close()
         except Exception:
             pass
+
+
+class AdamW:
+    """Owns a malt_adamw_state for a fixed list of (w, w_copy or None, g, m, v,
+    weight_decay) device tensors; m and v are zeroed at construction."""
+
+    def __init__(self, params, stream=None):
+        self.params = list(params)
+        self.state = malt_adamw_init_state(self.params, stream)
+
+    def step(self, hp: malt_adamw_hparams_t, stream=None, params=None):
+        malt_adamw_step(self.state, self.params if params is None else params, hp, stream)
+
+    def get_step(self) -> int:
+        return malt_adamw_get_step(self.state)
+
+    def set_step(self, t: int):
+        malt_adamw_set_step(self.state, t)
+
+    def close(self):
+        if self.state is not None:
+            malt_adamw_destroy_state(self.state)
+            self.state = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class WholeOptimizer:
+    """A whole-optimizer step of a model (Section 5.1 parameter grouping):
+    MALT or MALTER on the 2-D weight matrices, AdamW on every other tensor,
+    both enqueued on the same stream.  matrices: (W, G, M, l, r) as for
+    MaltOptimizer (fp32 W for master weights); copies: optional bf16 copy per
+    matrix (None entries for none); others: (w, w_copy, g, m, v, weight_decay)
+    as for AdamW."""
+
+    def __init__(self, matrices, others, copies=None, stream=None):
+        self.malt = MaltOptimizer(matrices, stream)
+        if copies is not None:
+            self.malt.set_weight_copies(copies)
+        self.adamw = AdamW(others, stream)
+
+    def step(self, hp: malt_hparams_t, adamw_hp: malt_adamw_hparams_t, malter: bool = False,
+             stream=None):
+        self.malt.step(hp, malter=malter, stream=stream)
+        self.adamw.step(adamw_hp, stream=stream)
+
+    def check(self) -> int:
+        return self.malt.check()
+
+    def close(self):
+        self.malt.close()
+        self.adamw.close()

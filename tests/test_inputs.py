@@ -108,3 +108,27 @@ def test_random_shapes():
     assert all(r % 8 == 0 and c % 8 == 0 and 8 <= r <= 776 and 8 <= c <= 776 for r, c in s)
     big = inputs.random_shapes(11, 5, max_dim=2056)
     assert all(8 <= r <= 2056 and 8 <= c <= 2056 for r, c in big)
+
+
+def test_gpt2_whole_parameter_counts_match_the_paper():
+    """The 2-D matrices MALT updates plus the tensors AdamW updates add up to
+    the model sizes Section 5.1 states: GPT-2 Small 124M, Medium 355M, Large
+    774M parameters (NanoGPT's padded vocabulary, tied head)."""
+    for name, millions in (("gpt2_small", 124), ("gpt2_medium", 355), ("gpt2_large", 774)):
+        total = inputs.WORKLOADS[name].elements + inputs.ADAMW_SETS[name].elements
+        assert round(total / 1e6) == millions, (name, total)
+
+
+def test_adamw_set_recipe():
+    aset = inputs.ADAMW_SETS["gpt2_small"]
+    names = [t[0] for t in aset.tensors]
+    assert names[:2] == ["wte", "wpe"] and len(names) == 2 + 8 * 12 + 2
+    assert all(wd == (0.1 if len(shape) == 2 else 0.0) for _, shape, wd in aset.tensors)
+    assert aset.lr == 0.0013 and inputs.ADAMW_SETS["gpt2_large"].lr == 0.0009
+    w = inputs.adamw_initial(aset, 0)
+    assert w.dtype == np.float32 and w.shape == (50304, 768) and abs(w.std() - 0.02) < 1e-3
+    assert np.all(inputs.adamw_initial(aset, names.index("h0.ln_1.weight")) == 1.0)
+    assert not np.any(inputs.adamw_initial(aset, names.index("h0.mlp.c_fc.bias")))
+    g0 = inputs.adamw_gradient(aset, 5, 0)
+    assert np.array_equal(g0, inputs.adamw_gradient(aset, 5, 0))
+    assert not np.array_equal(g0, inputs.adamw_gradient(aset, 5, 1))
