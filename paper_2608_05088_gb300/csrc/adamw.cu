@@ -53,20 +53,32 @@ struct AdamDesc {
     int32_t pad_;
 };
 
-struct AdamBind {
-    AdamPtrs p[kAdamBindChunk];
-    int32_t count, offset;
-    long long* tcount;      // advanced by the first chunk's launch
-};
-
 struct AdamHyper {
     float lr, beta1, beta2, eps;
 };
 
+struct AdamBind {
+    AdamPtrs p[kAdamBindChunk];
+    int32_t count, offset;
+    long long* tcount;      // advanced by the first chunk's launch
+    float* factors;         // [2]: lr / (1 - beta1^t), 1 / sqrt(1 - beta2^t)
+    AdamHyper h;
+};
+
+// Copies the caller's pointers; the first chunk's launch also advances the
+// step count t and computes the step's two bias-correction factors once (in
+// double: the update kernel itself does no fp64 arithmetic).
 __global__ void adamw_bind_kernel(const __grid_constant__ AdamBind B, AdamPtrs* __restrict__ table) {
     const int i = threadIdx.x;
     if (i < B.count) table[B.offset + i] = B.p[i];
-    if (i == 0 && B.tcount != nullptr) *B.tcount += 1;          // 1-based step count
+    if (i == 0 && B.tcount != nullptr) {
+        const long long tc = *B.tcount + 1;                      // 1-based step count
+        *B.tcount = tc;
+        const double t = static_cast<double>(tc);
+        B.factors[0] = static_cast<float>(static_cast<double>(B.h.lr) /
+                                          (1.0 - pow(static_cast<double>(B.h.beta1), t)));
+        B.factors[1] = static_cast<float>(1.0 / sqrt(1.0 - pow(static_cast<double>(B.h.beta2), t)));
+    }
 }
 
 __device__ __forceinline__ int find_tensor(const int32_t* __restrict__ pref, int n, int32_t x) {
@@ -101,19 +113,16 @@ __device__ __forceinline__ void adam1(float& w, float& m, float& v, float g, con
 
 __global__ void __launch_bounds__(kAdamThreads)
 adamw_kernel(const AdamDesc* __restrict__ desc, const AdamPtrs* __restrict__ ptrs,
-             const int32_t* __restrict__ pref, int n, const long long* __restrict__ tcount,
+             const int32_t* __restrict__ pref, int n, const float* __restrict__ factors,
              AdamHyper h) {
     const int k = find_tensor(pref, n, blockIdx.x);
     const AdamDesc d = desc[k];
     const AdamPtrs p = ptrs[k];
     const int64_t begin = static_cast<int64_t>(blockIdx.x - __ldg(pref + k)) * kAdamChunk;
     const int64_t end = d.numel < begin + kAdamChunk ? d.numel : begin + kAdamChunk;
-    // Bias corrections of step t (double, then the two fp32 factors).
-    const double t = static_cast<double>(*tcount);
-    const float step = static_cast<float>(static_cast<double>(h.lr) /
-                                          (1.0 - pow(static_cast<double>(h.beta1), t)));
-    const float inv_sqrt_bc2 =
-        static_cast<float>(1.0 / sqrt(1.0 - pow(static_cast<double>(h.beta2), t)));
+    // Bias corrections of this step t, computed by the bind launch.
+    const float step = factors[0];
+    const float inv_sqrt_bc2 = factors[1];
     const bool gbf = d.g_bf16 != 0;
     const int64_t vec_end = begin + ((end - begin) / kAdamVec) * kAdamVec;
     constexpr int64_t kPass = static_cast<int64_t>(kAdamThreads) * kAdamVec * kAdamInFlight;
@@ -201,6 +210,7 @@ struct malt_adamw_state {
     AdamPtrs* d_ptrs = nullptr;
     int32_t* d_pref = nullptr;
     long long* d_t = nullptr;
+    float* d_factors = nullptr;
     int32_t blocks = 0;
     cudaStream_t last_stream = nullptr;
 };
@@ -250,6 +260,7 @@ int malt_adamw_init_state(malt_adamw_state_t** out, const malt_adamw_param_t* pa
     st->d_ptrs = reinterpret_cast<AdamPtrs*>(base + o_ptrs);
     st->d_pref = reinterpret_cast<int32_t*>(base + o_pref);
     st->d_t = reinterpret_cast<long long*>(base + o_t);
+    st->d_factors = reinterpret_cast<float*>(base + o_t + 64);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     int rc = cuda_fail(cudaMemset(st->ws, 0, bytes), "cudaMemset(state)");
     if (rc == MALT_OK && n > 0)
@@ -293,6 +304,8 @@ int malt_adamw_step(malt_adamw_state_t* st, const malt_adamw_param_t* params, in
         B.count = cnt;
         B.offset = off;
         B.tcount = off == 0 ? st->d_t : nullptr;
+        B.factors = st->d_factors;
+        B.h = AdamHyper{hp->lr, hp->beta1, hp->beta2, hp->eps};
         for (int i = 0; i < cnt; ++i) {
             const malt_adamw_param_t& p = params[off + i];
             B.p[i] = AdamPtrs{p.w, p.w_copy, p.g, p.m, p.v, 1.f - hp->lr * p.weight_decay, 0};
@@ -302,7 +315,8 @@ int malt_adamw_step(malt_adamw_state_t* st, const malt_adamw_param_t* params, in
     }
     if (st->blocks == 0) return MALT_OK;
     const AdamHyper h{hp->lr, hp->beta1, hp->beta2, hp->eps};
-    adamw_kernel<<<st->blocks, kAdamThreads, 0, s>>>(st->d_desc, st->d_ptrs, st->d_pref, n, st->d_t, h);
+    adamw_kernel<<<st->blocks, kAdamThreads, 0, s>>>(st->d_desc, st->d_ptrs, st->d_pref, n,
+                                                     st->d_factors, h);
     ADAM_CUDA(cudaGetLastError(), "adamw_kernel");
     return MALT_OK;
 }

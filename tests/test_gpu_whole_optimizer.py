@@ -4,9 +4,10 @@ weight decay 0.1 (appendix table), and AdamW on every other tensor, against
 the fp64 oracles.
 
 Bars (fp32 arithmetic against fp64): AdamW moments within 1e-5 relative
-(Frobenius, per tensor); the AdamW update w_t - w_{t-1} within 1e-5 relative;
-master weights within 1e-6 (|w| + lr) elementwise, i.e. a few fp32 ulps of the
-weight and of the step; every bf16 copy equal, bit for bit, to the
+(Frobenius, per tensor); each element of the update w_t - w_{t-1} within 1e-5
+of the oracle's step (teacher-forced on the GPU's w_{t-1}) plus two fp32 ulps
+of w, the resolution at which an fp32 master can move; master weights within
+1e-6 (|w| + lr) elementwise; every bf16 copy equal, bit for bit, to the
 round-to-nearest-even of the GPU's own fp32 master (integer-exact work)."""
 import dataclasses
 
@@ -91,7 +92,12 @@ class AdamRun:
         m_hat = st.m / (1 - self.hp_ref.beta1 ** t)
         v_hat = st.v / (1 - self.hp_ref.beta2 ** t)
         step_ref = (1 - lr * wd) * self.w_prev[i] - lr * m_hat / (np.sqrt(v_hat) + self.hp_ref.eps)
-        assert _rel(w - self.w_prev[i], step_ref - self.w_prev[i]) < TOL_UPDATE, msg
+        # elementwise: 1e-5 of the step, plus the fp32 resolution of w itself
+        # (the decay product, the fused update and the store each round w to
+        # fp32: at most two ulps of w together)
+        d_gpu, d_ref = w - self.w_prev[i], step_ref - self.w_prev[i]
+        ulp = np.spacing(np.maximum(np.abs(w), np.abs(self.w_prev[i])).astype(np.float32))
+        assert np.all(np.abs(d_gpu - d_ref) <= TOL_UPDATE * np.abs(d_ref) + 2.0 * ulp), msg
         err = np.abs(w - self.w_ref[i])
         assert np.all(err <= TOL_MASTER * (np.abs(self.w_ref[i]) + lr)), (msg, float(err.max()))
         if self.wc[i] is not None:
