@@ -111,7 +111,7 @@ __device__ __forceinline__ void adam1(float& w, float& m, float& v, float g, con
     w = fmaf(-step, m / denom, decay * w);
 }
 
-__global__ void __launch_bounds__(kAdamThreads)
+__global__ void __launch_bounds__(kAdamThreads, 4)
 adamw_kernel(const AdamDesc* __restrict__ desc, const AdamPtrs* __restrict__ ptrs,
              const int32_t* __restrict__ pref, int n, const float* __restrict__ factors,
              AdamHyper h) {
