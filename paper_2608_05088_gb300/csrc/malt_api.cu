@@ -335,6 +335,7 @@ void plan_ns_groups(const std::vector<ShapeClass>& classes, int nmat, std::vecto
             C.tiles_q = (S.q + kBN - 1) / kBN;
             C.sym_begin = sym;
             C.full_begin = full;
+            C.bx_col_major = static_cast<int64_t>(S.p) * S.q * 2 > kBxColBytes ? 1 : 0;
             C.mat_of = S.d_mat_of;
             C.A = S.A;
             sym += ns_phase_tiles(C, kGram) * S.batch;

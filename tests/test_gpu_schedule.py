@@ -117,3 +117,16 @@ def test_unknown_schedule_rejected():
     with pytest.raises(malt.MaltError):
         run.opt.set_ns_schedule(7)
     run.close()
+
+
+def test_column_major_bx_order_bitwise_and_against_oracle():
+    """A frame whose X is larger than 32 MiB (2056 x 8192, bf16: 33.7 MB) lists
+    its B*X tiles column by column; with a ragged last tile row (2056 = 8 x 257)
+    both schedules agree bitwise and the step matches the oracle."""
+    wl = inputs.Workload("bxcol", 57, ((2056, 8192),), "bf16", 1.5, 0.02, "malt", 1)
+    run_both(wl, 1, schedules=[malt.MALT_NS_PHASED, malt.MALT_NS_PERSISTENT])
+    run = Run(wl)
+    run.step()
+    assert run.status() == malt.MALT_OK
+    run.assert_close(0)
+    run.close()
