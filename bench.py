@@ -36,7 +36,18 @@ UNIT = "steps/s"
 DEFAULT_WORKLOAD = "gpt2_large"
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 NCU_SUMMARY = os.path.join(ROOT, "profiles", "ns_gemm_gpt2_large_ncu.json")
-NS_SOURCE = os.path.join(ROOT, "paper_2608_05088_gb300", "csrc", "ns_gemm.cu")
+# The sources the Newton-Schulz kernel compiles from: the traffic figure of
+# the committed ncu summary holds only while all of them are unchanged.
+NS_SOURCES = [os.path.join(ROOT, "paper_2608_05088_gb300", "csrc", f)
+              for f in ("ns_gemm.cu", "common.cuh", "ptx.cuh")]
+
+
+def ns_sources_sha256() -> str:
+    h = hashlib.sha256()
+    for path in NS_SOURCES:
+        with open(path, "rb") as f:
+            h.update(hashlib.sha256(f.read()).digest())
+    return h.hexdigest()
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -188,14 +199,12 @@ def peaks():
 
 def ncu_traffic_per_launch(persistent: bool):
     """DRAM bytes per NS GEMM launch (of the schedule the timed steps used)
-    from the committed ncu summary, or None when the kernel source changed
-    since the capture."""
+    from the committed ncu summary, or None when a kernel source changed
+    since the capture or the summary has no figure for the schedule."""
     try:
         with open(NCU_SUMMARY) as f:
             s = json.load(f)
-        with open(NS_SOURCE, "rb") as f:
-            h = hashlib.sha256(f.read()).hexdigest()
-        if s.get("ns_gemm_sha256") != h:
+        if s.get("ns_sources_sha256") != ns_sources_sha256():
             return None
         key = "persistent_dram_bytes_per_launch_full_size" if persistent else \
               "dram_bytes_per_launch_full_size"

@@ -150,3 +150,16 @@ def test_clock_summary_fallbacks():
     got = bench.ClockSampler.summarise([["n/a"] + r[1:] for r in rows], t0, t0 + 0.55)
     assert got["samples"] == 22 and got["window"].startswith("all samples")
     assert bench.ClockSampler.summarise([], t0, t0 + 1) is None
+
+
+def test_roofline_traffic_holds_only_for_the_captured_kernel(tmp_path, monkeypatch):
+    """roofline.traffic comes from the committed ncu summary only while every
+    source the Newton-Schulz kernel compiles from is the one it was captured
+    with; a changed source makes it null."""
+    sys.path.insert(0, ROOT)
+    import bench
+    assert bench.ncu_traffic_per_launch(False) is not None
+    changed = tmp_path / "common.cuh"
+    changed.write_bytes(open(bench.NS_SOURCES[1], "rb").read() + b"// edited\n")
+    monkeypatch.setattr(bench, "NS_SOURCES", [bench.NS_SOURCES[0], str(changed), bench.NS_SOURCES[2]])
+    assert bench.ncu_traffic_per_launch(False) is None
