@@ -56,8 +56,8 @@ extern "C" {
 /* ---- status codes ------------------------------------------------------ */
 #define MALT_OK                   0
 #define MALT_ERR_INVALID_ARG     -1  /* null pointer, n < 0, bad hyperparameter */
-#define MALT_ERR_UNSUPPORTED     -2  /* rows or cols not a positive multiple of 8,
-                                        rows*cols >= 2^31, bad dtype */
+#define MALT_ERR_UNSUPPORTED     -2  /* rows or cols < 1, rows*cols >= 2^31 after
+                                        rounding each up to a multiple of 8, bad dtype */
 #define MALT_ERR_MISALIGNED      -3  /* a device pointer is not 16-byte aligned */
 #define MALT_ERR_SHAPE_CHANGED   -4  /* step called with shapes/dtypes other than at init */
 #define MALT_ERR_CUDA            -5  /* a CUDA runtime call failed (see malt_status_string) */
@@ -76,9 +76,13 @@ extern "C" {
  *   m       momentum M, rows x cols fp32, updated in place
  *   l, r    row statistics (rows fp32) and column statistics (cols fp32),
  *           updated in place
- * rows and cols must be positive multiples of 8, with rows*cols < 2^31 (the
- * kernels index a matrix's elements with 32-bit offsets).  W, G and M must not
- * overlap each other or another parameter's buffers. */
+ * rows and cols may be any positive sizes, with rows*cols < 2^31 after rounding
+ * each up to a multiple of 8 (the kernels index a matrix's elements with
+ * 32-bit offsets).  A matrix whose rows or cols are not multiples of 8 runs on
+ * zero-padded copies in the library's workspace: each step copies its W, G,
+ * M, l, r in and W, M, l, r back out (two extra passes over that matrix
+ * only), with the same results.  W, G and M must not overlap each other or
+ * another parameter's buffers. */
 typedef struct {
     void*        w;
     int32_t      w_dtype;
@@ -232,7 +236,8 @@ int malt_debug_wait_timeout(int64_t budget_ns, void* stream);
 #define MALT_KIND_SCALARS   8
 #define MALT_KIND_APPLY     9
 #define MALT_KIND_NS_PERSISTENT 10   /* all Newton-Schulz products, persistent schedule */
-#define MALT_NUM_KINDS     11
+#define MALT_KIND_PAD      11   /* copies of matrices with rows or cols not a multiple of 8 */
+#define MALT_NUM_KINDS     12
 int malt_profile_enable(malt_state_t* st, int32_t enable);
 int malt_profile_read(malt_state_t* st, double* ms_out, int64_t* launches_out, int32_t nkinds);
 

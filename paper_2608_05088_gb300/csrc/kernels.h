@@ -13,7 +13,32 @@ struct BindParams {
     int32_t offset;
 };
 
+// Matrices whose rows or cols are not multiples of 8 run on zero-padded
+// copies in the workspace (rows and cols rounded up to 8).  Before a step the
+// pad launch copies the caller's W, G, M, l, r in; after it the unpad launch
+// copies W, M, l, r back (and writes the bf16 copy of an fp32 W, if one is
+// registered).  The padding is zero at init and every stage keeps it zero.
+constexpr int kPadChunk = 48;      // matrices per pad / unpad launch
+constexpr int kPadRows = 8;        // rows per block (one warp per row)
+struct PadEntry {
+    void* w_user;  void* w_pad;    // W (bf16 when w_bf16, else fp32)
+    const void* g_user; void* g_pad;   // G (bf16 when g_bf16, else fp32)
+    float* m_user; float* m_pad;
+    float* l_user; float* l_pad;
+    float* r_user; float* r_pad;
+    void* wcopy_user;              // bf16 copy of an fp32 W (rows x cols), or null
+    int32_t m, n, n8;              // caller rows and cols; padded leading dimension
+    int32_t w_bf16, g_bf16;
+    int32_t block_begin;           // first block of this matrix in the launch
+};
+struct PadParams {
+    PadEntry e[kPadChunk];
+    int32_t count;
+};
+
 cudaError_t launch_bind(const BindParams& P, UserPtrs* table, cudaStream_t s);
+// in = true: caller -> padded copies; false: padded -> caller.
+cudaError_t launch_pad(const PadParams& P, int32_t blocks, bool in, cudaStream_t s);
 cudaError_t launch_stats(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* pref,
                          int nmat, int32_t blocks, float mu1, int with_stats, cudaStream_t s);
 cudaError_t launch_finalize(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* pref,

@@ -105,6 +105,19 @@ int cuda_fail(cudaError_t e, const char* what) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// Rows and cols as the kernels see them: rounded up to a multiple of 8 (a
+// matrix with other dimensions runs on zero-padded copies in the workspace).
+int64_t round8(int64_t x) { return (x + 7) / 8 * 8; }
+
+// Workspace copies of a matrix whose rows or cols are not multiples of 8.
+struct PadBuf {
+    void* w = nullptr;
+    void* g = nullptr;
+    float* m = nullptr;
+    float* l = nullptr;
+    float* r = nullptr;
+};
+
 }  // namespace
 
 struct malt_state {
@@ -113,6 +126,8 @@ struct malt_state {
     int num_sms = 0;
     std::vector<malt_param_t> shape0;      // shapes / dtypes fixed at init
     std::vector<void*> wcopy;              // bf16 copies of fp32 weights (malt_set_weight_copies)
+    std::vector<int> padded;               // matrices whose rows or cols are not multiples of 8
+    std::vector<PadBuf> padbuf;            // their zero-padded workspace copies (index = matrix)
     std::vector<MatDesc> hmats;
     std::vector<ShapeClass> classes;
     void* ws = nullptr;
@@ -172,9 +187,8 @@ namespace {
 int validate_param(const malt_param_t& p) {
     if (p.w == nullptr || p.g == nullptr || p.m == nullptr || p.l == nullptr || p.r == nullptr)
         return MALT_ERR_INVALID_ARG;
-    if (p.rows <= 0 || p.cols <= 0 || (p.rows % 8) != 0 || (p.cols % 8) != 0)
-        return MALT_ERR_UNSUPPORTED;
-    if (p.rows * p.cols >= (static_cast<int64_t>(1) << 31)) return MALT_ERR_UNSUPPORTED;
+    if (p.rows <= 0 || p.cols <= 0) return MALT_ERR_UNSUPPORTED;
+    if (round8(p.rows) * round8(p.cols) >= (static_cast<int64_t>(1) << 31)) return MALT_ERR_UNSUPPORTED;
     if ((p.w_dtype != MALT_F32 && p.w_dtype != MALT_BF16) ||
         (p.g_dtype != MALT_F32 && p.g_dtype != MALT_BF16))
         return MALT_ERR_UNSUPPORTED;
@@ -258,7 +272,9 @@ void build_classes(const malt_param_t* params, int n, std::vector<MatDesc>& hmat
     hmats.resize(n);
     std::map<std::pair<int, int>, int> cls_of;
     for (int i = 0; i < n; ++i) {
-        const int m = static_cast<int>(params[i].rows), c = static_cast<int>(params[i].cols);
+        // the kernels' view: rows and cols rounded up to multiples of 8
+        const int m = static_cast<int>(round8(params[i].rows));
+        const int c = static_cast<int>(round8(params[i].cols));
         const int p = std::min(m, c), q = std::max(m, c);
         auto it = cls_of.find({p, q});
         int k;
@@ -440,6 +456,20 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
             st->table_per_iter.push_back(table_per_iter(groups[gi]));
         }
     }
+    // Zero-padded copies of matrices whose rows or cols are not multiples of 8.
+    st->padbuf.assign(n, PadBuf{});
+    std::vector<size_t> o_pw(n), o_pg(n), o_pm(n), o_pl(n), o_pr(n);
+    for (int i = 0; i < n; ++i) {
+        if (params[i].rows % 8 == 0 && params[i].cols % 8 == 0) continue;
+        st->padded.push_back(i);
+        const MatDesc& d = st->hmats[i];
+        const size_t e = static_cast<size_t>(d.m) * d.n;
+        o_pw[i] = cv.take(e * (params[i].w_dtype == MALT_BF16 ? 2 : 4));
+        o_pg[i] = cv.take(e * (params[i].g_dtype == MALT_BF16 ? 2 : 4));
+        o_pm[i] = cv.take(e * sizeof(float));
+        o_pl[i] = cv.take(sizeof(float) * d.m);
+        o_pr[i] = cv.take(sizeof(float) * d.n);
+    }
     std::vector<size_t> o_table(tables.size());
     for (size_t gi = 0; gi < tables.size(); ++gi)
         o_table[gi] = cv.take(sizeof(NsEntry) * std::max<size_t>(tables[gi].size(), 1));
@@ -484,6 +514,14 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
     st->d_sched = reinterpret_cast<uint32_t*>(base + o_sched);
     for (size_t gi = 0; gi < tables.size(); ++gi)
         st->table_dev.push_back(reinterpret_cast<NsEntry*>(base + o_table[gi]));
+    for (int i : st->padded) {
+        PadBuf& b = st->padbuf[i];
+        b.w = base + o_pw[i];
+        b.g = base + o_pg[i];
+        b.m = F(o_pm[i]);
+        b.l = F(o_pl[i]);
+        b.r = F(o_pr[i]);
+    }
 
     // Block-prefix tables.
     std::vector<int32_t> pref[4];
@@ -563,10 +601,53 @@ int bind_pointers(malt_state* st, const malt_param_t* params, cudaStream_t s) {
         bp.offset = off;
         for (int i = 0; i < cnt; ++i) {
             const malt_param_t& p = params[off + i];
-            bp.p[i] = UserPtrs{p.w, p.g, p.m, p.l, p.r, st->wcopy[off + i]};
+            const PadBuf& b = st->padbuf[off + i];
+            // A padded matrix's kernels work on its workspace copies; its
+            // bf16 copy is written by the unpad launch, in the caller's layout.
+            bp.p[i] = b.w != nullptr ? UserPtrs{b.w, b.g, b.m, b.l, b.r, nullptr}
+                                     : UserPtrs{p.w, p.g, p.m, p.l, p.r, st->wcopy[off + i]};
         }
         LaunchScope ls(st, MALT_KIND_BIND, s);
         MALT_CUDA(launch_bind(bp, st->d_ptrs, s), "bind_kernel");
+    }
+    return MALT_OK;
+}
+
+// Copy the padded matrices' caller buffers into their workspace copies (in)
+// or back (out), kPadChunk matrices per launch.
+int run_padding(malt_state* st, const malt_param_t* params, bool in, cudaStream_t s) {
+    thread_local PadParams P;
+    for (size_t off = 0; off < st->padded.size(); off += kPadChunk) {
+        const int cnt = static_cast<int>(std::min<size_t>(kPadChunk, st->padded.size() - off));
+        std::memset(&P, 0, sizeof(P));
+        P.count = cnt;
+        int32_t blocks = 0;
+        for (int k = 0; k < cnt; ++k) {
+            const int i = st->padded[off + k];
+            const malt_param_t& p = params[i];
+            const PadBuf& b = st->padbuf[i];
+            PadEntry& e = P.e[k];
+            e.w_user = p.w;
+            e.w_pad = b.w;
+            e.g_user = p.g;
+            e.g_pad = b.g;
+            e.m_user = p.m;
+            e.m_pad = b.m;
+            e.l_user = p.l;
+            e.l_pad = b.l;
+            e.r_user = p.r;
+            e.r_pad = b.r;
+            e.wcopy_user = st->wcopy[i];
+            e.m = static_cast<int32_t>(p.rows);
+            e.n = static_cast<int32_t>(p.cols);
+            e.n8 = st->hmats[i].n;
+            e.w_bf16 = p.w_dtype == MALT_BF16;
+            e.g_bf16 = p.g_dtype == MALT_BF16;
+            e.block_begin = blocks;
+            blocks += static_cast<int32_t>((p.rows + kPadRows - 1) / kPadRows);
+        }
+        LaunchScope ls(st, MALT_KIND_PAD, s);
+        MALT_CUDA(launch_pad(P, blocks, in, s), in ? "pad_kernel (in)" : "pad_kernel (out)");
     }
     return MALT_OK;
 }
@@ -681,6 +762,12 @@ int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_h
     MALT_CUDA(cudaSetDevice(st->device), "cudaSetDevice");
     rc = bind_pointers(st, params, s);
     if (rc != MALT_OK) return rc;
+    if (!st->padded.empty()) {
+        // The padded copies are overwritten: the previous host step's weight
+        // read-back must be done (the read-back reads the caller's W).
+        rc = run_padding(st, params, true, s);
+        if (rc != MALT_OK) return rc;
+    }
     const int nm = st->nmat;
     {
         LaunchScope ls(st, MALT_KIND_STATS, s);
@@ -717,6 +804,10 @@ int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_h
         MALT_CUDA(launch_apply(st->d_mats, st->d_ptrs, st->d_scal, st->d_pref[3], nm,
                                st->blocks_apply, 1.f - hp->lr * hp->weight_decay, s),
                   "apply_kernel");
+    }
+    if (!st->padded.empty()) {
+        rc = run_padding(st, params, false, s);
+        if (rc != MALT_OK) return rc;
     }
     if (hooks != nullptr)
         MALT_CUDA(cudaEventRecord(hooks->record_applied, s), "cudaEventRecord(applied)");
@@ -920,11 +1011,14 @@ int malt_set_scalars(malt_state_t* st, const float* nu_host, int32_t n, int64_t 
 int malt_debug_direction(malt_state_t* st, int32_t idx, void* out, void* stream) {
     if (st == nullptr || idx < 0 || idx >= st->nmat || out == nullptr) return MALT_ERR_INVALID_ARG;
     const MatDesc& d = st->hmats[idx];
+    const malt_param_t& p = st->shape0[idx];
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     // O is stored in W's layout for every matrix (the last B*X epilogue
-    // writes a tall matrix's tiles transposed).
-    MALT_CUDA(cudaMemcpyAsync(out, d.O, static_cast<size_t>(d.m) * d.n * 2,
-                              cudaMemcpyDeviceToDevice, s), "cudaMemcpyAsync(O)");
+    // writes a tall matrix's tiles transposed), with leading dimension d.n
+    // (cols rounded up to 8); the caller's copy is rows x cols, dense.
+    MALT_CUDA(cudaMemcpy2DAsync(out, static_cast<size_t>(p.cols) * 2, d.O, static_cast<size_t>(d.n) * 2,
+                                static_cast<size_t>(p.cols) * 2, static_cast<size_t>(p.rows),
+                                cudaMemcpyDeviceToDevice, s), "cudaMemcpy2DAsync(O)");
     return MALT_OK;
 }
 
@@ -932,10 +1026,11 @@ int malt_debug_precond(malt_state_t* st, int32_t idx, float* L_out, float* R_out
     if (st == nullptr || idx < 0 || idx >= st->nmat || L_out == nullptr || R_out == nullptr)
         return MALT_ERR_INVALID_ARG;
     const MatDesc& d = st->hmats[idx];
+    const malt_param_t& p = st->shape0[idx];
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    MALT_CUDA(cudaMemcpyAsync(L_out, d.L, sizeof(float) * d.m, cudaMemcpyDeviceToDevice, s),
+    MALT_CUDA(cudaMemcpyAsync(L_out, d.L, sizeof(float) * p.rows, cudaMemcpyDeviceToDevice, s),
               "cudaMemcpyAsync(L)");
-    MALT_CUDA(cudaMemcpyAsync(R_out, d.R, sizeof(float) * d.n, cudaMemcpyDeviceToDevice, s),
+    MALT_CUDA(cudaMemcpyAsync(R_out, d.R, sizeof(float) * p.cols, cudaMemcpyDeviceToDevice, s),
               "cudaMemcpyAsync(R)");
     return MALT_OK;
 }
@@ -1039,8 +1134,8 @@ int malt_ns_schedule(const malt_param_t* params, int32_t n, int32_t ns_steps, in
         ns_steps > kMaxNsSteps || capacity < 0 || (capacity > 0 && out == nullptr))
         return MALT_ERR_INVALID_ARG;
     for (int i = 0; i < n; ++i)
-        if (params[i].rows <= 0 || params[i].cols <= 0 || params[i].rows % 8 != 0 ||
-            params[i].cols % 8 != 0 || params[i].rows * params[i].cols >= (int64_t{1} << 31))
+        if (params[i].rows <= 0 || params[i].cols <= 0 ||
+            round8(params[i].rows) * round8(params[i].cols) >= (int64_t{1} << 31))
             return MALT_ERR_UNSUPPORTED;
     std::vector<MatDesc> hmats;
     std::vector<ShapeClass> classes;
@@ -1078,7 +1173,7 @@ const char* malt_status_string(int code) {
     switch (code) {
         case MALT_OK: return "ok";
         case MALT_ERR_INVALID_ARG: return "invalid argument";
-        case MALT_ERR_UNSUPPORTED: return "unsupported shape or dtype (rows and cols must be positive multiples of 8, rows*cols < 2^31)";
+        case MALT_ERR_UNSUPPORTED: return "unsupported shape or dtype (rows and cols must be positive, with rows*cols < 2^31 after rounding each up to a multiple of 8)";
         case MALT_ERR_MISALIGNED: return "device pointer not 16-byte aligned";
         case MALT_ERR_SHAPE_CHANGED: return "parameter shapes or dtypes differ from init";
         case MALT_ERR_CUDA: return "CUDA runtime error";

@@ -35,6 +35,59 @@ __global__ void bind_kernel(const __grid_constant__ BindParams P, UserPtrs* __re
     if (i < P.count) table[P.offset + i] = P.p[i];
 }
 
+// ------------------------------------------------------------ pad / unpad
+// One block copies kPadRows rows of one matrix (one warp per row, lanes along
+// the row); the matrix's first block also copies l and r.
+template <typename T>
+__device__ __forceinline__ void copy_row(const T* __restrict__ src, T* __restrict__ dst, int n,
+                                         int lane) {
+    for (int j = lane; j < n; j += 32) dst[j] = src[j];
+}
+
+template <bool kIn>
+__global__ void __launch_bounds__(256) pad_kernel(const __grid_constant__ PadParams P) {
+    int k = 0;
+    while (k + 1 < P.count && P.e[k + 1].block_begin <= static_cast<int32_t>(blockIdx.x)) ++k;
+    const PadEntry& e = P.e[k];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int row = (static_cast<int>(blockIdx.x) - e.block_begin) * kPadRows + warp;
+    if (row < e.m) {
+        const size_t u = static_cast<size_t>(row) * e.n;      // caller layout, ld = n
+        const size_t q = static_cast<size_t>(row) * e.n8;     // padded layout, ld = n8
+        if (kIn) {
+            if (e.w_bf16)
+                copy_row(static_cast<const uint16_t*>(e.w_user) + u, static_cast<uint16_t*>(e.w_pad) + q, e.n, lane);
+            else
+                copy_row(static_cast<const float*>(e.w_user) + u, static_cast<float*>(e.w_pad) + q, e.n, lane);
+            if (e.g_bf16)
+                copy_row(static_cast<const uint16_t*>(e.g_user) + u, static_cast<uint16_t*>(e.g_pad) + q, e.n, lane);
+            else
+                copy_row(static_cast<const float*>(e.g_user) + u, static_cast<float*>(e.g_pad) + q, e.n, lane);
+            copy_row<float>(e.m_user + u, e.m_pad + q, e.n, lane);
+        } else {
+            if (e.w_bf16) {
+                copy_row(static_cast<const uint16_t*>(e.w_pad) + q, static_cast<uint16_t*>(e.w_user) + u, e.n, lane);
+            } else {
+                const float* src = static_cast<const float*>(e.w_pad) + q;
+                copy_row(src, static_cast<float*>(e.w_user) + u, e.n, lane);
+                if (e.wcopy_user != nullptr) {
+                    __nv_bfloat16* c = static_cast<__nv_bfloat16*>(e.wcopy_user) + u;
+                    for (int j = lane; j < e.n; j += 32) c[j] = __float2bfloat16_rn(src[j]);
+                }
+            }
+            copy_row<float>(e.m_pad + q, e.m_user + u, e.n, lane);
+        }
+    }
+    if (static_cast<int>(blockIdx.x) == e.block_begin) {
+        for (int i = threadIdx.x; i < e.m; i += blockDim.x) {
+            if (kIn) e.l_pad[i] = e.l_user[i]; else e.l_user[i] = e.l_pad[i];
+        }
+        for (int j = threadIdx.x; j < e.n; j += blockDim.x) {
+            if (kIn) e.r_pad[j] = e.r_user[j]; else e.r_user[j] = e.r_pad[j];
+        }
+    }
+}
+
 // ------------------------------------------------------------------ stats
 template <bool kStats>
 __global__ void __launch_bounds__(256)
@@ -116,6 +169,14 @@ __global__ void wait_probe_kernel(int32_t* status, uint64_t budget_ns) {
 // ------------------------------------------------------------------ launch
 cudaError_t launch_bind(const BindParams& P, UserPtrs* table, cudaStream_t s) {
     bind_kernel<<<1, kBindChunk, 0, s>>>(P, table);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_pad(const PadParams& P, int32_t blocks, bool in, cudaStream_t s) {
+    if (in)
+        pad_kernel<true><<<blocks, 256, 0, s>>>(P);
+    else
+        pad_kernel<false><<<blocks, 256, 0, s>>>(P);
     return cudaGetLastError();
 }
 

@@ -104,14 +104,14 @@ def stress_workload(rows: int, cols: int, sigma: float, ns_steps: int) -> Worklo
                     "bf16", sigma, 0.02, "malt", 3, ns_steps)
 
 
-def random_shapes(seed: int, count: int, max_dim: int = 776) -> tuple:
-    """`count` seeded (rows, cols) pairs, each a multiple of 8 in [8, max_dim]:
-    wide, tall and square matrices with ragged tiles in both directions, and
-    repeated frames (a shared NS shape class) where two draws coincide up to
-    orientation."""
-    rng = np.random.Generator(np.random.PCG64([7_000, seed]))
-    hi = max_dim // 8
-    shapes = [(8 * int(rng.integers(1, hi + 1)), 8 * int(rng.integers(1, hi + 1)))
+def random_shapes(seed: int, count: int, max_dim: int = 776, multiple: int = 8) -> tuple:
+    """`count` seeded (rows, cols) pairs, each a multiple of `multiple` in
+    [multiple, max_dim]: wide, tall and square matrices with ragged tiles in
+    both directions, and repeated frames (a shared NS shape class) where two
+    draws coincide up to orientation."""
+    rng = np.random.Generator(np.random.PCG64([7_000 + (multiple != 8), seed]))
+    hi = max_dim // multiple
+    shapes = [(multiple * int(rng.integers(1, hi + 1)), multiple * int(rng.integers(1, hi + 1)))
               for _ in range(count)]
     if count >= 2:
         shapes[-1] = shapes[0][::-1]          # one tall/wide pair in the same class

@@ -37,7 +37,7 @@ EXPORTS = ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
            "malt_adamw_get_step", "malt_adamw_set_step", "malt_adamw_destroy_state")
 NOALLOC_SCRATCH_FLOATS = 1048576
 KIND_NAMES = ("bind", "stats", "finalize", "prescale", "norms", "ns_gram", "ns_poly", "ns_bx",
-              "scalars", "apply", "ns_persistent")
+              "scalars", "apply", "ns_persistent", "pad")
 NS_KINDS = ("ns_gram", "ns_poly", "ns_bx", "ns_persistent")
 # Newton-Schulz schedules (malt_set_ns_schedule)
 MALT_NS_PHASED = 0

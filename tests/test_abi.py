@@ -60,10 +60,11 @@ def test_host_validation_without_gpu(lib):
     assert lib.malt_init_state(None, None, 0, None) == malt.MALT_ERR_INVALID_ARG
     assert lib.malt_init_state(ctypes.byref(st), None, -1, None) == malt.MALT_ERR_INVALID_ARG
     cases = [
-        (_param(rows=7), malt.MALT_ERR_UNSUPPORTED),
-        (_param(cols=12), malt.MALT_ERR_UNSUPPORTED),
         (_param(rows=0), malt.MALT_ERR_UNSUPPORTED),
+        (_param(cols=-3), malt.MALT_ERR_UNSUPPORTED),
         (_param(rows=65536, cols=65536), malt.MALT_ERR_UNSUPPORTED),
+        # 46341 x 46337 < 2^31, but rounded up to multiples of 8 it is not
+        (_param(rows=46337, cols=46341), malt.MALT_ERR_UNSUPPORTED),
         (_param(w=0), malt.MALT_ERR_INVALID_ARG),
         (_param(m=24), malt.MALT_ERR_MISALIGNED),
         (_param(wd=7), malt.MALT_ERR_UNSUPPORTED),

@@ -61,8 +61,8 @@ def test_host_buffer_step_matches_device_step(schedule):
     the host copies of W equal the device W after every step."""
     import numpy as np
     import torch
-    wl = inputs.Workload("hoststep", 42, ((256, 512), (392, 136), (520, 1544)), "bf16", 1.5, 0.02,
-                         "malter", 3)
+    wl = inputs.Workload("hoststep", 42, ((256, 512), (392, 136), (520, 1544), (250, 509)), "bf16",
+                         1.5, 0.02, "malter", 3)
     a = Run(wl, check=[])
     b = Run(wl, check=[])
     if schedule == "persistent":

@@ -273,3 +273,39 @@ def test_newton_schulz_settings(ns_steps, coeffs):
     for i in range(2):
         run.assert_close(i)
     run.close()
+
+
+UNALIGNED = ((1, 1), (7, 13), (13, 7), (100, 3), (3, 1000), (255, 511), (1001, 999), (250, 509),
+             (256, 512))
+
+
+@pytest.mark.parametrize("variant,g_dtype", [("malt", "f32"), ("malter", "bf16"), ("muon", "f32")])
+def test_unaligned_shapes(variant, g_dtype):
+    """Rows and cols that are not multiples of 8 (a 1 x 1 matrix, odd and
+    prime sizes, wide and tall): such a matrix runs on zero-padded copies.
+    250 x 509 shares its padded frame (256 x 512) with an aligned matrix.
+    fp32 and bf16 weights, 3 steps, every matrix checked against the oracle."""
+    wl = inputs.Workload("unaligned", 46, UNALIGNED, "f32", 1.5, 0.02, variant, 3)
+    run = Run(wl, w_dtypes=["f32", "bf16", "bf16", "f32", "f32", "bf16", "f32", "bf16", "f32"],
+              g_dtype=g_dtype)
+    for s_ in range(wl.steps):
+        run.step()
+        assert run.status() == 0
+        for i in range(len(UNALIGNED)):
+            run.assert_close(i, f"{variant} step {s_}")
+    run.close()
+
+
+@pytest.mark.parametrize("seed", [21, 22])
+def test_seeded_random_odd_shapes(seed):
+    """Ten seeded random shapes of any size up to 517 (most not multiples of
+    8), fp32 and bf16 weights, 2 MALTER steps, every matrix against the oracle."""
+    shapes = inputs.random_shapes(seed, 10, max_dim=517, multiple=1)
+    wl = inputs.Workload(f"odd{seed}", 47 + seed, shapes, "f32", 1.5, 0.02, "malter", 2)
+    run = Run(wl, w_dtypes=["f32", "bf16"] * 5)
+    for _ in range(wl.steps):
+        run.step()
+        assert run.status() == 0
+    for i in range(len(shapes)):
+        run.assert_close(i, f"seed {seed}")
+    run.close()

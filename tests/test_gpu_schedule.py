@@ -130,3 +130,11 @@ def test_column_major_bx_order_bitwise_and_against_oracle():
     assert run.status() == malt.MALT_OK
     run.assert_close(0)
     run.close()
+
+
+def test_unaligned_shapes_bitwise():
+    """Padded matrices (rows or cols not multiples of 8) give bitwise the same
+    results under every schedule."""
+    shapes = inputs.random_shapes(23, 10, max_dim=517, multiple=1)
+    wl = inputs.Workload("schedodd", 58, shapes, "f32", 1.5, 0.02, "malter", 2)
+    run_both(wl, 2, w_dtypes=["f32", "bf16"] * 5, g_dtype="bf16")

@@ -253,15 +253,19 @@ def test_whole_optimizer_gpt2_small():
 
 
 def test_weight_copies_need_fp32_weights():
+    """Copies are written for fp32 weights only; a matrix with odd sizes
+    (padded inside the library) gets its copy in the caller's layout."""
     import torch
-    wl = inputs.Workload("copies", 76, ((256, 512), (392, 136)), "f32", 1.0, 0.02, "malt", 1)
-    run = Run(wl, check=[], w_dtypes=["bf16", "f32"])
+    wl = inputs.Workload("copies", 76, ((256, 512), (392, 136), (250, 509)), "f32", 1.0, 0.02,
+                         "malt", 1)
+    run = Run(wl, check=[], w_dtypes=["bf16", "f32", "f32"])
     c = [torch.empty(s, dtype=torch.bfloat16, device="cuda:0") for s in wl.shapes]
     with pytest.raises(malt.MaltError):
         run.opt.set_weight_copies(c)                  # W of matrix 0 is bf16
-    run.opt.set_weight_copies([None, c[1]])
+    run.opt.set_weight_copies([None, c[1], c[2]])
     run.step(oracle=False)
     assert run.status() == malt.MALT_OK
-    assert torch.equal(c[1], run.W[1].to(torch.bfloat16))
+    for i in (1, 2):
+        assert torch.equal(c[i], run.W[i].to(torch.bfloat16))
     run.opt.set_weight_copies(None)
     run.close()

@@ -114,10 +114,20 @@ def test_more_classes_than_one_launch(malt):
     check_table(tab, shapes, 3)
 
 
+def test_unaligned_shapes_use_padded_frames(malt):
+    """Rows and cols need not be multiples of 8: such a matrix runs on a
+    zero-padded copy, so its table has the tiles of the padded frame, and a
+    padded matrix shares a class with an aligned matrix of that frame."""
+    odd = [(7, 13), (100, 3), (1001, 999), (250, 509), (256, 512), (1, 1)]
+    padded = [(-(-m // 8) * 8, -(-n // 8) * 8) for m, n in odd]
+    tab = malt.malt_ns_schedule(odd, 3)
+    check_table(tab, padded, 3)
+
+
 def test_bad_arguments(malt):
     with pytest.raises(malt.MaltError):
         malt.malt_ns_schedule([(256, 512)], 0)
     with pytest.raises(malt.MaltError):
         malt.malt_ns_schedule([(256, 512)], 65)
     with pytest.raises(malt.MaltError):
-        malt.malt_ns_schedule([(250, 512)], 5)
+        malt.malt_ns_schedule([(0, 512)], 5)

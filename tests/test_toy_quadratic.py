@@ -5,6 +5,7 @@ import pytest
 
 from paper_2608_05088_gb300 import inputs
 from paper_2608_05088_gb300 import toy_quadratic as tq
+from tests import bf16_ns_model
 
 
 @pytest.mark.parametrize("kappa", [10.0, 100.0, 1e3, 1e4])
@@ -59,11 +60,11 @@ def test_gpu_steps_match_oracle_teacher_forced(kappa, optimizer):
     With bf16 Newton-Schulz operands the direction error grows with the
     condition number of Mt: rounding the entries perturbs the weak singular
     directions by about 2^-9 sigma_max / sigma_min relative to themselves, and
-    those directions still weigh in O.  The 2e-2 direction bar therefore
-    applies where cond(Mt) <= 100 (as in the GPT-2 workloads); at the badly
-    conditioned steps of kappa = 1e4 (cond(Mt) up to ~1e4, where a CPU model
-    of the same bf16 arithmetic errs by up to 18 %) only a 25 % sanity bound
-    is asserted."""
+    those directions still weigh in O.  Every checked update must be within
+    the 2e-2 bar, except where a CPU model of that same bf16 arithmetic
+    (tests/bf16_ns_model.py) errs by 1.8e-2 or more on the step (the badly
+    conditioned steps of kappa = 1e4, cond(Mt) up to ~1e4); there the GPU's
+    update must be no worse than the model's, within 25 % + 2e-3."""
     import torch
     import oracle.malt_ref as ref
     import paper_2608_05088_gb300.malt as malt
@@ -99,12 +100,15 @@ def test_gpu_steps_match_oracle_teacher_forced(kappa, optimizer):
             err = np.linalg.norm(step_gpu - info["delta"]) / np.linalg.norm(info["delta"])
             sv = np.linalg.svd(info["Mt"], compute_uv=False)
             cond = sv[0] / sv[-1]
-            bar = 2e-2 if cond <= 100 else 0.25
             checked.append((t, cond, err))
-            assert err < bar, (t, cond, err)
+            if err >= 2e-2:
+                # bf16 operands cannot resolve this step's weak directions:
+                # the GPU must be no worse than a model of that arithmetic
+                model = bf16_ns_model.step_errors(info, ref.Hyper(lr=lr))["dW"]
+                assert model >= 0.9 * 2e-2 and err <= 1.25 * model + 2e-3, (t, cond, err, model)
     assert opt.check() == malt.MALT_OK
     opt.close()
-    assert any(c <= 100 for _, c, _ in checked), checked    # the tight bar was exercised
+    assert any(e < 2e-2 for _, _, e in checked), checked    # the paper's bar was exercised
 
 
 @pytest.mark.gpu

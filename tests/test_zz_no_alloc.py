@@ -74,7 +74,8 @@ def test_noalloc_stats_match_step_and_oracle_on_two_calls(shape, g_dtype):
         torch.cuda.synchronize()
         if step > 0:      # the first call on a device may load the library's module
             assert torch.cuda.mem_get_info()[0] == free_before
-        assert torch.cuda.memory_allocated() == allocated_before
+        # torch's own count may only fall (Python freeing a tensor meanwhile)
+        assert torch.cuda.memory_allocated() <= allocated_before
         assert opt.check() == malt.MALT_OK
         L_a, R_a = opt.precond(0)
         torch.cuda.synchronize()
