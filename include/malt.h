@@ -212,6 +212,12 @@ int malt_debug_precond(malt_state_t* st, int32_t idx, float* L_out, float* R_out
  *   reduction slice, block and thread index. */
 int malt_debug_timeout_site(const malt_state_t* st, int32_t* out5);
 int malt_debug_scalars(malt_state_t* st, float* out_host, int32_t n);
+/* malt_debug_check_guards: every buffer of the state's workspace is followed
+ *   by a 256-byte guard region filled with a fixed pattern at init.  Counts,
+ *   after the state's last stream has finished, the guard bytes that no
+ *   longer hold the pattern, into *bad_bytes (host): 0 unless a kernel wrote
+ *   past one of its buffers.  Synchronises. */
+int malt_debug_check_guards(malt_state_t* st, int64_t* bad_bytes);
 
 /* Exercise the bounded device-side wait used by the kernels: launch one
  * block that waits on a flag nothing ever sets, for at most budget_ns

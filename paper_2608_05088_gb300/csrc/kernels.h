@@ -54,6 +54,12 @@ cudaError_t launch_apply(const MatDesc* mats, const UserPtrs* ptrs, const MatSca
                          const int32_t* pref, int nmat, int32_t blocks, float decay,
                          cudaStream_t s);
 cudaError_t launch_wait_probe(int32_t* status, uint64_t budget_ns, cudaStream_t s);
+// Guard regions after the workspace buffers: kGuardBytes each at the listed
+// byte offsets of base.  check = false fills them with the pattern; check =
+// true adds the number of bytes that differ from it to *bad.
+constexpr size_t kGuardBytes = 256;
+cudaError_t launch_guards(void* base, const uint64_t* offsets, int32_t n, bool check,
+                          unsigned long long* bad, cudaStream_t s);
 
 // Newton-Schulz products over up to kMaxClasses shape classes on grid_pairs
 // CTA pairs (clusters of two).  mode kNsPhased: the items

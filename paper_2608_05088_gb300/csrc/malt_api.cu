@@ -82,11 +82,18 @@ struct ShapeClass {
     CUtensorMap stX[2], stA, stB, stO, stOt;   // epilogue store maps (stOt: O as [q][p])
 };
 
+// Workspace carving: 256-byte aligned buffers, each followed by a guard
+// region that init fills with a pattern; malt_debug_check_guards counts
+// guard bytes a kernel has overwritten (an out-of-bounds write detector for
+// the tests, where no memory checker runs).
 struct Carver {
     size_t off = 0;
+    std::vector<size_t> guards;
     size_t take(size_t bytes) {
         const size_t o = off;
         off += (bytes + 255) & ~static_cast<size_t>(255);
+        guards.push_back(off);
+        off += kGuardBytes;
         return o;
     }
 };
@@ -153,6 +160,9 @@ struct malt_state {
     std::vector<NsEntry*> table_dev;
     std::vector<int32_t> table_per_iter;
     int32_t last_timeout[5] = {};   // site record of the last timeout malt_check reported
+    uint64_t* d_guard_off = nullptr;   // byte offsets of the guard regions
+    unsigned long long* d_guard_bad = nullptr;   // corrupted guard bytes found by the check
+    int32_t nguards = 0;
     cudaStream_t last_stream = nullptr;
     // Profiling: event pairs recorded around launches, folded in on read.
     bool profiling = false;
@@ -474,6 +484,12 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
     for (size_t gi = 0; gi < tables.size(); ++gi)
         o_table[gi] = cv.take(sizeof(NsEntry) * std::max<size_t>(tables[gi].size(), 1));
 
+    // The guard list itself and the check's counter (not guarded).
+    const size_t nguards = cv.guards.size();
+    const size_t o_guard_off = cv.off;
+    cv.off += (sizeof(uint64_t) * std::max<size_t>(nguards, 1) + 255) & ~static_cast<size_t>(255);
+    const size_t o_guard_bad = cv.off;
+    cv.off += 256;
     st->ws_bytes = cv.off;
     if (cudaMalloc(&st->ws, st->ws_bytes) != cudaSuccess) {
         st->ws = nullptr;
@@ -573,6 +589,17 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
 
     // Upload the static tables (init is allowed to synchronise).
     MALT_CUDA(cudaMemset(st->ws, 0, st->ws_bytes), "cudaMemset(workspace)");
+    st->d_guard_off = reinterpret_cast<uint64_t*>(base + o_guard_off);
+    st->d_guard_bad = reinterpret_cast<unsigned long long*>(base + o_guard_bad);
+    st->nguards = static_cast<int32_t>(nguards);
+    if (nguards > 0) {
+        std::vector<uint64_t> goff(cv.guards.begin(), cv.guards.end());
+        MALT_CUDA(cudaMemcpy(st->d_guard_off, goff.data(), sizeof(uint64_t) * nguards,
+                             cudaMemcpyHostToDevice), "cudaMemcpy(guards)");
+        MALT_CUDA(launch_guards(base, st->d_guard_off, st->nguards, false, st->d_guard_bad, nullptr),
+                  "guard_kernel (fill)");
+        MALT_CUDA(cudaDeviceSynchronize(), "cudaDeviceSynchronize(guards)");
+    }
     if (n > 0) {
         MALT_CUDA(cudaMemcpy(st->d_mats, st->hmats.data(), sizeof(MatDesc) * n,
                              cudaMemcpyHostToDevice), "cudaMemcpy(mats)");
@@ -1032,6 +1059,22 @@ int malt_debug_precond(malt_state_t* st, int32_t idx, float* L_out, float* R_out
               "cudaMemcpyAsync(L)");
     MALT_CUDA(cudaMemcpyAsync(R_out, d.R, sizeof(float) * p.cols, cudaMemcpyDeviceToDevice, s),
               "cudaMemcpyAsync(R)");
+    return MALT_OK;
+}
+
+int malt_debug_check_guards(malt_state_t* st, int64_t* bad_bytes) {
+    if (st == nullptr || bad_bytes == nullptr) return MALT_ERR_INVALID_ARG;
+    *bad_bytes = 0;
+    if (st->nguards == 0) return MALT_OK;
+    cudaStream_t s = st->last_stream;
+    MALT_CUDA(cudaMemsetAsync(st->d_guard_bad, 0, sizeof(unsigned long long), s), "cudaMemsetAsync(guard count)");
+    MALT_CUDA(launch_guards(st->ws, st->d_guard_off, st->nguards, true, st->d_guard_bad, s),
+              "guard_kernel (check)");
+    unsigned long long bad = 0;
+    MALT_CUDA(cudaMemcpyAsync(&bad, st->d_guard_bad, sizeof(bad), cudaMemcpyDeviceToHost, s),
+              "cudaMemcpyAsync(guard count)");
+    MALT_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+    *bad_bytes = static_cast<int64_t>(bad);
     return MALT_OK;
 }
 

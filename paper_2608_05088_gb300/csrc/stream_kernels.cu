@@ -166,6 +166,25 @@ __global__ void wait_probe_kernel(int32_t* status, uint64_t budget_ns) {
     }
 }
 
+// ----------------------------------------------------------------- guards
+constexpr uint32_t kGuardWord = 0xA5C3E10Fu;
+
+// One block per guard region, one thread per 32-bit word.
+__global__ void guard_kernel(uint8_t* base, const uint64_t* __restrict__ offsets, bool check,
+                             unsigned long long* bad) {
+    uint32_t* g = reinterpret_cast<uint32_t*>(base + offsets[blockIdx.x]);
+    const int i = threadIdx.x;
+    if (!check) {
+        g[i] = kGuardWord;
+        return;
+    }
+    const uint32_t diff = g[i] ^ kGuardWord;
+    int nbytes = 0;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) nbytes += ((diff >> (8 * k)) & 0xffu) != 0;
+    if (nbytes != 0) atomicAdd(bad, static_cast<unsigned long long>(nbytes));
+}
+
 // ------------------------------------------------------------------ launch
 cudaError_t launch_bind(const BindParams& P, UserPtrs* table, cudaStream_t s) {
     bind_kernel<<<1, kBindChunk, 0, s>>>(P, table);
@@ -223,6 +242,13 @@ cudaError_t launch_apply(const MatDesc* mats, const UserPtrs* ptrs, const MatSca
     return cudaGetLastError();
 }
 
+
+cudaError_t launch_guards(void* base, const uint64_t* offsets, int32_t n, bool check,
+                          unsigned long long* bad, cudaStream_t s) {
+    guard_kernel<<<n, static_cast<int>(kGuardBytes / 4), 0, s>>>(static_cast<uint8_t*>(base), offsets,
+                                                                 check, bad);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_wait_probe(int32_t* status, uint64_t budget_ns, cudaStream_t s) {
     wait_probe_kernel<<<1, 32, 0, s>>>(status, budget_ns);

@@ -34,7 +34,8 @@ EXPORTS = ("malt_init_state", "malt_step", "malter_step", "malt_get_scalars",
            "malt_stats_noalloc", "malt_step_host", "muon_step", "malt_set_ns_schedule",
            "malt_ns_schedule", "malt_debug_timeout_site", "malt_debug_precond",
            "malt_set_weight_copies", "malt_adamw_init_state", "malt_adamw_step",
-           "malt_adamw_get_step", "malt_adamw_set_step", "malt_adamw_destroy_state")
+           "malt_adamw_get_step", "malt_adamw_set_step", "malt_adamw_destroy_state",
+           "malt_debug_check_guards")
 NOALLOC_SCRATCH_FLOATS = 1048576
 KIND_NAMES = ("bind", "stats", "finalize", "prescale", "norms", "ns_gram", "ns_poly", "ns_bx",
               "scalars", "apply", "ns_persistent", "pad")
@@ -130,6 +131,8 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.malt_set_ns_schedule.argtypes = [vp, i32]
     lib.malt_set_ns_schedule.restype = ctypes.c_int
     lib.malt_ns_schedule.argtypes = [P(malt_param_t), i32, i32, P(i32), i64, P(i64)]
+    lib.malt_debug_check_guards.argtypes = [vp, P(i64)]
+    lib.malt_debug_check_guards.restype = ctypes.c_int
     lib.malt_set_weight_copies.argtypes = [vp, P(vp), i32]
     lib.malt_set_weight_copies.restype = ctypes.c_int
     lib.malt_adamw_init_state.argtypes = [P(vp), P(malt_adamw_param_t), i32, vp]
@@ -262,6 +265,14 @@ def malt_debug_precond(st, idx: int, L_out, R_out, stream=None):
     _check(load().malt_debug_precond(st, idx, ctypes.c_void_p(L_out.data_ptr()),
                                      ctypes.c_void_p(R_out.data_ptr()), _stream_handle(stream)),
            "malt_debug_precond")
+
+
+def malt_debug_check_guards(st) -> int:
+    """Corrupted bytes in the workspace's guard regions (0 when no kernel
+    wrote past its buffers)."""
+    bad = ctypes.c_int64()
+    _check(load().malt_debug_check_guards(st, ctypes.byref(bad)), "malt_debug_check_guards")
+    return int(bad.value)
 
 
 def malt_debug_scalars(st, n: int) -> np.ndarray:
@@ -487,6 +498,9 @@ class MaltOptimizer:
         R = torch.empty(W.shape[1], dtype=torch.float32, device=W.device)
         malt_debug_precond(self.state, idx, L, R, stream)
         return L, R
+
+    def guard_bytes_corrupted(self) -> int:
+        return malt_debug_check_guards(self.state)
 
     def timeout_site(self):
         return malt_debug_timeout_site(self.state)

@@ -7,20 +7,15 @@ warmup-stable-decay schedule (for 5000 steps: linear warmup to lr_max over
 steps run through the library's C ABI (malt_step or muon_step); the gradient
 of the toy loss is the "model" and is formed with torch on the device.
 
-X (r x r) is embedded in an 8 x 8 zero-padded matrix because the library
-takes rows and columns in multiples of 8.  The embedding is exact: padded
-rows and columns get zero gradient, hence zero momentum, zero preconditioned
-momentum and zero Newton-Schulz output, and the graft norms are those of the
-r x r block.
+X is passed at its own r x r shape; the library runs matrices whose sizes
+are not multiples of 8 on zero-padded copies, with the results of the
+unpadded matrix.
 """
 from __future__ import annotations
 
 import numpy as np
 
 from . import inputs
-
-PAD = 8
-
 
 def wsd_lr(t: int, total: int = 5000, lr_max: float = 1e-3) -> float:
     """Learning rate of 0-based step t under the warmup-stable-decay schedule:
@@ -55,28 +50,26 @@ def run_gpu(kappa: float, optimizer: str = "malt", steps: int = 5000, lr_max: fl
     A, B, C = inputs.toy_quadratic_problem(kappa, seed=seed)
     r = A.shape[1]
     dev = torch.device("cuda")
-    At = torch.zeros((A.shape[0], PAD), dtype=torch.float32, device=dev)
-    Bt = torch.zeros((B.shape[0], PAD), dtype=torch.float32, device=dev)
-    At[:, :r] = torch.from_numpy(A).float()
-    Bt[:, :r] = torch.from_numpy(B).float()
+    At = torch.from_numpy(A).float().to(dev)
+    Bt = torch.from_numpy(B).float().to(dev)
     Ct = torch.from_numpy(C).float().to(dev)
-    X = torch.zeros((PAD, PAD), dtype=torch.float32, device=dev)
+    X = torch.zeros((r, r), dtype=torch.float32, device=dev)
     G = torch.zeros_like(X)
     M = torch.empty_like(X)
-    l = torch.empty(PAD, dtype=torch.float32, device=dev)
-    rr = torch.empty(PAD, dtype=torch.float32, device=dev)
+    l = torch.empty(r, dtype=torch.float32, device=dev)
+    rr = torch.empty(r, dtype=torch.float32, device=dev)
     opt = malt.MaltOptimizer([(X, G, M, l, rr)])
     _, fstar = optimum(A, B, C)
     ts, gaps = [], []
     for t in range(steps):
         if t % record_every == 0:
             ts.append(t)
-            gaps.append(objective(A, B, C, X[:r, :r].double().cpu().numpy()) - fstar)
+            gaps.append(objective(A, B, C, X.double().cpu().numpy()) - fstar)
         G.copy_(torch.mm(torch.mm(At.T, torch.mm(torch.mm(At, X), Bt.T) - Ct), Bt))
         hp = malt.hparams(lr=wsd_lr(t, steps, lr_max=lr_max), ns_steps=ns_steps)
         opt.step(hp, muon=(optimizer == "muon"))
     ts.append(steps)
-    Xf = X[:r, :r].double().cpu().numpy()
+    Xf = X.double().cpu().numpy()
     gaps.append(objective(A, B, C, Xf) - fstar)
     status = opt.check()
     opt.close()

@@ -57,8 +57,30 @@ def bf16_rounding(W_gpu, x_gpu, x_ref, slack, dW_ref):
                 straddle=float(np.mean(straddle)), straddle_allowed=allowed)
 
 
+CANARY = 64                    # elements of margin before and after every caller buffer
+CANARY_VALUE = -7.625e7         # a value no step writes (exact in fp32 and bf16)
+
+
+def guarded(shape, dtype, device):
+    """A contiguous tensor of `shape` inside a larger allocation whose CANARY
+    elements before and after hold CANARY_VALUE (16-byte aligned: the margin
+    is 256 bytes in fp32, 128 in bf16).  Returns (tensor, whole allocation)."""
+    import torch
+    n = int(np.prod(shape))
+    buf = torch.full((n + 2 * CANARY,), CANARY_VALUE, dtype=dtype, device=device)
+    return buf[CANARY:CANARY + n].view(shape), buf
+
+
+def canaries_intact(buf) -> bool:
+    import torch
+    return bool(torch.all(buf[:CANARY] == CANARY_VALUE) and torch.all(buf[-CANARY:] == CANARY_VALUE))
+
+
 class Run:
-    """One optimizer state on the GPU plus oracle states for `check` matrices."""
+    """One optimizer state on the GPU plus oracle states for `check` matrices.
+    Every caller buffer (W, G, M, l, r) sits between canary margins, and
+    close() checks them and the library's workspace guards: a kernel that
+    writes past any buffer fails the test."""
 
     def __init__(self, wl: inputs.Workload, check=None, g_dtype="f32", w_dtypes=None,
                  variant=None, device="cuda:0", ns_coeffs=ref.DEFAULT_NS_COEFFS, **hyper):
@@ -75,17 +97,22 @@ class Run:
         tdt = {"f32": torch.float32, "bf16": torch.bfloat16}
         self.W0 = {}
         self.W, self.G, self.M, self.l, self.r = [], [], [], [], []
+        self.bufs = []
         for i, (m, c) in enumerate(wl.shapes):
             w0 = inputs.initial_weight(wl, i)
             if self.w_dtypes[i] == "bf16":
                 w0 = inputs.bf16_representable(w0)
             if i in self.check:
                 self.W0[i] = w0.astype(np.float64)
-            self.W.append(torch.from_numpy(w0).to(self.dev).to(tdt[self.w_dtypes[i]]))
-            self.G.append(torch.zeros((m, c), dtype=tdt[g_dtype], device=self.dev))
-            self.M.append(torch.empty((m, c), dtype=torch.float32, device=self.dev))
-            self.l.append(torch.empty(m, dtype=torch.float32, device=self.dev))
-            self.r.append(torch.empty(c, dtype=torch.float32, device=self.dev))
+            for lst, shape, dt in ((self.W, (m, c), tdt[self.w_dtypes[i]]),
+                                   (self.G, (m, c), tdt[g_dtype]),
+                                   (self.M, (m, c), torch.float32), (self.l, (m,), torch.float32),
+                                   (self.r, (c,), torch.float32)):
+                t, buf = guarded(shape, dt, self.dev)
+                lst.append(t)
+                self.bufs.append(buf)
+            self.W[-1].copy_(torch.from_numpy(w0))
+            self.G[-1].zero_()
         self.params = list(zip(self.W, self.G, self.M, self.l, self.r))
         self.opt = malt.MaltOptimizer(self.params)
         # Extra hyperparameters (mu1, mu2, eps, weight_decay, ns_eps) go to both
@@ -226,4 +253,9 @@ class Run:
         return e
 
     def close(self):
+        """Check that no kernel wrote outside its buffers, then free the state."""
+        self.torch.cuda.synchronize()
+        assert self.opt.guard_bytes_corrupted() == 0, "a kernel wrote past a workspace buffer"
+        for k, buf in enumerate(self.bufs):
+            assert canaries_intact(buf), f"a kernel wrote past caller buffer {k} (W, G, M, l, r per matrix)"
         self.opt.close()

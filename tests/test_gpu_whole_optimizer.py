@@ -19,7 +19,7 @@ import oracle.adamw_ref as aref
 import oracle.malt_ref as ref
 import paper_2608_05088_gb300.malt as malt
 from paper_2608_05088_gb300 import inputs
-from tests.gpu_harness import Run
+from tests.gpu_harness import Run, canaries_intact, guarded
 
 pytestmark = pytest.mark.gpu
 
@@ -48,12 +48,20 @@ class AdamRun:
         self.shapes, self.wds, self.lr, self.g_dtype = shapes, wds, lr, g_dtype
         gdt = torch.float32 if g_dtype == "f32" else torch.bfloat16
         self.w0 = [(self.rng.standard_normal(s) * 0.02).astype(np.float32) for s in shapes]
-        self.w = [torch.from_numpy(x).to(dev) for x in self.w0]
-        self.wc = [torch.empty(s, dtype=torch.bfloat16, device=dev) if copies else None
-                   for s in shapes]
-        self.g = [torch.zeros(s, dtype=gdt, device=dev) for s in shapes]
-        self.m = [torch.empty(s, dtype=torch.float32, device=dev) for s in shapes]
-        self.v = [torch.empty(s, dtype=torch.float32, device=dev) for s in shapes]
+        # every buffer between canary margins (checked by close())
+        self.bufs = []
+
+        def buf(shape, dt):
+            t, b = guarded(shape, dt, dev)
+            self.bufs.append(b)
+            return t
+        self.w = [buf(s, torch.float32) for s in shapes]
+        for t, x in zip(self.w, self.w0):
+            t.copy_(torch.from_numpy(x))
+        self.wc = [buf(s, torch.bfloat16) if copies else None for s in shapes]
+        self.g = [buf(s, gdt).zero_() for s in shapes]
+        self.m = [buf(s, torch.float32) for s in shapes]
+        self.v = [buf(s, torch.float32) for s in shapes]
         self.params = list(zip(self.w, self.wc, self.g, self.m, self.v, wds))
         self.opt = malt.AdamW(self.params, stream)
         f32 = lambda x: float(np.float32(x))
@@ -61,6 +69,12 @@ class AdamRun:
         self.hp_ref = aref.AdamWHyper(lr=f32(lr), beta1=f32(0.9), beta2=f32(0.95), eps=f32(1e-8))
         self.w_ref = [x.astype(np.float64) for x in self.w0]
         self.st_ref = [aref.AdamWState.zeros(s) for s in shapes]
+
+    def close(self):
+        self.torch.cuda.synchronize()
+        for k, b in enumerate(self.bufs):
+            assert canaries_intact(b), f"a kernel wrote past AdamW buffer {k}"
+        self.opt.close()
 
     def draw(self):
         gs = []
@@ -127,7 +141,7 @@ def test_adamw_against_oracle_ragged_sizes():
         for i in range(len(shapes)):
             run.check(i, f"step {s}")
     assert run.opt.get_step() == 4
-    run.opt.close()
+    run.close()
 
 
 def test_adamw_bf16_gradients_without_copies():
@@ -138,7 +152,7 @@ def test_adamw_bf16_gradients_without_copies():
         run.torch.cuda.synchronize()
         for i in range(len(shapes)):
             run.check(i, f"step {s}")
-    run.opt.close()
+    run.close()
 
 
 def test_adamw_zero_gradient_is_pure_decay():
@@ -157,7 +171,7 @@ def test_adamw_zero_gradient_is_pure_decay():
             want = (want * decay).astype(np.float32)
         assert np.array_equal(run.w[i].cpu().numpy(), want)
         assert not torch.any(run.m[i]) and not torch.any(run.v[i])
-    run.opt.close()
+    run.close()
 
 
 def test_adamw_checkpoint_and_graph_replay():
@@ -198,8 +212,8 @@ def test_adamw_checkpoint_and_graph_replay():
     for i in range(2):
         for x, y in ((a.w[i], c.w[i]), (a.m[i], c.m[i]), (a.v[i], c.v[i]), (a.wc[i], c.wc[i])):
             assert torch.equal(x, y)
-    a.opt.close()
-    c.opt.close()
+    a.close()
+    c.close()
 
 
 def test_adamw_rejects_changed_sizes():
@@ -211,7 +225,7 @@ def test_adamw_rejects_changed_sizes():
     with pytest.raises(malt.MaltError):
         run.opt.step(run.hp, params=other)
     torch.cuda.synchronize()
-    run.opt.close()
+    run.close()
 
 
 def test_whole_optimizer_gpt2_small():
@@ -249,7 +263,7 @@ def test_whole_optimizer_gpt2_small():
         for i in range(len(wl.shapes)):
             assert torch.equal(copies[i], mats.W[i].to(torch.bfloat16))
     mats.close()
-    adam.opt.close()
+    adam.close()
 
 
 def test_weight_copies_need_fp32_weights():
