@@ -52,3 +52,20 @@ def test_wrong_gpu_rounding_is_caught_even_when_it_matches_the_oracle():
     W = ref.round_to_bf16(x_ref)
     r = bf16_rounding(W, x_gpu, x_ref, slack, dW_ref)
     assert r["own_mismatch"] > 0
+
+
+def test_canary_margins_catch_writes_past_a_buffer():
+    """The harness's caller buffers sit between canary margins; a write just
+    before or just past a buffer (planted here, on the CPU) is caught, writes
+    inside it are not."""
+    import torch
+    from tests.gpu_harness import CANARY, canaries_intact, guarded
+    for dtype in (torch.float32, torch.bfloat16):
+        t, buf = guarded((5, 7), dtype, "cpu")
+        assert t.is_contiguous() and t.data_ptr() % 16 == 0 and canaries_intact(buf)
+        t.fill_(3.0)
+        assert canaries_intact(buf)
+        for k in (CANARY - 1, CANARY + t.numel()):      # just before, just after
+            _, b2 = guarded((5, 7), dtype, "cpu")
+            b2[k] = 1.0
+            assert not canaries_intact(b2), (dtype, k)
