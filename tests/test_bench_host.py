@@ -153,12 +153,17 @@ def test_clock_summary_fallbacks():
 
 
 def test_roofline_traffic_holds_only_for_the_captured_kernel(tmp_path, monkeypatch):
-    """roofline.traffic comes from the committed ncu summary only while every
-    source the Newton-Schulz kernel compiles from is the one it was captured
-    with; a changed source makes it null."""
+    """roofline.traffic comes from an ncu summary only while every source the
+    Newton-Schulz kernel compiles from is the one it was captured with; a
+    changed source makes it null."""
     sys.path.insert(0, ROOT)
     import bench
-    assert bench.ncu_traffic_per_launch(False) is not None
+    summary = tmp_path / "ncu.json"
+    summary.write_text(json.dumps({"ns_sources_sha256": bench.ns_sources_sha256(),
+                                   "dram_bytes_per_launch_full_size": 1.5e9}))
+    monkeypatch.setattr(bench, "NCU_SUMMARY", str(summary))
+    assert bench.ncu_traffic_per_launch(False) == 1.5e9
+    assert bench.ncu_traffic_per_launch(True) is None          # no figure for that schedule
     changed = tmp_path / "common.cuh"
     changed.write_bytes(open(bench.NS_SOURCES[1], "rb").read() + b"// edited\n")
     monkeypatch.setattr(bench, "NS_SOURCES", [bench.NS_SOURCES[0], str(changed), bench.NS_SOURCES[2]])
