@@ -197,6 +197,25 @@ def peaks():
         return FALLBACK_PEAKS, "fallback"
 
 
+def ncu_tensor_pipe():
+    """Tensor-pipe busy % of peak of the Gram, Poly and B*X launches from the
+    committed ncu summary, weighted by their captured durations (the NS mix
+    of one iteration), or None when a kernel source changed since."""
+    try:
+        with open(NCU_SUMMARY) as f:
+            s = json.load(f)
+        if s.get("ns_sources_sha256") != ns_sources_sha256():
+            return None
+        tp = s["tensor_pipe_pct_of_peak_elapsed"]
+        dur = tp["durations_us"]
+        kinds = ("gram", "poly", "bx")
+        mix = sum(tp[k] * dur[k] for k in kinds) / sum(dur[k] for k in kinds)
+        return {"per_product": {k: tp[k] for k in kinds}, "duration_weighted": round(mix, 2),
+                "source": "ncu, first 12 GPT-2 Large layers (profiles/ns_gemm_gpt2_large_first12l.md)"}
+    except Exception:
+        return None
+
+
 def ncu_traffic_per_launch(persistent: bool):
     """DRAM bytes per NS GEMM launch (of the schedule the timed steps used)
     from the committed ncu summary, or None when a kernel source changed
@@ -716,6 +735,7 @@ def run_malt(args):
                 # what the tensor cores execute: symmetric products as whole
                 # 256 x 256 tiles on and above the diagonal
                 "issued_tflops": wl.ns_flops_issued() * args.steps / (ns_ms / 1e3) / 1e12,
+                "tensor_pipe_pct_ncu": ncu_tensor_pipe() if wl.name.startswith("gpt2_large") else None,
                 "launch_avg_ms": ns_ms / max(ns_launches, 1)}
     elems = wl.elements
     wbytes = 2 if wl.weight_dtype == "bf16" else 4
