@@ -27,6 +27,8 @@
 #include <cstring>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "../../include/malt.h"
 
 namespace {
@@ -215,6 +217,12 @@ struct malt_adamw_state {
     cudaStream_t last_stream = nullptr;
 };
 
+namespace {
+// Bind launches and the update launch of one step (after validation).
+int enqueue_adamw(malt_adamw_state* st, const malt_adamw_param_t* params, int32_t n,
+                  const malt_adamw_hparams_t* hp, cudaStream_t s);
+}  // namespace
+
 extern "C" {
 
 int malt_adamw_init_state(malt_adamw_state_t** out, const malt_adamw_param_t* params, int32_t n,
@@ -297,6 +305,18 @@ int malt_adamw_step(malt_adamw_state_t* st, const malt_adamw_param_t* params, in
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     st->last_stream = s;
     ADAM_CUDA(cudaSetDevice(st->device), "cudaSetDevice");
+    nvtxRangePushA("malt_adamw_step");
+    const int rc = enqueue_adamw(st, params, n, hp, s);
+    nvtxRangePop();
+    return rc;
+}
+
+}  // extern "C"
+
+namespace {
+
+int enqueue_adamw(malt_adamw_state* st, const malt_adamw_param_t* params, int32_t n,
+                  const malt_adamw_hparams_t* hp, cudaStream_t s) {
     AdamBind B;
     for (int off = 0; off == 0 || off < n; off += kAdamBindChunk) {
         const int cnt = std::min(kAdamBindChunk, n - off);
@@ -320,6 +340,10 @@ int malt_adamw_step(malt_adamw_state_t* st, const malt_adamw_param_t* params, in
     ADAM_CUDA(cudaGetLastError(), "adamw_kernel");
     return MALT_OK;
 }
+
+}  // namespace
+
+extern "C" {
 
 int malt_adamw_get_step(malt_adamw_state_t* st, int64_t* t_host) {
     if (st == nullptr || t_host == nullptr) return MALT_ERR_INVALID_ARG;

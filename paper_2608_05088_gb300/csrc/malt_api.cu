@@ -16,6 +16,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <algorithm>
 #include <cstdio>
@@ -245,15 +246,28 @@ cudaEvent_t take_event(malt_state* st) {
     return e;
 }
 
+// NVTX range names of the kernel kinds (MALT_KIND_*), for timeline tools.
+const char* const kKindRange[MALT_NUM_KINDS] = {
+    "malt:bind", "malt:stats", "malt:finalize", "malt:prescale", "malt:norms", "malt:ns_gram",
+    "malt:ns_poly", "malt:ns_bx", "malt:scalars", "malt:apply", "malt:ns_persistent", "malt:pad"};
+
+// An NVTX range over a scope (host-side enqueue; a timeline tool maps it to
+// the GPU work it launches).  Costs a pointer check when no tool is attached.
+struct NvtxRange {
+    explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+};
+
 // Bracket one launch (or launch group) of a kernel kind with events when
-// profiling is on; always counts the launches.
+// profiling is on, and with an NVTX range; always counts the launches.
 struct LaunchScope {
     malt_state* st;
     int kind;
     cudaStream_t s;
     cudaEvent_t a = nullptr;
+    NvtxRange range;
     LaunchScope(malt_state* st_, int kind_, cudaStream_t s_, int launches = 1)
-        : st(st_), kind(kind_), s(s_) {
+        : st(st_), kind(kind_), s(s_), range(kKindRange[kind_]) {
         st->prof_launches[kind] += launches;
         if (st->profiling) {
             a = take_event(st);
@@ -779,6 +793,7 @@ StepHyper step_hyper(const malt_hparams_t* hp, int malter) {
 
 int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_hparams_t* hp,
              void* stream, int flavour, const PipeHooks* hooks = nullptr) {
+    const NvtxRange range(flavour == kMalter ? "malter_step" : flavour == kMuon ? "muon_step" : "malt_step");
     const int malter = flavour == kMalter ? 1 : 0;
     const int muon = flavour == kMuon ? 1 : 0;
     int rc = validate_step(st, params, n, hp);
