@@ -71,6 +71,49 @@ def barrier():
         dist.barrier()
 
 
+def host_link_bound(g_host, g_dev, w_dev, w_host, step_ms, e2e_per_gpu, reps=3):
+    """The host link's bound on the end-to-end rate: the same per-tensor
+    copies as one host step (every gradient in, every weight out), timed
+    alone in each direction and both directions at once, with no kernels
+    running.  A pipelined host step can go no faster than the slower of the
+    device-resident step and the concurrent copies."""
+    import torch
+    up, down = torch.cuda.Stream(), torch.cuda.Stream()
+
+    def h2d():
+        with torch.cuda.stream(up):
+            for d, h in zip(g_dev, g_host):
+                d.copy_(h, non_blocking=True)
+
+    def d2h():
+        with torch.cuda.stream(down):
+            for h, d in zip(w_host, w_dev):
+                h.copy_(d, non_blocking=True)
+
+    def both():
+        h2d()
+        d2h()
+
+    def wall_ms(fn):
+        fn()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(reps):
+            fn()
+        torch.cuda.synchronize()
+        return (time.perf_counter() - t0) * 1e3 / reps
+
+    bi = sum(t.numel() * t.element_size() for t in g_host)
+    bo = sum(t.numel() * t.element_size() for t in w_host)
+    t_in, t_out, t_both = wall_ms(h2d), wall_ms(d2h), wall_ms(both)
+    bound_ms = max(step_ms, t_both)
+    return {"h2d_gbs": bi / t_in / 1e6, "d2h_gbs": bo / t_out / 1e6,
+            "concurrent_ms": t_both, "device_step_ms": step_ms,
+            "bound_steps_per_s": 1e3 / bound_ms,
+            "frac": e2e_per_gpu * bound_ms / 1e3,
+            "bound": "host link" if t_both > step_ms else "device step"}
+
+
 def max_over_ranks(x: float, device=None) -> float:
     """Maximum of a host scalar over all ranks (timing only, never data)."""
     import torch
@@ -690,8 +733,11 @@ def run_malt(args):
         torch.cuda.synchronize()
         barrier()
         t0 = time.perf_counter()
+        ends = []
         for s_ in range(args.steps):
             opt.step_host(hp, G_host, W_host, malter=malter, params=param_sets[s_ % 2])
+            ends.append(torch.cuda.Event(enable_timing=True))
+            ends[-1].record(stream)           # the end of the step's kernels
         status = opt.check()                  # waits for the compute and both copy streams
         torch.cuda.synchronize()
         te = time.perf_counter() - t0
@@ -702,6 +748,15 @@ def run_malt(args):
                "api": "malt_step_host (copies overlapped with compute)"}
         if status != malt.MALT_OK:
             raise SystemExit("e2e step failed")
+        link = host_link_bound(G_host, G2, W, W_host, t_ms / args.steps, e2e["value"] / world)
+        # Steady state: the spacing of consecutive steps' ends, once the
+        # pipeline is full (the timed region also holds its fill and drain:
+        # the first step's gradient copy and the last step's weight copy).
+        gaps = [a.elapsed_time(b) for a, b in zip(ends[1:], ends[2:])]
+        if gaps:
+            link["pipelined_ms_per_step"] = statistics.median(gaps)
+            link["pipelined_frac_of_bound"] = 1e3 / link["bound_steps_per_s"] / link["pipelined_ms_per_step"]
+        e2e["link"] = link
 
     if rank != 0:
         return

@@ -224,10 +224,15 @@ __device__ __forceinline__ void finalize_entry(const MatDesc& d, const UserPtrs&
 // the statistics pass (warp w owns 8 rows, lane 8 consecutive columns, four
 // rows of loads in flight) and written as bf16 in place of its NS frame; a
 // tall matrix's NS frame is Mt^T, so its block walks four 64 x 64 sub-tiles
-// through shared memory (tile: 64 x 65 floats) and writes each transposed.
+// through shared memory and writes each transposed.
+// tile: two 64 x 64 float buffers (kPreTileFloats, 16-byte aligned), used in
+// turn.  Row r of a buffer holds its 16 float4 chunks XOR-permuted by
+// (r / 8) mod 8, so that both the row-wise float4 writes and the column-wise
+// reads (eight rows 8 apart per warp) hit 32 distinct banks.
 // red: 8 float2.
+constexpr int kPreTileFloats = 2 * 64 * 64;
 __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs& up, int local,
-                                               int malter, int tid, float (*tile)[65],
+                                               int malter, int tid, float* tile,
                                                float2* red) {
     constexpr int P = kLdPlain;
     const int m = d.m, n = d.n;
@@ -325,6 +330,7 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
             const int cs = c0 + sub * 64;
             if (cs >= n) break;                          // uniform across the block
             const int col = cs + cc;
+            float* __restrict__ tb = tile + (sub & 1) * (64 * 64);
             float4 R4 = make_float4(0.f, 0.f, 0.f, 0.f);
             if (col < n) R4 = ld_f4<P>(Rv + col);
 #pragma unroll
@@ -359,26 +365,29 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
                         s_lgr = fmaf(a3, a3, fmaf(a2, a2, fmaf(a1, a1, fmaf(a0, a0, s_lgr))));
                     }
                 }
-                tile[rr][cc + 0] = v0; tile[rr][cc + 1] = v1;
-                tile[rr][cc + 2] = v2; tile[rr][cc + 3] = v3;
+                *reinterpret_cast<float4*>(tb + rr * 64 + (((t & 15) ^ ((rr >> 3) & 7)) << 2)) =
+                    make_float4(v0, v1, v2, v3);
             }
             if (sub + 2 < kSubs) load_sub(sub + 2, mq[sub & 1]);
+            // One barrier per sub-tile: the buffer written next was last read
+            // two sub-tiles ago, before every thread passed the previous barrier.
             __syncthreads();
-            // Output row = column of Mt, 8 consecutive rows of Mt per thread.
+            // Output row = column of Mt, 8 consecutive rows of Mt per thread;
+            // those rows share one chunk permutation, t mod 8.
+            const int seg = (t & 7) * 8, sw = t & 7;
 #pragma unroll
             for (int pass = 0; pass < 2; ++pass) {
                 const int oc = pass * 32 + (t >> 3);
-                const int seg = (t & 7) * 8;
                 const int gcol = cs + oc, grow = r0 + seg;
                 if (gcol < n && grow < m) {
+                    const int pc = ((((oc >> 2) ^ sw) << 2) | (oc & 3));
                     float v[8];
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) v[j] = tile[seg + j][oc];
+                    for (int j = 0; j < 8; ++j) v[j] = tb[(seg + j) * 64 + pc];
                     *reinterpret_cast<uint4*>(d.X0 + static_cast<size_t>(gcol) * m + grow) =
                         pack8_bf16(v);
                 }
             }
-            __syncthreads();                                       // tile is reused by the next sub-tile
         }
     }
     // One fixed-order reduction of both partial sums.

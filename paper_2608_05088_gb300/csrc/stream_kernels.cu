@@ -112,10 +112,10 @@ finalize_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ p
 }
 
 // --------------------------------------------------------------- prescale
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(256, 3)
 prescale_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
                 const int32_t* __restrict__ pref, int nmat, int malter) {
-    __shared__ float tile[64][65];
+    __shared__ __align__(16) float tile[blk::kPreTileFloats];
     __shared__ float2 red[8];
     const int g = find_mat(pref, nmat, blockIdx.x);
     blk::prescale_block(mats[g], ptrs[g], blockIdx.x - __ldg(pref + g), malter, threadIdx.x, tile,
