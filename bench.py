@@ -71,7 +71,7 @@ def barrier():
         dist.barrier()
 
 
-def host_link_bound(g_host, g_dev, w_dev, w_host, step_ms, e2e_per_gpu, reps=3):
+def host_link_bound(g_host, g_dev, w_dev, w_host, step_ms, e2e_per_gpu, reps=5):
     """The host link's bound on the end-to-end rate: the same per-tensor
     copies as one host step (every gradient in, every weight out), timed
     alone in each direction and both directions at once, with no kernels
@@ -95,13 +95,17 @@ def host_link_bound(g_host, g_dev, w_dev, w_host, step_ms, e2e_per_gpu, reps=3):
         d2h()
 
     def wall_ms(fn):
+        # median of single runs: the host link on these machines now and then
+        # stalls a copy for tens of milliseconds
         fn()
         torch.cuda.synchronize()
-        t0 = time.perf_counter()
+        times = []
         for _ in range(reps):
+            t0 = time.perf_counter()
             fn()
-        torch.cuda.synchronize()
-        return (time.perf_counter() - t0) * 1e3 / reps
+            torch.cuda.synchronize()
+            times.append((time.perf_counter() - t0) * 1e3)
+        return statistics.median(times)
 
     bi = sum(t.numel() * t.element_size() for t in g_host)
     bo = sum(t.numel() * t.element_size() for t in w_host)

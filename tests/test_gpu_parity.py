@@ -12,7 +12,7 @@ import numpy as np
 import pytest
 
 from paper_2608_05088_gb300 import inputs
-from tests.gpu_harness import Run
+from tests.gpu_harness import Run, bf16_rounding
 
 pytestmark = pytest.mark.gpu
 
@@ -181,12 +181,22 @@ def test_gpt2_medium_malter_sampled():
 
 def test_gpt2_large_bench_configuration():
     """The benchmark's own configuration: all 144 GPT-2 Large matrices in one
-    grouped step (bf16 W, fp32 state, 5 NS iterations), 2 MALT steps.  One
-    matrix of each shape is checked in full against the oracle; every
-    matrix's statistics l, r against fp64 row / column sums of its
-    gradients (a property that holds at any size)."""
+    grouped step (bf16 W, fp32 state, 5 NS iterations), 2 MALT steps.
+
+    * Ten matrices, every shape of the first, a middle and the last layer
+      (the first and last entries of the launch's work lists), are checked in
+      full against the oracle.
+    * Every matrix's statistics l, r against fp64 row / column sums of its
+      gradients.
+    * Every matrix's graft and update against the step's own intermediates
+      (properties that hold at any size): ||O||_F and ||D||_F = ||L O R||_F
+      from the last GEMM epilogue's partial sums against fp64 norms of the
+      step's O, L, R (Algorithm 1, graft line), and the stored bf16 W against
+      the round-to-nearest-even of W_prev - s L O R with the step's scale s
+      (Algorithm 1, update line)."""
+    import torch
     wl = inputs.WORKLOADS["gpt2_large"]
-    check = [0, 1, 2, 3]
+    check = [0, 1, 2, 3, 69, 70, 140, 141, 142, 143]
     run = Run(wl, check=check)
     sq_rows = {}
     sq_cols = {}
@@ -198,16 +208,30 @@ def test_gpt2_large_bench_configuration():
             r_, c_ = np.sum(G64 * G64, axis=1), np.sum(G64 * G64, axis=0)
             sq_rows[i] = mu2 * sq_rows.get(i, 0.0) + (1 - mu2) * r_
             sq_cols[i] = mu2 * sq_cols.get(i, 0.0) + (1 - mu2) * c_
+        if s == 1:
+            w_prev = [w.cpu() for w in run.W]
         run.step(grads=grads)
     assert run.status() == 0
     for i in check:
         run.assert_close(i)
+    scalars = run.opt.debug_scalars()
     for i in range(len(wl.shapes)):
         l_gpu = run.host(run.l[i])
         r_gpu = run.host(run.r[i])
         assert np.max(np.abs(l_gpu - sq_rows[i]) / sq_rows[i]) < 1e-5, i
         assert np.max(np.abs(r_gpu - sq_cols[i]) / sq_cols[i]) < 1e-5, i
-        assert np.all(np.isfinite(run.host(run.W[i])))
+        W = run.host(run.W[i])
+        assert np.all(np.isfinite(W))
+        O = run.host(run.opt.direction(i))
+        Lg, Rg = (run.host(t) for t in run.opt.precond(i))
+        D = Lg[:, None] * O * Rg[None, :]
+        nO, nD = np.linalg.norm(O), np.linalg.norm(D)
+        sc = scalars[i]
+        assert abs(sc[0] - nO) / nO < 1e-4 and abs(sc[1] - nD) / nD < 1e-4, (i, sc[:2], nO, nD)
+        dW = float(sc[6]) * D
+        W_pre = run.decay_gpu * w_prev[i].to(torch.float64).numpy() - dW
+        e = bf16_rounding(W, W_pre, W_pre, 2.0 ** -21 * (np.abs(W_pre) + np.abs(dW)), dW)
+        assert e["own_mismatch"] == 0, (i, e)
     run.close()
 
 
