@@ -1,7 +1,7 @@
 """A CPU model of the Newton-Schulz arithmetic the GPU path is required to use
 (test infrastructure).
 
-The benchmark spec fixes bf16 Newton-Schulz operands with fp32 accumulation.  On
+The GPU path computes Newton-Schulz with bf16 operands and fp32 accumulation.  On
 most inputs that arithmetic lands well inside the 2e-2 direction bar; on a
 few (a thin matrix with three singular values, the very ill-conditioned steps
 of the toy quadratic) the arithmetic itself reaches or passes it, whatever
