@@ -61,7 +61,9 @@ extern "C" {
 #define MALT_ERR_MISALIGNED      -3  /* a device pointer is not 16-byte aligned */
 #define MALT_ERR_SHAPE_CHANGED   -4  /* step called with shapes/dtypes other than at init */
 #define MALT_ERR_CUDA            -5  /* a CUDA runtime call failed (see malt_status_string) */
-#define MALT_ERR_TIMEOUT         -6  /* a device-side wait ran out of its time budget */
+#define MALT_ERR_TIMEOUT         -6  /* a device-side wait ran out of its time budget
+                                        (1 s plus 66 ns per column of the launch's
+                                        longest Newton-Schulz reduction) */
 #define MALT_ERR_OUT_OF_MEMORY   -7  /* workspace allocation failed at init */
 
 /* ---- element types ----------------------------------------------------- */

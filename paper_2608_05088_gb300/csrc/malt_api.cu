@@ -33,7 +33,13 @@ using namespace malt;
 
 namespace {
 
-constexpr uint64_t kWaitBudgetNs = 1000000000ull;  // 1 s per device-side wait
+// Time budget of every device-side wait: 1 s, plus the time one 256 x 256
+// output tile of the launch's longest reduction could take at a tenth of a
+// CTA pair's share of the bf16 peak (2 x 256 x 256 flops per unit of K at
+// 2 TFLOP/s), so that the budget still flags a hang, never an elongated
+// matrix whose Gram product reduces over hundreds of millions of columns.
+constexpr uint64_t kWaitBudgetNs = 1000000000ull;
+constexpr uint64_t kWaitNsPerK = 66;
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
@@ -598,7 +604,9 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         P.status = st->d_status;
         P.queue = st->d_sched + gi;
         P.done = st->d_sched + st->sched_groups_pad;
-        P.budget_ns = kWaitBudgetNs;
+        uint64_t kmax = 0;                // the Gram's K = q is the longest reduction
+        for (int j = 0; j < P.nclasses; ++j) kmax = std::max<uint64_t>(kmax, P.cls[j].q);
+        P.budget_ns = kWaitBudgetNs + kmax * kWaitNsPerK;
     }
 
     // Upload the static tables (init is allowed to synchronise).

@@ -39,6 +39,19 @@ __device__ __forceinline__ float warp_sum(float v) {
 
 // Sum of v over the first nthreads threads (a multiple of 32) in a fixed
 // order; every thread of the block calls it, the result is valid in tid 0.
+// Compensated (Kahan) summation in fp32: the error of the total stays near
+// one rounding however many terms are added (no reassociation: the library
+// is compiled without fast-math).
+struct CompensatedSum {
+    float s = 0.f, c = 0.f;
+    __device__ __forceinline__ void add(float x) {
+        const float y = x - c;
+        const float t = s + y;
+        c = (t - s) - y;
+        s = t;
+    }
+};
+
 __device__ __forceinline__ float block_sum(float v, float* sh /* >= 32 */, int tid, int nthreads) {
     v = warp_sum(v);
     const int w = tid >> 5, lane = tid & 31;
@@ -195,6 +208,9 @@ __device__ __forceinline__ void stats_block(const MatDesc& d, const UserPtrs& up
 // --------------------------------------------------------------- finalize
 // Entry `local` of the matrix's m + n statistics: row i = local (< m) or
 // column j = local - m.  identity (Muon): L = R = 1, statistics untouched.
+// The per-block partial sums are added with compensation: a row of a matrix
+// near the size limit has 8192 of them (a column up to 262144), which a plain
+// fp32 sum in sequence would carry to a relative error near 1e-5.
 __device__ __forceinline__ void finalize_entry(const MatDesc& d, const UserPtrs& up, int local,
                                                float mu2, float eps, int identity) {
     constexpr int P = kLdPlain;
@@ -204,16 +220,16 @@ __device__ __forceinline__ void finalize_entry(const MatDesc& d, const UserPtrs&
     }
     if (local < d.m) {
         const int i = local;
-        float s = 0.f;
-        for (int cb = 0; cb < d.stat_cb; ++cb) s += ld_f<P>(d.rowpart + static_cast<size_t>(cb) * d.m + i);
-        const float l = fmaf(mu2, up.l[i], (1.f - mu2) * s);
+        CompensatedSum s;
+        for (int cb = 0; cb < d.stat_cb; ++cb) s.add(ld_f<P>(d.rowpart + static_cast<size_t>(cb) * d.m + i));
+        const float l = fmaf(mu2, up.l[i], (1.f - mu2) * s.s);
         up.l[i] = l;
         d.L[i] = powf(l + eps, -0.125f);
     } else {
         const int j = local - d.m;
-        float s = 0.f;
-        for (int rb = 0; rb < d.stat_rb; ++rb) s += ld_f<P>(d.colpart + static_cast<size_t>(rb) * d.n + j);
-        const float r = fmaf(mu2, up.r[j], (1.f - mu2) * s);
+        CompensatedSum s;
+        for (int rb = 0; rb < d.stat_rb; ++rb) s.add(ld_f<P>(d.colpart + static_cast<size_t>(rb) * d.n + j));
+        const float r = fmaf(mu2, up.r[j], (1.f - mu2) * s.s);
         up.r[j] = r;
         d.R[j] = powf(r + eps, -0.125f);
     }
@@ -416,13 +432,15 @@ __device__ __forceinline__ void norms_matrix(const MatDesc& d, MatScalars* sc, f
                                              int malter, int tid, float* red) {
     constexpr int P = kLdPlain;
     const int tiles = d.pre_tr * d.pre_tc;
-    float a = 0.f, b = 0.f;
+    // each thread's share of the block partials with compensation (512 of
+    // them per thread for a matrix near the size limit), then one fp32 tree
+    CompensatedSum as, bs;
     for (int i = tid; i < tiles; i += kThreads) {
-        a += ld_f<P>(d.prepart + 2 * i);
-        b += ld_f<P>(d.prepart + 2 * i + 1);
+        as.add(ld_f<P>(d.prepart + 2 * i));
+        bs.add(ld_f<P>(d.prepart + 2 * i + 1));
     }
-    a = block_sum(a, red, tid, kThreads);
-    b = block_sum(b, red, tid, kThreads);
+    const float a = block_sum(as.s, red, tid, kThreads);
+    const float b = block_sum(bs.s, red, tid, kThreads);
     if (tid == 0) {
         const float nrm = sqrtf(a);
         sc->norm_mt = nrm;
@@ -441,16 +459,18 @@ __device__ __forceinline__ void scalars_matrix(const MatDesc& d, MatScalars* sc,
                                                const long long* tcount, const StepHyper& hp,
                                                int tid, float* red) {
     constexpr int P = kLdPlain;
-    float a = 0.f, b = 0.f;
-    // One partial per epilogue warp per GEMM tile of the last iteration.
+    CompensatedSum as, bs;
+    // One partial per epilogue warp per GEMM tile of the last iteration, each
+    // thread's share added with compensation (thousands per thread near the
+    // size limit).
     if (tid < kScalarThreads) {
         for (int i = tid; i < kNsPartsPerTile * d.ns_tiles; i += kScalarThreads) {
-            a += ld_f<P>(d.nspart + 2 * i);
-            b += ld_f<P>(d.nspart + 2 * i + 1);
+            as.add(ld_f<P>(d.nspart + 2 * i));
+            bs.add(ld_f<P>(d.nspart + 2 * i + 1));
         }
     }
-    a = block_sum(a, red, tid, kScalarThreads);
-    b = block_sum(b, red, tid, kScalarThreads);
+    const float a = block_sum(as.s, red, tid, kScalarThreads);
+    const float b = block_sum(bs.s, red, tid, kScalarThreads);
     if (tid == 0) {
         MatScalars s;
         {
