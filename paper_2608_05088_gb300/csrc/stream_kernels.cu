@@ -89,8 +89,11 @@ __global__ void __launch_bounds__(256) pad_kernel(const __grid_constant__ PadPar
 }
 
 // ------------------------------------------------------------------ stats
+// The streaming kernels' minimum resident blocks per SM (statistics 3,
+// prescale 4, apply 8) trade registers for resident warps: more warps per SM
+// kept more of HBM busy than more loads in flight per thread did.
 template <bool kStats>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(256, 3)
 stats_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
              const int32_t* __restrict__ pref, int nmat, float mu1) {
     __shared__ __align__(16) float colsh[8 * kStatCols];
@@ -112,7 +115,7 @@ finalize_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ p
 }
 
 // --------------------------------------------------------------- prescale
-__global__ void __launch_bounds__(256, 3)
+__global__ void __launch_bounds__(256, 4)
 prescale_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
                 const int32_t* __restrict__ pref, int nmat, int malter) {
     __shared__ __align__(16) float tile[blk::kPreTileFloats];
@@ -141,7 +144,7 @@ scalars_kernel(const MatDesc* __restrict__ mats, MatScalars* __restrict__ scal,
 }
 
 // ------------------------------------------------------------------ apply
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(256, 8)
 apply_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
              const MatScalars* __restrict__ scal, const int32_t* __restrict__ pref, int nmat,
              float decay) {
