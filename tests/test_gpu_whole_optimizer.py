@@ -130,7 +130,7 @@ class AdamRun:
 
 def test_adamw_against_oracle_ragged_sizes():
     """Tensors of every size class: sizes not a multiple of 4 (scalar tail),
-    one element, runs over several 8192-element blocks, 2-D embeddings; with
+    one element, runs over several 4096-element blocks, 2-D embeddings; with
     and without decay; 4 steps, every element checked."""
     shapes = [(1,), (3,), (7,), (768,), (2304,), (8195,), (40000,), (97, 131), (1024, 768)]
     wds = [0.0, 0.1, 0.0, 0.0, 0.1, 0.0, 0.1, 0.1, 0.1]
