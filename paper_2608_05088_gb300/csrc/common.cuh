@@ -15,11 +15,11 @@ namespace malt {
 // Statistics kernel tile (rows x cols of W per block).
 constexpr int kStatRows = 64;
 constexpr int kStatCols = 256;
-// Prescale block (rows x cols of Mt); the apply pass of a tall matrix uses
-// the same block shape.
+// Prescale block (rows x cols of Mt).
 constexpr int kPreRows = 64;
 constexpr int kPreCols = 256;
-// Apply kernel (wide matrices): contiguous elements per block.
+// Apply kernel: contiguous elements per block (O is stored in W's layout, so
+// wide and tall matrices stream alike).
 constexpr int kApplyElems = 16384;
 // Newton-Schulz GEMM: a CTA pair computes a kTileM x kBN output tile; each CTA
 // owns kBM rows of it, loads kBM rows of A and kBN/2 rows (N) of B per kBK
