@@ -338,7 +338,7 @@ def run_reference(args):
               f"state), after one warm-up step of 4 matrices")
     out = {"metric": METRIC, "value": value, "unit": UNIT, "impl": "reference",
            "n_gpus": world, "steps": 1, "warmup": 1,
-           "requested": {"steps": args.steps, "warmup": args.warmup},
+           "requested": getattr(args, "requested", {"steps": args.steps, "warmup": args.warmup}),
            "ms_per_step": t_step * 1e3, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": dict(workload_config(wl), ns_schedule=args.ns_schedule),
@@ -861,6 +861,7 @@ def main():
     ap.add_argument("--stress-k", type=int, default=None,
                     help="stress sweep: only this Newton-Schulz iteration count")
     args = ap.parse_args()
+    args.requested = {"steps": args.steps, "warmup": args.warmup}
     if args.warmup < 3:
         args.warmup = 3
     if args.compare_cublas:
