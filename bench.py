@@ -694,22 +694,38 @@ def run_malt(args):
 
     # ---- the same engine as Muon (identity preconditioners, no statistics):
     # the optimizer-only counterpart of the paper's MALT-vs-Muon overhead table.
+    # Muon and MALT run in alternating blocks of steps on the same state, so
+    # that both see the same clocks under the power cap.
     muon = None
     if not args.no_muon:
         for _ in range(2):
             opt.step(hp, muon=True)
         torch.cuda.synchronize()
         barrier()
-        m0 = torch.cuda.Event(enable_timing=True)
-        m1 = torch.cuda.Event(enable_timing=True)
-        m0.record(stream)
-        for _ in range(args.steps):
-            opt.step(hp, muon=True)
-        m1.record(stream)
-        torch.cuda.synchronize()
-        tm = max_over_ranks(m0.elapsed_time(m1), dev) / args.steps
-        muon = {"ms_per_step": tm, "malt_ms_per_step": t_ms / args.steps,
-                "malt_overhead_vs_muon": (t_ms / args.steps) / tm - 1.0}
+        block = max(1, args.steps // 2)
+        t_muon = t_malt = 0.0
+        for _ in range(4):
+            for is_muon in (True, False):
+                m0 = torch.cuda.Event(enable_timing=True)
+                m1 = torch.cuda.Event(enable_timing=True)
+                m0.record(stream)
+                for _ in range(block):
+                    if is_muon:
+                        opt.step(hp, muon=True)
+                    else:
+                        opt.step(hp, malter=malter)
+                m1.record(stream)
+                torch.cuda.synchronize()
+                if is_muon:
+                    t_muon += m0.elapsed_time(m1)
+                else:
+                    t_malt += m0.elapsed_time(m1)
+        tm = max_over_ranks(t_muon, dev) / (4 * block)
+        tmalt = max_over_ranks(t_malt, dev) / (4 * block)
+        muon = {"ms_per_step": tm, "malt_ms_per_step": tmalt,
+                "malt_overhead_vs_muon": tmalt / tm - 1.0,
+                "method": f"4 alternating blocks of {block} Muon and {block} "
+                          f"{'MALTER' if malter else 'MALT'} steps on one state"}
         if opt.check() != malt.MALT_OK:
             raise SystemExit("muon step failed")
 
