@@ -237,8 +237,9 @@ __device__ __forceinline__ void finalize_entry(const MatDesc& d, const UserPtrs&
 
 // --------------------------------------------------------------- prescale
 // Block `local` = kPreRows x kPreCols of Mt.  A wide matrix is streamed like
-// the statistics pass (warp w owns 8 rows, lane 8 consecutive columns, four
-// rows of loads in flight) and written as bf16 in place of its NS frame; a
+// the statistics pass (warp w owns 8 rows, lane 8 consecutive columns,
+// kPreBatch rows of loads in flight) and written as bf16 in place of its NS
+// frame; a
 // tall matrix's NS frame is Mt^T, so its block walks four 64 x 64 sub-tiles
 // through shared memory and writes each transposed.
 // tile: two 64 x 64 float buffers (kPreTileFloats, 16-byte aligned), used in
@@ -247,6 +248,13 @@ __device__ __forceinline__ void finalize_entry(const MatDesc& d, const UserPtrs&
 // reads (eight rows 8 apart per warp) hit 32 distinct banks.
 // red: 8 float2.
 constexpr int kPreTileFloats = 2 * 64 * 64;
+// Loads in flight per thread: rows of a wide block loaded together, and
+// sub-tiles of a tall block loaded ahead.  Small, so that the kernel fits 4
+// blocks per SM in 64 registers without spilling: resident warps keep more of
+// HBM busy than loads in flight per thread (4 and 2 spilled at 4 blocks per SM
+// and streamed 7 % slower on GPT-2 Large, 14 % on a 16384 x 4096 matrix).
+constexpr int kPreBatch = 2;
+constexpr int kPreAhead = 1;
 __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs& up, int local,
                                                int malter, int tid, float* tile,
                                                float2* red) {
@@ -276,11 +284,11 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
         }
         const int row0 = r0 + warp * 8;
 #pragma unroll
-        for (int rb = 0; rb < 8; rb += 4) {
-            float mv[4][8], li[4];
-            bool ok[4];
+        for (int rb = 0; rb < 8; rb += kPreBatch) {
+            float mv[kPreBatch][8], li[kPreBatch];
+            bool ok[kPreBatch];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
+            for (int u = 0; u < kPreBatch; ++u) {
                 const int row = row0 + rb + u;
                 ok[u] = colok && row < m;
                 li[u] = 0.f;
@@ -294,7 +302,7 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
                 }
             }
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
+            for (int u = 0; u < kPreBatch; ++u) {
                 if (!ok[u]) continue;
                 const int row = row0 + rb + u;
                 const size_t off = static_cast<size_t>(row) * n + col;
@@ -319,7 +327,7 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
     } else {
         // Keep the M loads of the next sub-tile in flight while this one goes
         // through shared memory: each 64 x 64 sub-tile is four rows of one
-        // float4 per thread, loaded two sub-tiles ahead.
+        // float4 per thread, loaded kPreAhead sub-tiles ahead.
         const int cc = (t & 15) * 4;
         constexpr int kSubs = kPreCols / 64;
         float li[4];
@@ -338,9 +346,9 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
                                 : make_float4(0.f, 0.f, 0.f, 0.f);
             }
         };
-        float4 mq[2][4];
-        load_sub(0, mq[0]);
-        load_sub(1, mq[1]);
+        float4 mq[kPreAhead][4];
+#pragma unroll
+        for (int a = 0; a < kPreAhead; ++a) load_sub(a, mq[a]);
 #pragma unroll
         for (int sub = 0; sub < kSubs; ++sub) {
             const int cs = c0 + sub * 64;
@@ -357,7 +365,7 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
                 if (row < m && col < n) {
                     const size_t off = static_cast<size_t>(row) * n + col;
                     const float Li = li[pass];
-                    const float4 q = mq[sub & 1][pass];
+                    const float4 q = mq[sub % kPreAhead][pass];
                     v0 = Li * q.x * R4.x; v1 = Li * q.y * R4.y;
                     v2 = Li * q.z * R4.z; v3 = Li * q.w * R4.w;
                     // explicit fused multiply-adds: the same rounding wherever
@@ -384,7 +392,7 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
                 *reinterpret_cast<float4*>(tb + rr * 64 + (((t & 15) ^ ((rr >> 3) & 7)) << 2)) =
                     make_float4(v0, v1, v2, v3);
             }
-            if (sub + 2 < kSubs) load_sub(sub + 2, mq[sub & 1]);
+            if (sub + kPreAhead < kSubs) load_sub(sub + kPreAhead, mq[sub % kPreAhead]);
             // One barrier per sub-tile: the buffer written next was last read
             // two sub-tiles ago, before every thread passed the previous barrier.
             __syncthreads();
