@@ -44,8 +44,12 @@ cudaError_t launch_stats(const MatDesc* mats, const UserPtrs* ptrs, const int32_
 cudaError_t launch_finalize(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* pref,
                             int nmat, int32_t total, float mu2, float eps, long long* tcount,
                             int identity, cudaStream_t s);
-cudaError_t launch_prescale(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* pref,
-                            int nmat, int32_t blocks, int malter, cudaStream_t s);
+// Prescale: `wide` wide matrices (ids[0 .. wide), wide_blocks blocks) in one
+// launch, then `tall` tall ones (ids[wide ..), tall_blocks blocks) in another;
+// pref is the block prefix over ids.
+cudaError_t launch_prescale(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* ids,
+                            const int32_t* pref, int wide, int32_t wide_blocks, int tall,
+                            int32_t tall_blocks, int malter, cudaStream_t s);
 cudaError_t launch_norms(const MatDesc* mats, MatScalars* scal, int nmat, float ns_eps,
                          int malter, cudaStream_t s);
 cudaError_t launch_scalars(const MatDesc* mats, MatScalars* scal, const long long* tcount,

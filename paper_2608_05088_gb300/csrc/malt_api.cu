@@ -153,6 +153,11 @@ struct malt_state {
     int32_t* d_status = nullptr;
     int32_t* d_pref[4] = {nullptr, nullptr, nullptr, nullptr};  // stats, fin, pre, apply
     int32_t blocks_stats = 0, total_fin = 0, blocks_pre = 0, blocks_apply = 0;
+    // The prescale pass runs wide and tall matrices in two launches (their
+    // blocks differ): d_pre_ids lists the wide matrices, then the tall ones,
+    // and d_pref[2] is the block prefix in that order.
+    int32_t* d_pre_ids = nullptr;
+    int32_t pre_wide = 0, blocks_pre_wide = 0;
     // Newton-Schulz work lists, one per group of up to kMaxClasses classes,
     // and the persistent schedule's counters: [groups_pad] claim counters,
     // then [3 * kMaxNsSteps][nmat] finished-tile signals.
@@ -469,6 +474,7 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
     const size_t o_status = cv.take(sizeof(int32_t) * kStatusWords);
     size_t o_pref[4];
     for (int j = 0; j < 4; ++j) o_pref[j] = cv.take(sizeof(int32_t) * (n + 1));
+    const size_t o_pre_ids = cv.take(sizeof(int32_t) * std::max(n, 1));
     const int ngroups = (nc + kMaxClasses - 1) / kMaxClasses;
     st->sched_groups_pad = ((ngroups + 63) / 64) * 64;
     const size_t o_sched = cv.take(sizeof(uint32_t) * (st->sched_groups_pad +
@@ -547,6 +553,7 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
     st->d_t = reinterpret_cast<long long*>(base + o_t);
     st->d_status = reinterpret_cast<int32_t*>(base + o_status);
     for (int j = 0; j < 4; ++j) st->d_pref[j] = reinterpret_cast<int32_t*>(base + o_pref[j]);
+    st->d_pre_ids = reinterpret_cast<int32_t*>(base + o_pre_ids);
     st->d_sched = reinterpret_cast<uint32_t*>(base + o_sched);
     for (size_t gi = 0; gi < tables.size(); ++gi)
         st->table_dev.push_back(reinterpret_cast<NsEntry*>(base + o_table[gi]));
@@ -562,17 +569,24 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
     // Block-prefix tables.
     std::vector<int32_t> pref[4];
     for (int j = 0; j < 4; ++j) pref[j].assign(n + 1, 0);
+    std::vector<int32_t> pre_ids;
+    for (int tall = 0; tall < 2; ++tall)
+        for (int i = 0; i < n; ++i)
+            if (st->hmats[i].trans == tall) pre_ids.push_back(i);
     for (int i = 0; i < n; ++i) {
         const MatDesc& d = st->hmats[i];
         pref[0][i + 1] = pref[0][i] + d.stat_rb * d.stat_cb;
         pref[1][i + 1] = pref[1][i] + d.m + d.n;
-        pref[2][i + 1] = pref[2][i] + d.pre_tr * d.pre_tc;
+        const MatDesc& e = st->hmats[pre_ids[i]];        // prescale order: wide, then tall
+        pref[2][i + 1] = pref[2][i] + e.pre_tr * e.pre_tc;
+        if (e.trans == 0) st->pre_wide = i + 1;
         // apply: contiguous runs of kApplyElems (O is in W's layout)
         pref[3][i + 1] = pref[3][i] + mat_apply_blocks(d);
     }
     st->blocks_stats = pref[0][n];
     st->total_fin = pref[1][n];
     st->blocks_pre = pref[2][n];
+    st->blocks_pre_wide = pref[2][st->pre_wide];
     st->blocks_apply = pref[3][n];
 
     // Tensor maps of every class buffer.
@@ -628,6 +642,8 @@ int plan_and_allocate(malt_state* st, const malt_param_t* params, int n) {
         for (int j = 0; j < 4; ++j)
             MALT_CUDA(cudaMemcpy(st->d_pref[j], pref[j].data(), sizeof(int32_t) * (n + 1),
                                  cudaMemcpyHostToDevice), "cudaMemcpy(prefix)");
+        MALT_CUDA(cudaMemcpy(st->d_pre_ids, pre_ids.data(), sizeof(int32_t) * n,
+                             cudaMemcpyHostToDevice), "cudaMemcpy(prescale order)");
         for (int k = 0; k < nc; ++k) {
             const ShapeClass& C = st->classes[k];
             MALT_CUDA(cudaMemcpy(C.d_mat_of, C.mats.data(), sizeof(int32_t) * C.batch,
@@ -830,9 +846,11 @@ int run_step(malt_state* st, const malt_param_t* params, int32_t n, const malt_h
                                   hp->mu2, hp->eps, st->d_t, muon, s), "finalize_kernel");
     }
     {
-        LaunchScope ls(st, MALT_KIND_PRESCALE, s);
-        MALT_CUDA(launch_prescale(st->d_mats, st->d_ptrs, st->d_pref[2], nm, st->blocks_pre,
-                                  malter, s), "prescale_kernel");
+        const int wide = st->pre_wide, tall = nm - st->pre_wide;
+        LaunchScope ls(st, MALT_KIND_PRESCALE, s, (wide > 0) + (tall > 0));
+        MALT_CUDA(launch_prescale(st->d_mats, st->d_ptrs, st->d_pre_ids, st->d_pref[2], wide,
+                                  st->blocks_pre_wide, tall, st->blocks_pre - st->blocks_pre_wide,
+                                  malter, s), "prescale kernels");
     }
     if (hooks != nullptr)   // stats and prescale are the only readers of G
         MALT_CUDA(cudaEventRecord(hooks->record_g_consumed, s), "cudaEventRecord(G consumed)");

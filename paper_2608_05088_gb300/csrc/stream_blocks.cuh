@@ -249,12 +249,16 @@ __device__ __forceinline__ void finalize_entry(const MatDesc& d, const UserPtrs&
 // red: 8 float2.
 constexpr int kPreTileFloats = 2 * 64 * 64;
 // Loads in flight per thread: rows of a wide block loaded together, and
-// sub-tiles of a tall block loaded ahead.  Small, so that the kernel fits 4
-// blocks per SM in 64 registers without spilling: resident warps keep more of
-// HBM busy than loads in flight per thread (4 and 2 spilled at 4 blocks per SM
-// and streamed 7 % slower on GPT-2 Large, 14 % on a 16384 x 4096 matrix).
+// sub-tiles of a tall block loaded ahead.  Small, so that the wide blocks fit
+// 5 per SM in 48 registers and the tall ones 4 per SM in 64 registers without
+// spilling: resident warps keep more of HBM busy than loads in flight per
+// thread (four rows and two sub-tiles spilled at 4 blocks per SM and streamed
+// 7 % slower on GPT-2 Large, 14 % on a 16384 x 4096 matrix; one row at 6
+// blocks per SM was 2 % slower on GPT-2 Large and 5-10 % on wide stress
+// matrices).
 constexpr int kPreBatch = 2;
 constexpr int kPreAhead = 1;
+template <bool kTall>
 __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs& up, int local,
                                                int malter, int tid, float* tile,
                                                float2* red) {
@@ -262,8 +266,8 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
     const int m = d.m, n = d.n;
     // A tall matrix's blocks walk down a column band first, so the blocks
     // resident at once write neighbouring pieces of the same X0 rows.
-    const int tr = d.trans ? local % d.pre_tr : local / d.pre_tc;
-    const int tc = d.trans ? local / d.pre_tr : local - tr * d.pre_tc;
+    const int tr = kTall ? local % d.pre_tr : local / d.pre_tc;
+    const int tc = kTall ? local / d.pre_tr : local - tr * d.pre_tc;
     const int r0 = tr * kPreRows, c0 = tc * kPreCols;
     const int t = tid, warp = t >> 5, lane = t & 31;
     const float* __restrict__ Lv = d.L;
@@ -272,7 +276,7 @@ __device__ __forceinline__ void prescale_block(const MatDesc& d, const UserPtrs&
     const bool gbf = d.g_bf16 != 0;
     float s_mt = 0.f, s_lgr = 0.f;
 
-    if (!d.trans) {
+    if constexpr (!kTall) {
         const int col = c0 + lane * 8;
         const bool colok = col < n;
         float rj[8];

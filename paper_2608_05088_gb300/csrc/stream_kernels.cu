@@ -90,8 +90,9 @@ __global__ void __launch_bounds__(256) pad_kernel(const __grid_constant__ PadPar
 
 // ------------------------------------------------------------------ stats
 // The streaming kernels' minimum resident blocks per SM (statistics 3,
-// prescale 4, apply 8) trade registers for resident warps: more warps per SM
-// kept more of HBM busy than more loads in flight per thread did.
+// prescale 5 for wide matrices and 4 for tall ones, apply 8) trade registers
+// for resident warps: more warps per SM kept more of HBM busy than more loads
+// in flight per thread did.
 template <bool kStats>
 __global__ void __launch_bounds__(256, 3)
 stats_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
@@ -115,14 +116,32 @@ finalize_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ p
 }
 
 // --------------------------------------------------------------- prescale
+// One launch for the wide matrices, one for the tall ones (their NS frame is
+// Mt^T, written through shared-memory transposes): ids lists the launch's
+// matrices and pref its block prefix.
+__global__ void __launch_bounds__(256, 5)
+prescale_wide_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
+                     const int32_t* __restrict__ ids, const int32_t* __restrict__ pref, int count,
+                     int malter) {
+    __shared__ float2 red[8];
+    const int32_t x = blockIdx.x;
+    const int k = find_mat(pref, count, x);
+    const int g = __ldg(ids + k);
+    blk::prescale_block<false>(mats[g], ptrs[g], x - __ldg(pref + k), malter, threadIdx.x, nullptr,
+                               red);
+}
+
 __global__ void __launch_bounds__(256, 4)
-prescale_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
-                const int32_t* __restrict__ pref, int nmat, int malter) {
+prescale_tall_kernel(const MatDesc* __restrict__ mats, const UserPtrs* __restrict__ ptrs,
+                     const int32_t* __restrict__ ids, const int32_t* __restrict__ pref, int count,
+                     int32_t base, int malter) {
     __shared__ __align__(16) float tile[blk::kPreTileFloats];
     __shared__ float2 red[8];
-    const int g = find_mat(pref, nmat, blockIdx.x);
-    blk::prescale_block(mats[g], ptrs[g], blockIdx.x - __ldg(pref + g), malter, threadIdx.x, tile,
-                        red);
+    const int32_t x = base + static_cast<int32_t>(blockIdx.x);   // pref continues the wide launch's
+    const int k = find_mat(pref, count, x);
+    const int g = __ldg(ids + k);
+    blk::prescale_block<true>(mats[g], ptrs[g], x - __ldg(pref + k), malter, threadIdx.x, tile,
+                              red);
 }
 
 // ------------------------------------------------------------------ norms
@@ -220,10 +239,20 @@ cudaError_t launch_finalize(const MatDesc* mats, const UserPtrs* ptrs, const int
     return cudaGetLastError();
 }
 
-cudaError_t launch_prescale(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* pref,
-                            int nmat, int32_t blocks, int malter, cudaStream_t s) {
-    prescale_kernel<<<blocks, 256, 0, s>>>(mats, ptrs, pref, nmat, malter);
-    return cudaGetLastError();
+cudaError_t launch_prescale(const MatDesc* mats, const UserPtrs* ptrs, const int32_t* ids,
+                            const int32_t* pref, int wide, int32_t wide_blocks, int tall,
+                            int32_t tall_blocks, int malter, cudaStream_t s) {
+    if (wide > 0 && wide_blocks > 0) {
+        prescale_wide_kernel<<<wide_blocks, 256, 0, s>>>(mats, ptrs, ids, pref, wide, malter);
+        const cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    if (tall > 0 && tall_blocks > 0) {
+        prescale_tall_kernel<<<tall_blocks, 256, 0, s>>>(mats, ptrs, ids + wide, pref + wide, tall,
+                                                         wide_blocks, malter);
+        return cudaGetLastError();
+    }
+    return cudaSuccess;
 }
 
 cudaError_t launch_norms(const MatDesc* mats, MatScalars* scal, int nmat, float ns_eps,
