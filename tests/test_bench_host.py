@@ -39,7 +39,7 @@ def test_max_over_ranks_gloo_two_ranks():
 
 def test_reference_arm_prints_contract_line():
     out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
-                          "--workload", "single_256x512", "--steps", "2", "--warmup", "3"],
+                          "--workload", "single_256x512", "--steps", "2", "--warmup", "1"],
                          capture_output=True, text=True, timeout=600, cwd=ROOT)
     assert out.returncode == 0, out.stderr
     line = json.loads(out.stdout.strip().splitlines()[-1])
@@ -50,7 +50,7 @@ def test_reference_arm_prints_contract_line():
     assert line["cpu_baseline"]["kind"] == "oracle"
     assert line["e2e"]["h2d_bytes_per_step"] == 0
     # one real step over the whole parameter set, reported as what ran
-    assert line["steps"] == 1 and line["requested"] == {"steps": 2, "warmup": 3}
+    assert line["steps"] == 1 and line["requested"] == {"steps": 2, "warmup": 1}
     assert abs(line["ms_per_step"] * line["value"] - 1e3) < 1e-6 * 1e3
     # the same config keys as the GPU arm's line
     sys.path.insert(0, ROOT)
