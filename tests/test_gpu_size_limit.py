@@ -1,8 +1,9 @@
 """Matrices at the C ABI's size limit: rows x cols just under 2^31 elements.
 
 Two elongated shapes, 1024 x 2097144 and its transpose (2^31 - 8192
-elements each), one MALT step each with bf16 W and fp32 state.  Element
-offsets reach 2^31 - 8, byte offsets of the fp32 buffers 2^33; the Gram
+elements each), one MALT step each with bf16 W and fp32 state, and one
+MALTER step of the tall one (its prescale also re-reads G for ||L G R||).
+Element offsets reach 2^31 - 8, byte offsets of the fp32 buffers 2^33; the Gram
 product reduces over 2,097,144 columns; the tall matrix runs every
 transposed path (prescale through shared memory, O stored in W's layout).
 The fp64 oracle would take hours at this size, so the step is checked
@@ -19,6 +20,9 @@ step's inputs and its own intermediates:
   within 1e-4 of fp64 norms of the step's O, L, R;
 * Newton-Schulz output: finite, with mean squared singular value
   ||O||_F^2 / min(rows, cols) inside the band of the quintic;
+* MALTER: ||L G R||^2 within 1e-4 of the fp64 sum over the step's L, R and
+  G, nu = (1 - mu2) ||L G R||^2 and alpha = 1 at t = 1 (Algorithm 2, nu_t
+  and alpha_t lines);
 * update: on sampled rows (the first, the last and random ones) the stored
   bf16 W is the round-to-nearest-even of W_prev - s L O R, s the step's
   scale, wherever no rounding boundary lies within the kernel's fp32 slack
@@ -41,8 +45,9 @@ def _row_chunks(rows, cols):
         yield r0, min(rows, r0 + step)
 
 
-@pytest.mark.parametrize("rows,cols", LIMIT_SHAPES)
-def test_size_limit(rows, cols):
+@pytest.mark.parametrize("rows,cols,malter", [(r, c, False) for r, c in LIMIT_SHAPES] +
+                         [(LIMIT_SHAPES[1][0], LIMIT_SHAPES[1][1], True)])
+def test_size_limit(rows, cols, malter):
     import torch
     import paper_2608_05088_gb300.malt as malt
     assert rows * cols < 2 ** 31 and rows * cols > 2 ** 31 - 2 ** 14
@@ -60,7 +65,7 @@ def test_size_limit(rows, cols):
     W_prev = W.clone()
     opt = malt.MaltOptimizer([(W, G, M, l, r)])
     hp = malt.hparams(lr=0.02)
-    opt.step(hp)
+    opt.step(hp, malter=malter)
     assert opt.check() == malt.MALT_OK
     torch.cuda.synchronize()
 
@@ -88,15 +93,26 @@ def test_size_limit(rows, cols):
     torch.cuda.synchronize()
     so = 0.0
     sd = 0.0
+    slgr = 0.0
     for r0, r1 in _row_chunks(rows, cols):
         o = O[r0:r1].cpu().double()
         assert bool(torch.isfinite(o).all()), (r0, r1)
         d = L[r0:r1, None] * o * R[None, :]
         so += float((o * o).sum())
         sd += float((d * d).sum())
+        if malter:
+            lgr = L[r0:r1, None] * G[r0:r1].cpu().double() * R[None, :]
+            slgr += float((lgr * lgr).sum())
     nO, nD = np.sqrt(so), np.sqrt(sd)
     sc = opt.debug_scalars()[0]
     assert abs(sc[0] - nO) / nO < 1e-4 and abs(sc[1] - nD) / nD < 1e-4, (sc[:2], nO, nD)
+    if malter:
+        # Algorithm 2 at t = 1 from zero state: nu = (1 - mu2) ||L G R||^2, and
+        # alpha = sqrt(1 - mu2) ||Mt|| / ((1 - mu1 + eps)(sqrt(nu) + eps)) with
+        # Mt = (1 - mu1) L G R, i.e. 1 up to eps terms
+        assert abs(sc[3] - slgr) / slgr < 1e-4, (sc[3], slgr)
+        assert abs(sc[4] - (1.0 - float(mu2)) * slgr) / ((1.0 - float(mu2)) * slgr) < 1e-4
+        assert abs(sc[5] - 1.0) < 1e-4, sc[5]
     # 5 quintic iterations leave every normalised singular value of a
     # full-rank input in roughly [0.68, 1.2] (bf16 adds a few percent)
     assert 0.4 < so / min(rows, cols) < 1.5, so / min(rows, cols)
