@@ -6,8 +6,8 @@
 // 3-D TMA descriptor serves the whole class, and every grouped element-wise
 // launch gets a block-prefix table.  A step then enqueues, on the caller's
 // stream and without any host synchronisation:
-//   bind (caller pointers) -> stats -> finalize -> prescale -> norms
-//   -> Newton-Schulz -> scalars -> apply,
+//   bind (caller pointers) -> stats -> finalize -> prescale (wide matrices,
+//   then tall ones) -> norms -> Newton-Schulz -> scalars -> apply,
 // where Newton-Schulz runs, per group of up to kMaxClasses classes, either as
 // one persistent launch over all k x (Gram, Poly, BX) products or as one
 // launch per product (the phased schedule); by default a group whose Gram

@@ -37,8 +37,6 @@ __device__ __forceinline__ float warp_sum(float v) {
     return v;
 }
 
-// Sum of v over the first nthreads threads (a multiple of 32) in a fixed
-// order; every thread of the block calls it, the result is valid in tid 0.
 // Compensated (Kahan) summation in fp32: the error of the total stays near
 // one rounding however many terms are added (no reassociation: the library
 // is compiled without fast-math).
@@ -52,6 +50,8 @@ struct CompensatedSum {
     }
 };
 
+// Sum of v over the first nthreads threads (a multiple of 32) in a fixed
+// order; every thread of the block calls it, the result is valid in tid 0.
 __device__ __forceinline__ float block_sum(float v, float* sh /* >= 32 */, int tid, int nthreads) {
     v = warp_sum(v);
     const int w = tid >> 5, lane = tid & 31;
