@@ -835,6 +835,19 @@ def run_malt(args):
         mem[kind] = {"ms_per_step": ms / args.steps, "bytes_per_elem": bytes_per_elem,
                      "achieved_gbs": gbs,
                      "frac_of_hbm": (gbs / float(pk["hbm_gbs"])) if gbs else None}
+    # finalize: per matrix, the per-block partial sums of G^2 (one per 256-column
+    # block for each row, one per 64-row block for each column: the statistics
+    # kernel's tile) in, l and r in and out, L and R out, all fp32
+    fin_bytes = 0.0
+    for m_, n_ in wl.shapes:
+        m8, n8 = -(-m_ // 8) * 8, -(-n_ // 8) * 8
+        fin_bytes += 4.0 * (m8 * -(-n8 // 256) + n8 * -(-m8 // 64)) + 16.0 * (m8 + n8)
+    ms = prof["finalize"][0]
+    gbs = fin_bytes * args.steps / (ms / 1e3) / 1e9 if ms > 0 else None
+    mem["finalize"] = {"ms_per_step": ms / args.steps, "bytes_per_step": fin_bytes,
+                       "achieved_gbs": gbs,
+                       "frac_of_hbm": (gbs / float(pk["hbm_gbs"])) if gbs else None,
+                       "note": "about 0.1 B per element: latency-bound, not bandwidth-bound"}
     breakdown = {k: round(v[0] / args.steps, 4) for k, v in prof.items()}
     launches = sum(v[1] for v in prof.values())
 
